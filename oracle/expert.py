@@ -1,0 +1,219 @@
+"""Oracle: one rolling action-expert step in fp64 (test infrastructure).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg
+may import this module; the CUDA library never does, and nothing here imports
+the library.  Plain numpy, float64 throughout (the appended noise is the
+float32 sequence of ``oracle.noise``).  No blocking, fusion or reordering:
+each function is the definition it cites, in the order the paper states it.
+
+The paper (Sec. 3.1, Eq. 1 and Eq. 3) defines the step as: one forward pass of
+the flow-matching action expert v_theta(A, tau, c, delta_p) over the K-slot
+buffer, a per-slot Euler update by the slot's flow-time step, release of the
+first slot, a shift, and the append of a Gaussian slot.  The expert's
+internals are not printed in the paper; the readings used here are:
+
+* time convention t = 1 - tau (t = 1 pure noise); slot j (0-based, j = 0 is
+  released next) carries t_j, staggered t_j = (j+1)/H;  dt_j = t_j - t_{j-1},
+  t_{-1} = 0 (Eq. 3 uses the uniform 1/K);
+* conditioning (App. A.1, pi0.5): cond = MLP_t(emb(t_j)) + MLP_d(emb(delta_b)),
+  MLP = Linear -> SiLU -> Linear, emb = sinusoidal with periods geometric from
+  4e-3 to 4;
+* adaRMSNorm: x / sqrt(mean(x^2) + 1e-6) * (1 + scale) + shift, with
+  (scale, shift) a slice of mod = cond @ W_mod + b_mod (two norms per layer and
+  one final norm);
+* VLM context (Eq. 2) = a per-layer prefix K/V cache; FOP tokens z (Eq. 4)
+  enter every layer as extra keys/values through that layer's own K/V
+  projection of RMSNorm(z) * (1 + gamma_l);
+* attention: grouped-query, query head h reads KV head h // (Hq/Hkv); keys are
+  [valid prefix | FOP | the H action slots]; full bidirectional mask (a
+  ``slot_isolated`` test mask lets action query j see only action key j);
+  no positional encoding; scale 1/sqrt(hd);
+* MLP: GeGLU with the tanh form of GELU; no biases in QKV / O / MLP.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from .noise import action_noise
+
+EPS = 1e-6
+
+
+def _f64(a):
+    return np.asarray(a, dtype=np.float64)
+
+
+def sinusoidal(x, width: int) -> np.ndarray:
+    """Sinusoidal embedding [N, width] of scalars x [N]: first half sin(x w_i),
+    second half cos(x w_i), w_i = 2 pi / p_i, periods p_i geometric from 4e-3
+    (i = 0) to 4.0 (i = width/2 - 1)."""
+    half = width // 2
+    i = np.arange(half, dtype=np.float64)
+    period = 4e-3 * (4.0 / 4e-3) ** (i / (half - 1))
+    ang = _f64(x)[:, None] * (2.0 * np.pi / period)[None, :]
+    return np.concatenate([np.sin(ang), np.cos(ang)], axis=1)
+
+
+def silu(x):
+    return x / (1.0 + np.exp(-x))
+
+
+def gelu_tanh(x):
+    """0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3))) (Hendrycks & Gimpel)."""
+    return 0.5 * x * (1.0 + np.tanh(np.sqrt(2.0 / np.pi) * (x + 0.044715 * x ** 3)))
+
+
+def rmsnorm(x):
+    """x / sqrt(mean(x^2) + eps) over the last axis."""
+    return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + EPS)
+
+
+def ada_rmsnorm(x, scale, shift):
+    """adaRMSNorm with per-row modulation: rmsnorm(x) * (1 + scale) + shift."""
+    return rmsnorm(x) * (1.0 + scale) + shift
+
+
+def mlp2(e, w1, b1, w2, b2):
+    """Linear -> SiLU -> Linear."""
+    return silu(e @ _f64(w1) + _f64(b1)) @ _f64(w2) + _f64(b2)
+
+
+def conditioning(cfg, W, slot_times, delta):
+    """cond[b, j] = MLP_t(emb(t_j)) + MLP_d(emb(delta_b))  (App. A.1: the offset
+    MLP's embedding is added to the flow-timestep embedding; every slot keeps
+    its own t_j and all slots share delta_b).  Returns [B, H, D]."""
+    D = cfg.width
+    ht = mlp2(sinusoidal(slot_times, D), W["t_w1"], W["t_b1"], W["t_w2"], W["t_b2"])   # [H, D]
+    hd = mlp2(sinusoidal(delta, D), W["d_w1"], W["d_b1"], W["d_w2"], W["d_b2"])        # [B, D]
+    return hd[:, None, :] + ht[None, :, :]
+
+
+def modulation(cfg, W, cond):
+    """mod = cond @ W_mod + b_mod: [B, H, 4 L D + 2 D]."""
+    return cond @ _f64(W["mod_w"]) + _f64(W["mod_b"])
+
+
+def mod_slice(cfg, mod, layer: int, which: int):
+    """(scale, shift) of norm ``which`` (0: before attention, 1: before the MLP)
+    of ``layer``; layer == cfg.layers selects the final norm."""
+    D = cfg.width
+    base = 4 * D * layer + 2 * D * which
+    return mod[..., base:base + D], mod[..., base + D:base + 2 * D]
+
+
+def attention(q, k, v, valid=None):
+    """Softmax attention of one KV head.
+
+    q [Nq, hd], k/v [Nk, hd], valid: optional bool [Nq, Nk] (True = visible).
+    Returns [Nq, hd].  Masked keys are excluded from the softmax."""
+    s = (q @ k.T) / np.sqrt(q.shape[-1])
+    if valid is not None:
+        s = np.where(valid, s, -np.inf)
+    s = s - s.max(axis=-1, keepdims=True)
+    p = np.exp(s)
+    p = p / p.sum(axis=-1, keepdims=True)
+    return p @ v
+
+
+def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta,
+                    mask: str = "full", trace: dict | None = None):
+    """v_theta(A, t, c, delta) for B robots: [B, H, A] float64 (Eq. 3's velocity).
+
+    buffer [B, H, A]; slot_times [H]; ctx_k / ctx_v [L, B, Hkv, >=prefix_len, hd];
+    fop [B, F, D]; delta [B].  ``trace`` (optional dict) receives intermediates.
+    """
+    B, H, A = buffer.shape
+    D, L = cfg.width, cfg.layers
+    Hq, Hkv, hd = cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim
+    G = Hq // Hkv
+    F = fop.shape[1]
+    P = int(prefix_len)
+
+    cond = conditioning(cfg, W, _f64(slot_times), _f64(delta))
+    mod = modulation(cfg, W, cond)
+    x = _f64(buffer) @ _f64(W["in_w"]) + _f64(W["in_b"])         # residual stream [B, H, D]
+    zn = rmsnorm(_f64(fop))                                        # [B, F, D]
+
+    nk = P + F + H
+    valid = np.ones((H, nk), dtype=bool)
+    if mask == "slot_isolated":
+        valid[:, P + F:] = np.eye(H, dtype=bool)
+    elif mask != "full":
+        raise ValueError(mask)
+
+    for l in range(L):
+        wqkv = _f64(W["w_qkv"][l])
+        sc, sh = mod_slice(cfg, mod, l, 0)
+        y = ada_rmsnorm(x, sc, sh)                                  # [B, H, D]
+        yf = zn * (1.0 + _f64(W["fop_gamma"][l]))                  # [B, F, D]
+        qkv = y @ wqkv                                              # [B, H, NQKV]
+        kvf = yf @ wqkv[:, Hq * hd:]                                # [B, F, 2 Hkv hd]
+        q = qkv[..., :Hq * hd].reshape(B, H, Hq, hd)
+        ka = qkv[..., Hq * hd:(Hq + Hkv) * hd].reshape(B, H, Hkv, hd)
+        va = qkv[..., (Hq + Hkv) * hd:].reshape(B, H, Hkv, hd)
+        kf = kvf[..., :Hkv * hd].reshape(B, F, Hkv, hd)
+        vf = kvf[..., Hkv * hd:].reshape(B, F, Hkv, hd)
+        o = np.empty((B, H, Hq, hd))
+        for b in range(B):
+            for g in range(Hkv):
+                keys = np.concatenate([_f64(ctx_k[l, b, g, :P]), kf[b, :, g], ka[b, :, g]])
+                vals = np.concatenate([_f64(ctx_v[l, b, g, :P]), vf[b, :, g], va[b, :, g]])
+                for h in range(g * G, (g + 1) * G):
+                    o[b, :, h] = attention(q[b, :, h], keys, vals, valid)
+        x = x + o.reshape(B, H, Hq * hd) @ _f64(W["w_o"][l])
+        sc2, sh2 = mod_slice(cfg, mod, l, 1)
+        y2 = ada_rmsnorm(x, sc2, sh2)
+        hmid = gelu_tanh(y2 @ _f64(W["w_gate"][l])) * (y2 @ _f64(W["w_up"][l]))
+        x = x + hmid @ _f64(W["w_down"][l])
+        if trace is not None:
+            trace.setdefault("x", []).append(x.copy())
+
+    scf, shf = mod_slice(cfg, mod, L, 0)
+    v = ada_rmsnorm(x, scf, shf) @ _f64(W["out_w"]) + _f64(W["out_b"])
+    if trace is not None:
+        trace.update(cond=cond, mod=mod)
+    return v
+
+
+def slot_dt(slot_times):
+    """dt_j = t_j - t_{j-1} with t_{-1} = 0 (Eq. 3's Delta tau per slot)."""
+    t = _f64(slot_times)
+    return np.diff(np.concatenate([[0.0], t]))
+
+
+def euler_roll(buffer, velocity, slot_times, seeds, counters):
+    """Eq. 3 then the release / shift / append that follows it.
+
+    a'_j = a_j + dt_j v_j for every slot; slot 0 (now at t = 0) is released; the
+    remaining H-1 slots move forward; the new last slot is the Gaussian action
+    of index n_b (the robot's counter), which then advances by one.
+    Returns (released [B, A], new buffer [B, H, A], new counters [B]).
+    """
+    a = _f64(buffer) + slot_dt(slot_times)[None, :, None] * _f64(velocity)
+    released = a[:, 0].copy()
+    B, H, A = a.shape
+    counters = np.asarray(counters, dtype=np.uint64)
+    fresh = np.stack([action_noise(int(seeds[b]), counters[b], A) for b in range(B)]) \
+        if B else np.zeros((0, A), np.float32)
+    new = np.concatenate([a[:, 1:], _f64(fresh)[:, None, :]], axis=1)
+    return released, new, counters + np.uint64(1)
+
+
+def roll_step(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, seeds, counters,
+              mask: str = "full"):
+    """One rolling action-expert step.  Returns (released, new buffer, new
+    counters, velocity)."""
+    v = expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, mask)
+    released, new, counters = euler_roll(buffer, v, slot_times, seeds, counters)
+    return released, new, counters, v
+
+
+def reset(cfg, seeds, H: int | None = None):
+    """Warm start with no extra initialization (App. A.1): every slot j holds
+    the Gaussian action of index j; the next appended action has index H.
+    Returns (buffer [B, H, A] float32, counters [B] uint64)."""
+    H = cfg.slots if H is None else H
+    B = len(seeds)
+    buf = np.stack([action_noise(int(s), np.arange(H, dtype=np.uint64), cfg.action_dim) for s in seeds]) \
+        if B else np.zeros((0, H, cfg.action_dim), np.float32)
+    return buf.astype(np.float32), np.full(B, H, dtype=np.uint64)

@@ -1,0 +1,315 @@
+"""Pins of the fp64 oracle of the rolling step (Eq. 1, Eq. 3, Sec. 3.1, App. A.1).
+
+Nothing here re-types the oracle's formulas: each test checks it against a
+library routine, a brute-force loop, a closed form of Euler integration, or a
+structural law the step must obey (equivariance, batch independence, slot
+isolation, GQA expansion, residual identity).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import expert, noise
+
+TINY = synth.ExpertConfig(layers=2, width=32, n_q_heads=4, n_kv_heads=2, head_dim=8, mlp_dim=48,
+                          slots=5, action_dim=3, prefix=7, fop_tokens=2, batch=2, dtype="fp32")
+
+
+def _inputs(cfg, seed=0, prefix_len=None, std=0.2):
+    W = synth.make_weights(cfg, seed, std=std)
+    k, v = synth.make_context(cfg, 100)
+    z = synth.make_fop(cfg, 200)
+    t = synth.staggered_times(cfg.slots)
+    d = synth.make_delta(cfg.batch, [2, 5][:cfg.batch] + [1] * max(0, cfg.batch - 2), cfg.slots)
+    buf, cnt = expert.reset(cfg, synth.robot_seeds(7, cfg.batch))
+    return W, buf, t, k, v, cfg.prefix if prefix_len is None else prefix_len, z, d, cnt
+
+
+# ----------------------------------------------------------------------------- parts
+
+@pytest.mark.parametrize("nq,nk,hd", [(1, 1, 4), (3, 7, 8), (6, 12, 5)])
+def test_attention_vs_bruteforce_and_sdpa(nq, nk, hd):
+    rng = np.random.default_rng(nq * 100 + nk)
+    q, k, v = rng.standard_normal((nq, hd)), rng.standard_normal((nk, hd)), rng.standard_normal((nk, hd))
+    valid = rng.random((nq, nk)) < 0.7
+    valid[:, 0] = True
+    got = expert.attention(q, k, v, valid)
+    for i in range(nq):   # brute force, one query at a time
+        s = [sum(q[i, c] * k[j, c] for c in range(hd)) / np.sqrt(hd) for j in range(nk) if valid[i, j]]
+        vv = [v[j] for j in range(nk) if valid[i, j]]
+        w = np.exp(np.array(s) - max(s))
+        np.testing.assert_allclose(got[i], (w[:, None] * np.array(vv)).sum(0) / w.sum(), rtol=1e-12)
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.tensor(q)[None], torch.tensor(k)[None], torch.tensor(v)[None],
+        attn_mask=torch.tensor(valid)[None])[0].numpy()
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_attention_single_key_returns_value():
+    v = np.array([[1.5, -2.0, 3.0]])
+    out = expert.attention(np.ones((4, 3)), np.array([[0.3, 0.1, -9.0]]), v)
+    np.testing.assert_array_equal(out, np.repeat(v, 4, axis=0))
+
+
+def test_ada_rmsnorm_of_constant_row():
+    sc = np.linspace(-0.5, 0.5, 16)
+    sh = np.linspace(1.0, 2.0, 16)
+    for c in (3.0, -40.0):   # eps = 1e-6 is negligible next to c^2
+        y = expert.ada_rmsnorm(np.full(16, c), sc, sh)
+        np.testing.assert_allclose(y, np.sign(c) * (1 + sc) + sh, rtol=1e-6)
+
+
+def test_activations_vs_torch():
+    x = np.linspace(-6, 6, 101)
+    tx = torch.tensor(x)
+    np.testing.assert_allclose(expert.gelu_tanh(x), torch.nn.functional.gelu(tx, approximate="tanh").numpy(),
+                               rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(expert.silu(x), torch.nn.functional.silu(tx).numpy(), rtol=1e-13, atol=1e-15)
+
+
+def test_sinusoidal_embedding_frequencies():
+    D = 64
+    e0 = expert.sinusoidal(np.array([0.0]), D)[0]
+    np.testing.assert_array_equal(e0, np.r_[np.zeros(D // 2), np.ones(D // 2)])
+    # component i completes a full period at x = p_i; p_0 = 4e-3, p_last = 4
+    for i, p in ((0, 4e-3), (D // 2 - 1, 4.0)):
+        e = expert.sinusoidal(np.array([p, p / 4]), D)
+        assert abs(e[0, i]) < 1e-12 and abs(e[0, D // 2 + i] - 1) < 1e-12
+        assert abs(e[1, i] - 1) < 1e-12 and abs(e[1, D // 2 + i]) < 1e-12
+
+
+# ----------------------------------------------------------------------------- Euler / roll
+
+
+def _rollout(cfg, steps, slot_times, field, seeds):
+    """Run ``steps`` rolls from the reset buffer with an externally given
+    velocity field(step, buffer) -> [B, H, A]; returns released [steps, B, A]."""
+    buf, cnt = expert.reset(cfg, seeds)
+    buf = buf.astype(np.float64)
+    out = []
+    for s in range(steps):
+        rel, buf, cnt = expert.euler_roll(buf, field(s, buf), slot_times, seeds, cnt)
+        out.append(rel)
+    return np.array(out)
+
+
+def _received_time(n, t):
+    """Sum of dt an action with index n has received when released: t_min(n, H-1)."""
+    return t[min(n, len(t) - 1)]
+
+
+@pytest.mark.parametrize("schedule", ["staggered", "quadratic"])
+def test_euler_constant_field_closed_form(schedule):
+    cfg = TINY.replace(batch=2, slots=6, action_dim=5)
+    H = cfg.slots
+    t = synth.staggered_times(H) if schedule == "staggered" else (((np.arange(H) + 1) / H) ** 2).astype(np.float32)
+    seeds = synth.robot_seeds(11, 2)
+    c = np.array([0.5, -1.0, 2.0, 0.0, 3.0])
+    rel = _rollout(cfg, 3 * H, t, lambda s, b: np.broadcast_to(c, b.shape), seeds)
+    for n in range(3 * H):
+        for b in range(2):
+            a0 = noise.action_noise(int(seeds[b]), n, cfg.action_dim).astype(np.float64)
+            np.testing.assert_allclose(rel[n, b], a0 + c * float(_received_time(n, t)), rtol=0, atol=1e-12)
+
+
+def test_euler_dt_invariant_each_action_integrates_time_once():
+    # unit field: released - initial noise = total flow time integrated = 1 after warm start
+    cfg = TINY.replace(batch=1, slots=7, action_dim=2)
+    t = synth.staggered_times(cfg.slots)
+    seeds = synth.robot_seeds(3, 1)
+    rel = _rollout(cfg, 4 * cfg.slots, t, lambda s, b: np.ones_like(b), seeds)
+    for n in range(4 * cfg.slots):
+        a0 = noise.action_noise(int(seeds[0]), n, 2).astype(np.float64)
+        want = 1.0 if n >= cfg.slots - 1 else (n + 1) / cfg.slots
+        np.testing.assert_allclose(rel[n, 0] - a0, want, rtol=0, atol=1e-7)
+
+
+def test_euler_linear_and_time_fields_closed_form():
+    cfg = TINY.replace(batch=1, slots=5, action_dim=3)
+    H = cfg.slots
+    t = synth.staggered_times(H)
+    dt = np.diff(np.r_[0.0, t.astype(np.float64)])
+    seeds = synth.robot_seeds(4, 1)
+    alpha = -0.7
+    rel = _rollout(cfg, 3 * H, t, lambda s, b: alpha * b, seeds)
+    f = lambda tt: np.sin(3 * tt) + tt ** 2   # noqa: E731
+    rel_t = _rollout(cfg, 3 * H, t, lambda s, b: np.broadcast_to(f(t.astype(np.float64))[None, :, None], b.shape), seeds)
+    for n in range(3 * H):
+        a0 = noise.action_noise(int(seeds[0]), n, 3).astype(np.float64)
+        k = min(n, H - 1)
+        np.testing.assert_allclose(rel[n, 0], a0 * np.prod(1 + alpha * dt[:k + 1]), rtol=1e-12)
+        np.testing.assert_allclose(rel_t[n, 0], a0 + np.sum(f(t[:k + 1].astype(np.float64)) * dt[:k + 1]),
+                                   rtol=1e-12, atol=1e-12)
+
+
+def test_ideal_single_target_field_releases_targets_in_order():
+    # v*(a, t) = (target - a) / t is the flow-matching field of one data point
+    # (Eq. 5: a^tau = (1 - tau) eps + tau a_hat, velocity a_hat - eps); Euler is
+    # exact on it, so every released action equals its own target, from the
+    # very first (warm-start) step on.
+    cfg = TINY.replace(batch=2, slots=6, action_dim=4)
+    H = cfg.slots
+    t = synth.staggered_times(H).astype(np.float64)
+    steps = 4 * H
+    targets = np.random.default_rng(9).standard_normal((steps + H, 2, 4))
+    seeds = synth.robot_seeds(21, 2)
+
+    def field(s, buf):
+        tgt = np.stack([targets[s + j] for j in range(H)], axis=1)   # slot j holds action s + j
+        return (tgt - buf) / t[None, :, None]
+
+    rel = _rollout(cfg, steps, t.astype(np.float32), field, seeds)
+    np.testing.assert_allclose(rel, targets[:steps], rtol=0, atol=1e-12)
+
+
+def test_reset_and_append_bookkeeping():
+    cfg = TINY.replace(batch=3, slots=4, action_dim=6)
+    seeds = synth.robot_seeds(1 << 40, 3)
+    buf, cnt = expert.reset(cfg, seeds)
+    for b in range(3):
+        for j in range(4):
+            np.testing.assert_array_equal(buf[b, j], noise.action_noise(int(seeds[b]), j, 6))
+    assert list(cnt) == [4, 4, 4]
+    rel, new, cnt2 = expert.euler_roll(buf, np.zeros_like(buf), synth.staggered_times(4), seeds, cnt)
+    np.testing.assert_array_equal(rel, buf[:, 0])
+    np.testing.assert_array_equal(new[:, :3], buf[:, 1:])
+    for b in range(3):
+        np.testing.assert_array_equal(new[b, 3], noise.action_noise(int(seeds[b]), 4, 6))
+    assert list(cnt2) == [5, 5, 5]
+
+
+# ----------------------------------------------------------------------------- the network
+
+
+def test_batch_independence():
+    cfg = TINY.replace(batch=3)
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    full = expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d)
+    for b in range(3):
+        one = expert.expert_velocity(cfg.replace(batch=1), W, buf[b:b + 1], t, k[:, b:b + 1], v[:, b:b + 1], P,
+                                     z[b:b + 1], d[b:b + 1])
+        np.testing.assert_allclose(full[b], one[0], rtol=1e-12, atol=1e-14)
+
+
+def test_slot_permutation_equivariance():
+    # full mask, no positional encoding: slots are told apart only by their times
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    perm = np.array([3, 0, 4, 1, 2])
+    a = expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d)
+    b = expert.expert_velocity(cfg, W, buf[:, perm], t[perm], k, v, P, z, d)
+    np.testing.assert_allclose(b, a[:, perm], rtol=1e-11, atol=1e-13)
+
+
+def test_prefix_permutation_and_padding_are_ignored():
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg, prefix_len=5)
+    a = expert.expert_velocity(cfg, W, buf, t, k, v, 5, z, d)
+    perm = np.r_[np.random.default_rng(2).permutation(5), 5, 6]
+    k2, v2 = k[:, :, :, perm].copy(), v[:, :, :, perm].copy()
+    k2[:, :, :, 5:] = 1e3
+    v2[:, :, :, 5:] = -1e3
+    b = expert.expert_velocity(cfg, W, buf, t, k2, v2, 5, z, d)
+    np.testing.assert_allclose(b, a, rtol=1e-11, atol=1e-13)
+
+
+def test_gqa_equals_mha_with_repeat_interleaved_kv():
+    cfg = TINY            # Hq 4, Hkv 2: heads 0,1 read KV head 0; heads 2,3 read KV head 1
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    hd, Hq, Hkv = cfg.head_dim, cfg.n_q_heads, cfg.n_kv_heads
+    G = Hq // Hkv
+    mha = cfg.replace(n_kv_heads=Hq)
+    W2 = dict(W)
+    wq = W["w_qkv"][:, :, :Hq * hd]
+    wk = W["w_qkv"][:, :, Hq * hd:(Hq + Hkv) * hd].reshape(cfg.layers, cfg.width, Hkv, hd)
+    wv = W["w_qkv"][:, :, (Hq + Hkv) * hd:].reshape(cfg.layers, cfg.width, Hkv, hd)
+    rep = lambda w: np.repeat(w, G, axis=2).reshape(cfg.layers, cfg.width, Hq * hd)  # noqa: E731
+    W2["w_qkv"] = np.concatenate([wq, rep(wk), rep(wv)], axis=2)
+    a = expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d)
+    b = expert.expert_velocity(mha, W2, buf, t, np.repeat(k, G, axis=2), np.repeat(v, G, axis=2), P, z, d)
+    np.testing.assert_allclose(b, a, rtol=1e-11, atol=1e-13)
+
+
+def test_slot_isolated_step_equals_independent_single_slot_calls():
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    whole = expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d, mask="slot_isolated")
+    for j in range(cfg.slots):
+        one = expert.expert_velocity(cfg.replace(slots=1), W, buf[:, j:j + 1], t[j:j + 1], k, v, P, z, d)
+        np.testing.assert_allclose(whole[:, j], one[:, 0], rtol=1e-11, atol=1e-13)
+    full = expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d)
+    assert np.max(np.abs(full - whole)) > 1e-6      # the masks really differ
+
+
+def test_zero_output_projections_make_layers_identity():
+    # x <- x + attn(...) W_o and x <- x + mlp(...) W_down: with both W zero the
+    # layers are the identity and the expert reduces to its zero-layer form
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    W0 = dict(W, w_o=np.zeros_like(W["w_o"]), w_down=np.zeros_like(W["w_down"]))
+    a = expert.expert_velocity(cfg, W0, buf, t, k, v, P, z, d)
+    c0 = cfg.replace(layers=0)
+    Wz = {n: (W[n][:0] if n in ("fop_gamma", "w_qkv", "w_o", "w_gate", "w_up", "w_down") else W[n]) for n in W}
+    Wz["mod_w"], Wz["mod_b"] = W["mod_w"][:, -2 * cfg.width:], W["mod_b"][-2 * cfg.width:]
+    b = expert.expert_velocity(c0, Wz, buf, t, k, v, P, z, d)
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-14)
+    # ... while the full network differs from it
+    assert np.max(np.abs(expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d) - b)) > 1e-3
+
+
+def test_uniform_queries_average_prefix_values_over_all_keys():
+    # W_q = 0 makes every score 0 (uniform softmax over the P + F + H visible
+    # keys); zero K/V projections make FOP and action values 0, so the first
+    # layer's attention output is sum(prefix V) / (P + F + H) per head.
+    cfg = TINY.replace(layers=1)
+    Hq, Hkv, hd = cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim
+    W, buf, t, k, v, _, z, d, _ = _inputs(cfg)
+    P = 5
+    W1 = dict(W, w_qkv=np.zeros_like(W["w_qkv"]), w_gate=np.zeros_like(W["w_gate"]))
+    tr = {}
+    expert.expert_velocity(cfg, W1, buf, t, k, v, P, z, d, trace=tr)
+    x0 = buf.astype(np.float64) @ W["in_w"] + W["in_b"]
+    G = Hq // Hkv
+    o = np.zeros((cfg.batch, Hq * hd))
+    for b in range(cfg.batch):
+        for h in range(Hq):
+            o[b, h * hd:(h + 1) * hd] = v[0, b, h // G, :P].astype(np.float64).sum(0) / (P + cfg.fop_tokens + cfg.slots)
+    want = x0 + (o @ W["w_o"][0].astype(np.float64))[:, None, :]
+    np.testing.assert_allclose(tr["x"][0], want, rtol=1e-11, atol=1e-13)
+
+
+def test_roll_step_composes_velocity_and_roll():
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, cnt = _inputs(cfg)
+    seeds = synth.robot_seeds(7, cfg.batch)
+    rel, new, cnt2, vel = expert.roll_step(cfg, W, buf, t, k, v, P, z, d, seeds, cnt)
+    np.testing.assert_allclose(rel, buf[:, 0] + t[0] * vel[:, 0], rtol=1e-12)
+    assert np.all(cnt2 == cnt + 1)
+    np.testing.assert_allclose(new[:, :-1], buf[:, 1:] + np.diff(np.r_[0, t.astype(np.float64)])[None, 1:, None]
+                               * vel[:, 1:], rtol=1e-12)
+
+
+def test_conditioning_with_permutation_weights_vs_torch_silu():
+    # W1 a permutation, W2 diagonal: cond = silu(emb(t) permuted + b1) * s + b2
+    # for the time MLP, plus the same for the offset MLP (App. A.1: the offset
+    # embedding is added to the flow-timestep embedding).  A transposed or
+    # misplaced operand moves entries and fails this.
+    cfg = TINY.replace(width=16)
+    D = cfg.width
+    rng = np.random.default_rng(3)
+    W = {}
+    want = {}
+    x = {"t": np.array([0.2, 0.6, 1.0]), "d": np.array([0.0, 0.35])}
+    for m in ("t", "d"):
+        pi = rng.permutation(D)
+        P = np.zeros((D, D))
+        P[np.arange(D), pi] = 1.0
+        b1, s, b2 = rng.standard_normal(D), rng.standard_normal(D), rng.standard_normal(D)
+        W.update({f"{m}_w1": P, f"{m}_b1": b1, f"{m}_w2": np.diag(s), f"{m}_b2": b2})
+        e = expert.sinusoidal(x[m], D)
+        moved = np.empty_like(e)
+        moved[:, pi] = e
+        want[m] = torch.nn.functional.silu(torch.tensor(moved + b1)).numpy() * s + b2
+    cond = expert.conditioning(cfg, W, x["t"], x["d"])
+    np.testing.assert_allclose(cond, want["d"][:, None, :] + want["t"][None, :, :], rtol=1e-12, atol=1e-13)
