@@ -1,0 +1,393 @@
+"""Benchmark of the rolling action-expert step on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+A step is one rolling step (conditioning, L transformer layers over the H
+action slots attending to the VLM prefix K/V and the FOP tokens, velocity
+head, Euler update, release, shift, Philox append) for B robots.  Default
+workload: the pi0.5-shaped bf16 expert at batch 1 (18 layers, width 1024, 8
+query heads / 1 KV head of 256, GeGLU 4096, H = 50 slots of dim 32, prefix 816
+tokens, 16 FOP tokens), with a new VLM context swapped in from a side stream
+every 10 steps.  Inputs are seeded synthetic tensors of those shapes; the
+787 MB of weights streamed per step exceed the 129 MB L2, so no L2 flush is
+needed between timed steps.
+
+``value`` is whole-job robot-steps per second (steps/s x robots), the max over
+ranks of the timed region; each rank runs its own robots (replicas, weak
+scaling, no collective on the data path).  ``--impl reference`` times the fp64
+CPU oracle on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p, "measured"
+    except OSError:
+        return PEAKS_FALLBACK, "fallback"
+
+
+# ----------------------------------------------------------------------------- algorithmic work
+
+
+def step_work(cfg, B, P):
+    """Algorithmic bytes and FLOPs of one step as this library computes it:
+    every weight read once, the prefix K/V of each robot read once, inputs and
+    outputs once.  Conditioning MLPs run on H time rows + B offset rows and the
+    modulation Dense on those H + B rows (mod is linear in cond)."""
+    es = 2 if cfg.dtype == "bf16" else 4
+    D, L, H, A, F, Fm = cfg.width, cfg.layers, cfg.slots, cfg.action_dim, cfg.fop_tokens, cfg.mlp_dim
+    nqkv, qd, md = cfg.n_qkv, cfg.q_dim, cfg.mod_dim
+    w_elems = 4 * D * D + D * md + L * (D * nqkv + qd * D + 3 * D * Fm) + D * A
+    f32_params = 4 * D + md + A * D + D + L * D + A
+    kv = B * L * cfg.n_kv_heads * P * cfg.head_dim * 2 * es
+    io = B * F * D * es + B * H * A * 4 * 2 + B * A * 4 + H * 4 + B * 4
+    bytes_ = w_elems * es + f32_params * 4 + kv + io
+    flops = (2 * (H + B) * 2 * D * D + 2 * (H + B) * D * md
+             + L * (2 * B * (H + F) * D * nqkv + 4 * B * cfg.n_q_heads * H * (P + F + H) * cfg.head_dim
+                    + 2 * B * H * qd * D + 2 * B * H * D * 2 * Fm + 2 * B * H * Fm * D)
+             + 2 * B * H * D * A)
+    proj_flops = (2 * (H + B) * 2 * D * D + 2 * (H + B) * D * md
+                  + L * (2 * B * (H + F) * D * nqkv + 2 * B * H * qd * D + 2 * B * H * D * 3 * Fm) + 2 * B * H * D * A)
+    return {"bytes": bytes_, "flops": flops, "proj_flops": proj_flops, "weight_bytes": w_elems * es, "kv_bytes": kv}
+
+
+def kind_work(kind, cfg, B, P):
+    """Algorithmic (bytes, flops) of ONE launch of a kernel kind: its weights,
+    input activations and outputs, each counted once."""
+    es = 2 if cfg.dtype == "bf16" else 4
+    D, H, A, F, Fm = cfg.width, cfg.slots, cfg.action_dim, cfg.fop_tokens, cfg.mlp_dim
+    nqkv, qd, md = cfg.n_qkv, cfg.q_dim, cfg.mod_dim
+    BH, BY = B * H, B * (H + F)
+    if kind == "gemm_gate_up":
+        return (2 * Fm * D + BH * D + BH * Fm) * es, 2 * BH * D * 2 * Fm
+    if kind == "gemm_down":
+        return (D * Fm + BH * Fm) * es + BH * D * 8, 2 * BH * Fm * D
+    if kind == "gemm_qkv":
+        return (nqkv * D + BY * D + BY * nqkv) * es, 2 * BY * D * nqkv
+    if kind == "gemm_o":
+        return (D * qd + BH * qd) * es + BH * D * 8, 2 * BH * qd * D
+    if kind == "gemm_mod":
+        return (md * D + (H + B) * D) * es + (H + B) * md * 4, 2 * (H + B) * D * md
+    if kind == "attention":
+        kv = B * cfg.n_kv_heads * P * cfg.head_dim * 2 * es
+        return kv + (BY * nqkv + BH * qd) * es, 4 * B * cfg.n_q_heads * H * (P + F + H) * cfg.head_dim
+    return None, None
+
+
+# ----------------------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- reference arm (CPU oracle)
+
+
+def run_reference(args, cfg, rank):
+    """Time the fp64 CPU oracle on a bounded sample of the workload."""
+    if rank != 0:
+        return
+    from oracle import expert
+    B = cfg.batch
+    sample_b = min(B, 1)
+    W = synth.make_weights(cfg, 0)
+    k, v = synth.make_context(cfg, 1000, sample_b)
+    z = synth.make_fop(cfg, 2000, sample_b)
+    t = synth.staggered_times(cfg.slots)
+    d = synth.make_delta(sample_b, 2, cfg.slots)
+    seeds = synth.robot_seeds(7, sample_b)
+    buf, cnt = expert.reset(cfg, seeds)
+    for _ in range(args.warmup and 1):
+        expert.roll_step(cfg, W, buf, t, k, v, cfg.prefix, z, d, seeds, cnt)
+    times = []
+    for _ in range(max(1, args.steps)):
+        t0 = time.perf_counter()
+        rel, buf, cnt, _ = expert.roll_step(cfg, W, buf, t, k, v, cfg.prefix, z, d, seeds, cnt)
+        times.append(time.perf_counter() - t0)
+    per_robot_step = float(np.mean(times)) / sample_b
+    value = 1.0 / (per_robot_step * B) * B     # robot-steps per second
+    cores = os.cpu_count()
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_robot_step * B * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(cfg),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"{sample_b} robot(s) of the workload, {len(times)} step(s), numpy fp64"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+METRIC = "rolling-step throughput (robot-steps/s); p50/p99 step latency reported alongside"
+UNIT = "robot-steps/s"
+
+
+def workload_config(cfg):
+    return {"workload": f"rolling action-expert step, {cfg.layers}L d{cfg.width} Hq{cfg.n_q_heads}/Hkv{cfg.n_kv_heads}"
+                        f" hd{cfg.head_dim} GeGLU{cfg.mlp_dim}, H={cfg.slots} A={cfg.action_dim}, "
+                        f"prefix {cfg.prefix}, FOP {cfg.fop_tokens}, batch {cfg.batch}, {cfg.dtype}",
+            "batch": cfg.batch, "slots": cfg.slots, "prefix": cfg.prefix, "layers": cfg.layers,
+            "width": cfg.width, "dtype": cfg.dtype, "l2": "working set (weights + prefix K/V) > 129 MB L2; no flush"}
+
+
+def cpu_baseline(cfg, budget_s=20.0):
+    """Oracle on one robot of the workload, as many steps as fit ~budget_s."""
+    from oracle import expert
+    W = synth.make_weights(cfg, 0)
+    k, v = synth.make_context(cfg, 1000, 1)
+    z = synth.make_fop(cfg, 2000, 1)
+    t = synth.staggered_times(cfg.slots)
+    d = synth.make_delta(1, 2, cfg.slots)
+    seeds = synth.robot_seeds(7, 1)
+    buf, cnt = expert.reset(cfg, seeds)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        _, buf, cnt, _ = expert.roll_step(cfg, W, buf, t, k, v, cfg.prefix, z, d, seeds, cnt)
+        n += 1
+        if time.perf_counter() - t0 > budget_s / 2 or n >= 20:
+            break
+    dt = (time.perf_counter() - t0) / n
+    return {"value": 1.0 / dt, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"1 robot, {n} step(s) of the workload, numpy fp64 ({dt * 1e3:.0f} ms/robot-step)"}
+
+
+# ----------------------------------------------------------------------------- our arm
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--config", default="pi05_bf16_b1", choices=sorted(synth.PRESETS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--swap-every", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-steps", type=int, default=3)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    cfg = synth.PRESETS[args.config]
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, cfg, rank)
+        return
+
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_34170_gb300 import RollingSession, ravel_profile_step, ravel_roll_step
+
+    B, P = cfg.batch, cfg.prefix
+    W = synth.make_weights(cfg, 0)
+    sess = RollingSession(cfg, W, local)
+    del W
+    seeds = synth.robot_seeds(7 + 1000 * rank, B)
+    sess.reset(seeds)
+    dtype = sess.dtype
+    ctxs = []
+    for cs in (1000 + rank * 100, 5000 + rank * 100):
+        k, v = synth.make_context(cfg, cs, B)
+        ctxs.append((torch.from_numpy(k).to("cuda", dtype), torch.from_numpy(v).to("cuda", dtype)))
+        del k, v
+    sess.set_context(*ctxs[0], P)
+    side = torch.cuda.Stream()
+    z = torch.from_numpy(synth.make_fop(cfg, 2000 + rank, B)).to("cuda", dtype)
+    t_d = torch.from_numpy(synth.staggered_times(cfg.slots)).cuda()
+    deltas = [torch.from_numpy(synth.make_delta(B, 2 + (s % 10), cfg.slots)).cuda() for s in range(10)]
+    delta = torch.empty_like(deltas[0])
+    released, velocity = sess.released, None
+    st = torch.cuda.current_stream()
+
+    def one_step(s):
+        if args.swap_every and s % args.swap_every == 0 and s > 0:
+            sess.set_context(*ctxs[(s // args.swap_every) % 2], P, side_stream=side)
+        delta.copy_(deltas[s % 10], non_blocking=True)
+        ravel_roll_step(sess.handle, sess.buffer, t_d, z if cfg.fop_tokens else None, delta, released, velocity, st)
+
+    for s in range(args.warmup):
+        one_step(s)
+    torch.cuda.synchronize()
+    kernels_per_step = sess.kernel_count()
+
+    # ---- timed region: K steps, one event pair per step
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_all0, t_all1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    t_all0.record(st)
+    for s in range(args.steps):
+        ev[s][0].record(st)
+        one_step(args.warmup + s)
+        ev[s][1].record(st)
+    t_all1.record(st)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    total_ms = t_all0.elapsed_time(t_all1)
+    lat = np.array([a.elapsed_time(b) for a, b in ev])
+    if world > 1:
+        tt = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    value = world * B * args.steps / (total_ms / 1e3)
+
+    # ---- e2e: through the C ABI with host buffers, H2D of the step inputs and D2H of the released action
+    z_h = z.cpu().pin_memory()
+    d_h = [d.cpu().pin_memory() for d in deltas]
+    rel_h = torch.empty((B, cfg.action_dim), dtype=torch.float32).pin_memory()
+    z_dev = torch.empty_like(z)
+    for s in range(3):
+        z_dev.copy_(z_h, non_blocking=True)
+        delta.copy_(d_h[s % 10], non_blocking=True)
+        ravel_roll_step(sess.handle, sess.buffer, t_d, z_dev if cfg.fop_tokens else None, delta, released, None, st)
+        rel_h.copy_(released, non_blocking=True)
+        st.synchronize()
+    n_e2e = max(20, args.steps // 2)
+    t0 = time.perf_counter()
+    for s in range(n_e2e):
+        z_dev.copy_(z_h, non_blocking=True)
+        delta.copy_(d_h[s % 10], non_blocking=True)
+        ravel_roll_step(sess.handle, sess.buffer, t_d, z_dev if cfg.fop_tokens else None, delta, released, None, st)
+        rel_h.copy_(released, non_blocking=True)
+        st.synchronize()
+    e2e_s = (time.perf_counter() - t0) / n_e2e
+    h2d = z_h.numel() * z_h.element_size() + B * 4
+    d2h = B * cfg.action_dim * 4
+
+    # ---- per-kernel durations (eager step, events after every launch)
+    per_kind = {}
+    for _ in range(args.profile_steps):
+        for kind, ms in ravel_profile_step(sess.handle, sess.buffer, t_d, z if cfg.fop_tokens else None, delta,
+                                           released, None, st):
+            per_kind.setdefault(kind, []).append(ms)
+    tot = {k: sum(v) / args.profile_steps for k, v in per_kind.items()}
+    grand = sum(tot.values())
+    dom = max(tot, key=tot.get)
+    nlaunch = len(per_kind[dom]) / args.profile_steps
+    avg_ms = float(np.mean(per_kind[dom]))
+    peaks, peak_src = load_peaks()
+    kb, kf = kind_work(dom, cfg, B, P)
+    work = step_work(cfg, B, P)
+    bound = "hbm" if B * cfg.slots <= 512 else "tensor"
+    if bound == "hbm" and kb:
+        achieved, peak, unit = kb / (avg_ms * 1e-3) / 1e9, peaks["hbm_gbs"], "GB/s"
+    elif kf:
+        achieved, peak, unit = kf / (avg_ms * 1e-3) / 1e12, peaks["bf16_tflops_sustained"], "TFLOP/s"
+    else:
+        achieved, peak, unit = None, None, None
+    step_roof_s = max(work["bytes"] / (peaks["hbm_gbs"] * 1e9), work["flops"] / (peaks["bf16_tflops"] * 1e12))
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic (seeded N(0,0.02) weights, N(0,1) prefix/FOP)",
+        "config": dict(workload_config(cfg), parallelism=f"replicas x{world}",
+                       context_swap_every=args.swap_every),
+        "p50_us": float(np.percentile(lat, 50) * 1e3), "p99_us": float(np.percentile(lat, 99) * 1e3),
+        "steps_per_s": args.steps / (total_ms / 1e3),
+        "step_roofline": {"bytes": work["bytes"], "flops": work["flops"], "time_us": step_roof_s * 1e6,
+                          "frac_of_p50": step_roof_s * 1e6 / float(np.percentile(lat, 50) * 1e3),
+                          "peaks": peak_src},
+        "roofline": {"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                     "frac": (achieved / peak) if achieved else None, "traffic": None,
+                     "launches_per_step": nlaunch, "avg_launch_us": avg_ms * 1e3,
+                     "share_of_step": tot[dom] / grand, "peak_source": f"{peak_src} (MEASURED_PEAKS.json)"},
+        "kernel_shares": {k: round(v / grand, 4) for k, v in sorted(tot.items(), key=lambda x: -x[1])},
+        "e2e": {"value": world * B / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": kernels_per_step * args.steps + (args.steps // args.swap_every if args.swap_every else 0),
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        del ctxs
+        out["cpu_baseline"] = cpu_baseline(cfg)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    sess.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

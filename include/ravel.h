@@ -1,0 +1,182 @@
+/*
+ * ravel.h -- C ABI of the GB300 rolling action-expert step.
+ *
+ * The step is the inner loop of RAVEL (asynchronous rolling inference for
+ * flow-based VLAs): one denoising pass of the flow-matching action expert over
+ * an H-slot action buffer whose slots sit at staggered flow times, followed by
+ * a per-slot Euler update, release of the first slot, a shift and the append
+ * of a fresh Gaussian slot (paper Sec. 3.1, Eq. 1 and Eq. 3).  The expert
+ * attends to the latest cached VLM prefix K/V (Eq. 2), reused across steps
+ * until a new one arrives (Sec. 3.2), plus Fast-Observation-Pathway tokens
+ * (Eq. 4), and is conditioned on each slot's flow time and on the context age
+ * delta_p = p / K (Sec. 3.1; App. A.1).
+ *
+ * Conventions shared by every call:
+ *  - B robots, H slots, A action dims, D width, L layers, Hq / Hkv query / KV
+ *    heads, hd head dim, Fm MLP width, P prefix tokens, F FOP tokens.
+ *  - Flow time t = 1 - tau (t = 1 is pure noise).  Slot j (0-based; j = 0 is
+ *    released next) carries slot_times[j]; the Euler step of slot j is
+ *    dt_j = t_j - t_{j-1} with t_{-1} = 0 (the staggered schedule t_j = (j+1)/H
+ *    gives the paper's uniform 1/K).
+ *  - Every pointer argument documented "device" must be device memory on the
+ *    library's device; "host" must be host memory.  Pointers are borrowed for
+ *    the duration of the call and, for device pointers passed to asynchronous
+ *    calls, until the work enqueued on the given stream has completed.
+ *  - Streams are cudaStream_t values passed as void*.  NULL means the legacy
+ *    default stream.
+ *  - Every call returns a status and never aborts.  Asynchronous CUDA errors
+ *    and errors raised by kernels (the device error word) surface on a later
+ *    call as RAVEL_ECUDA / RAVEL_EDEVICE / RAVEL_ETIMEOUT.
+ *  - A handle is not thread-safe: calls on one handle must be serialised.
+ */
+#ifndef RAVEL_H_
+#define RAVEL_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  RAVEL_OK = 0,
+  RAVEL_EINVAL = 1,      /* a null pointer or an argument out of its domain */
+  RAVEL_ESHAPE = 2,      /* a size outside the handle's configuration */
+  RAVEL_ENOMEM = 3,      /* device or host allocation failed */
+  RAVEL_ECUDA = 4,       /* a CUDA call failed; ravel_last_error() has the text */
+  RAVEL_ENOCONTEXT = 5,  /* ravel_roll_step before any ravel_set_context */
+  RAVEL_EBUSY = 6,       /* ravel_set_context while the previous swap is pending */
+  RAVEL_EDEVICE = 7,     /* a kernel raised the device error word (e.g. bad prefix length) */
+  RAVEL_ETIMEOUT = 8,    /* a bounded device-side wait ran out */
+  RAVEL_ENOTREADY = 9    /* a call that needs ravel_reset first */
+} ravel_status;
+
+enum { RAVEL_FP32 = 0, RAVEL_BF16 = 1 };
+enum { RAVEL_MASK_FULL = 0, RAVEL_MASK_SLOT_ISOLATED = 1 };
+
+/* Shape of the expert and capacity of the handle. */
+typedef struct {
+  int layers;       /* L */
+  int width;        /* D, even */
+  int n_q_heads;    /* Hq, a multiple of n_kv_heads */
+  int n_kv_heads;   /* Hkv */
+  int head_dim;     /* hd, a multiple of 8, at most 256 */
+  int mlp_dim;      /* Fm, a multiple of 64 */
+  int slots;        /* H (the paper's K with one action per slot) */
+  int action_dim;   /* A */
+  int max_prefix;   /* largest prefix length a context may carry */
+  int fop_tokens;   /* F (0 allowed) */
+  int max_batch;    /* largest B accepted by ravel_reset */
+  int dtype;        /* RAVEL_FP32: all arithmetic fp32; RAVEL_BF16: weights, prefix,
+                       FOP tokens and GEMM activations bf16, fp32 accumulation,
+                       fp32 residual stream, norms, softmax and buffer */
+  int mask_mode;    /* RAVEL_MASK_FULL: every action query sees the valid prefix,
+                       all FOP tokens and all H slots; RAVEL_MASK_SLOT_ISOLATED
+                       (a test mode): action query j sees the prefix, the FOP
+                       tokens and slot j only */
+} ravel_config;
+
+/*
+ * Expert parameters, float32, math layout y = x @ W + b (W is [in, out],
+ * row-major).  Per-layer tensors are stacked on a leading L axis.
+ *   t_w1,t_w2 [D,D]  t_b1,t_b2 [D]   flow-time MLP  (Linear, SiLU, Linear)
+ *   d_w1,d_w2 [D,D]  d_b1,d_b2 [D]   context-offset MLP (App. A.1)
+ *   mod_w [D, 4LD+2D]  mod_b [4LD+2D] adaRMSNorm modulation; columns of layer l
+ *                     are (scale1, shift1, scale2, shift2) at 4lD, then the
+ *                     final norm's (scale, shift) at 4LD
+ *   in_w [A,D] in_b [D]              action in-projection
+ *   fop_gamma [L,D]                  per-layer FOP-token RMSNorm gain (1 + gamma)
+ *   w_qkv [L,D,(Hq+2Hkv)hd]          columns [Q heads | K heads | V heads]
+ *   w_o [L,Hq hd,D]  w_gate,w_up [L,D,Fm]  w_down [L,Fm,D]
+ *   out_w [D,A] out_b [A]            velocity head
+ * on_device = 0: host pointers; 1: device pointers.  ravel_create copies and
+ * repacks everything; the caller keeps ownership.  In RAVEL_BF16 mode values
+ * are rounded to bf16 (nearest, ties to even).
+ */
+typedef struct {
+  const float *t_w1, *t_b1, *t_w2, *t_b2;
+  const float *d_w1, *d_b1, *d_w2, *d_b2;
+  const float *mod_w, *mod_b;
+  const float *in_w, *in_b;
+  const float *fop_gamma;
+  const float *w_qkv, *w_o, *w_gate, *w_up, *w_down;
+  const float *out_w, *out_b;
+  int on_device;
+} ravel_weights;
+
+typedef struct ravel_ctx ravel_t;
+
+/* Validate cfg, allocate the handle on `device` (the CUDA ordinal), pack the
+ * weights into HBM and allocate the double-buffered context, activations and
+ * step state for cfg.max_batch robots.  Synchronous.  On success *out owns all
+ * of it until ravel_destroy. */
+ravel_status ravel_create(const ravel_config* cfg, const ravel_weights* w, int device, ravel_t** out);
+
+/* Free everything the handle owns (after synchronising its device).  NULL is a no-op. */
+void ravel_destroy(ravel_t* r);
+
+/* Start a rollout of `batch` robots (warm start without extra initialisation,
+ * App. A.1): robot b's noise seed is seeds[b] (host, [batch]); slot j of
+ * buffer (device, float32 [batch, H, A], written) receives the Gaussian action
+ * of index j, and the robot's next appended action gets index H.  Enqueued on
+ * `stream`.  A new batch size invalidates the current context (set it again). */
+ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* buffer, void* stream);
+
+/* Install a new VLM context (Eq. 2): k and v are device arrays
+ * [L, B, Hkv, prefix_len, hd] of the handle's dtype (float32 or bf16) for the
+ * current batch B.  The copy goes into the inactive half of the double buffer
+ * on `side_stream`, after the last enqueued step has finished reading it, so
+ * steps on other streams continue meanwhile; the next ravel_roll_step makes
+ * its stream wait for the copy and then switches to the new context.  The
+ * caller may reuse k / v once the side stream has passed this call.
+ * 1 <= prefix_len <= max_prefix, else RAVEL_ESHAPE.  A second call before a
+ * step has consumed the first returns RAVEL_EBUSY. */
+ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int prefix_len, void* side_stream);
+
+/* One rolling step (Eq. 3 plus release / shift / append) for the current
+ * batch, enqueued on `stream` as one CUDA-graph launch:
+ *   buffer      device float32 [B, H, A], read and updated in place
+ *   slot_times  device float32 [H], increasing, slot_times[H-1] = 1 for the
+ *               paper's schedule
+ *   obs_tokens  device [B, F, D] FOP tokens of the handle's dtype (NULL iff F = 0)
+ *   delta       device float32 [B], context age p/K (+ bias) per robot
+ *   released    device float32 [B, A], written: the action released by each robot
+ *   velocity    device float32 [B, H, A] or NULL: the expert's velocity
+ * The step graph is captured on first use and re-captured when any of these
+ * pointers changes; graph capture needs no caller action. */
+ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                             const float* delta, float* released, float* velocity, void* stream);
+
+/* Per-robot action counters (the index of the next appended action), host
+ * uint64 [B].  get synchronises the handle's device; set is synchronous and
+ * lets a rollout resume bit-exactly. */
+ravel_status ravel_get_state(ravel_t* r, uint64_t* counters);
+ravel_status ravel_set_state(ravel_t* r, const uint64_t* counters);
+
+/* Number of kernel launches one ravel_roll_step graph contains (0 before the
+ * first step). */
+int ravel_step_kernel_count(const ravel_t* r);
+
+/* ravel_roll_step run eagerly (no graph) with a CUDA event after every kernel
+ * launch, for per-kernel timing: same arguments and effects, plus host
+ * outputs launch_ms [cap] (duration of each launch in ms) and launch_kind
+ * [cap] (kind id, see ravel_kernel_kind_name); *n_launches receives the
+ * number of launches (entries beyond cap are dropped).  The stream is first
+ * held for ~5 ms so that all launches are queued before the first one starts.
+ * Synchronous. */
+ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                                const float* delta, float* released, float* velocity, void* stream,
+                                float* launch_ms, int* launch_kind, int cap, int* n_launches);
+
+/* Name of a kernel kind id of ravel_profile_step ("gemm_down", ...). */
+const char* ravel_kernel_kind_name(int kind);
+
+/* Static text of a status; per-handle text of the last error (never NULL). */
+const char* ravel_status_string(ravel_status s);
+const char* ravel_last_error(const ravel_t* r);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RAVEL_H_ */

@@ -1,0 +1,106 @@
+// Internal launch API of the rolling-step kernels (host side).  Every launcher
+// enqueues on `st` and returns the launch's cudaError_t.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ravel {
+
+enum Dtype { DT_F32 = 0, DT_BF16 = 1 };
+
+// Bits of the device error word (one int in HBM, OR-ed by kernels, read by the host).
+enum : int {
+  ERR_PREFIX_LEN = 1 << 0,   // the active context's prefix length was out of range
+  ERR_TIMEOUT = 1 << 1,      // a bounded mbarrier / flag wait ran out
+  ERR_SHAPE = 1 << 2,        // a kernel was launched with sizes it cannot handle
+};
+
+// Kernel attributes (dynamic shared memory limits); called once per handle,
+// outside any stream capture.
+cudaError_t init_simt_kernels();
+
+// ---- weight packing ---------------------------------------------------------
+// dst[n][k] = src[k][n] converted to `dt` (src float32 [K, N] row-major).
+// interleave64: dst row of column n is (n/64)*128 + off + n%64 (gate/up tiles).
+cudaError_t launch_pack_transpose(const float* src, int K, int N, void* dst, Dtype dt, int interleave64,
+                                  int off, cudaStream_t st);
+cudaError_t launch_convert(const float* src, size_t n, void* dst, Dtype dt, cudaStream_t st);
+
+// ---- conditioning -------------------------------------------------------------
+// E[r][:] = sinusoidal(x_r) for r < H (x = slot_times[r]) and H <= r < H+B
+// (x = delta[r-H]); periods geometric from 4e-3 to 4; fp64 angles.
+cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, void* E, Dtype dt,
+                         cudaStream_t st);
+
+// ---- generic projection GEMM: out[m][n] = sum_k A[m][k] W[n][k] (W K-major) ----
+enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2 };
+struct GemmArgs {
+  const void* A; int lda;       // [M][K] activations of dtype dt
+  const void* W; int ldw;       // [N][K] weights of dtype dt
+  int M, N, K;
+  Epi epi;
+  void* out; int ldo;           // EPI_STORE*: dtype `out_dt`; EPI_ADD_F32: float, += result
+  Dtype out_dt;
+  const float* bias;            // [N] or null
+};
+cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
+
+// ---- adaRMSNorm rows ---------------------------------------------------------
+// Action rows r < B*H (b = r / H, j = r % H):
+//   Y[r] = x[r] * rsqrt(mean(x[r]^2) + 1e-6) * (1 + sc) + sh,
+//   sc[c] = modv[j][off+c] + modv[H+b][off+c] + mod_b[off+c], sh likewise at off+D.
+// FOP rows B*H + b*F + f (when fop != null): Y = z * rsqrt(mean(z^2)+1e-6) * (1 + gamma).
+struct NormArgs {
+  const float* x; int B, H, D;
+  const float* modv; int mod_ld; const float* mod_b; int off;
+  const void* fop; int F; const float* gamma;
+  void* Y;
+};
+cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
+
+// ---- action in-projection: x[b*H+j][c] = sum_a buf[b][j][a] in_w[a][c] + in_b[c] ----
+cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b,
+                           float* x, cudaStream_t st);
+
+// ---- GeGLU on the interleaved gate/up GEMM output --------------------------------
+cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cudaStream_t st);
+
+// ---- attention ---------------------------------------------------------------
+struct AttnArgs {
+  const void* qkv; int ld_qkv;      // rows: B*H action rows, then B*F FOP rows
+  const void* ctx_k0; const void* ctx_k1;   // the two context slots [L][Bmax][Hkv][Pmax][hd]
+  const void* ctx_v0; const void* ctx_v1;
+  const int* ctx_state;             // device: [0] active slot, [1] prefix length
+  int layer, Bmax, Pmax;
+  int B, H, F, Hq, Hkv, hd;
+  int mask_mode;
+  void* out; int ld_out;            // [B*H][Hq*hd]
+  int* err;
+};
+cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st);
+
+// ---- rolling tail: Euler, release, shift, append ------------------------------------
+struct TailArgs {
+  float* buffer;             // [B][H][A] in place
+  const float* vel;          // [B*H][A]
+  const float* slot_times;   // [H]
+  float* released;           // [B][A]
+  float* vel_out;            // optional copy of vel ([B][H][A])
+  const uint64_t* seeds;     // [B]
+  uint64_t* counters;        // [B], advanced by one
+  int B, H, A;
+};
+cudaError_t launch_tail(const TailArgs& a, cudaStream_t st);
+
+// buffer[b][j] = noise(seeds[b], j) for j < H; counters[b] = H.
+cudaError_t launch_reset(float* buffer, const uint64_t* seeds, uint64_t* counters, int B, int H, int A,
+                         cudaStream_t st);
+
+// Busy-wait on the device for `ns` nanoseconds (globaltimer), then return.
+cudaError_t launch_delay(unsigned long long ns, cudaStream_t st);
+
+// ctx_state = {slot, prefix_len}
+cudaError_t launch_flip(int* ctx_state, int slot, int prefix_len, cudaStream_t st);
+
+}  // namespace ravel

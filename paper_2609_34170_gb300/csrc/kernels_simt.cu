@@ -1,0 +1,502 @@
+// SIMT kernels of the rolling step: weight packing, conditioning embedding,
+// adaRMSNorm, action in-projection, generic projection GEMM (fp32 FFMA; the
+// exact path of fp32 mode), GeGLU, grouped-query attention, and the rolling
+// tail (Euler update, release, shift, Philox append).
+#include "common.cuh"
+#include "kernels.h"
+#include "noise.cuh"
+
+namespace ravel {
+
+// ============================================================================ packing
+
+template <typename T>
+__global__ void pack_transpose_kernel(const float* __restrict__ src, int K, int N, T* __restrict__ dst,
+                                      int interleave64, int off) {
+  __shared__ float tile[32][33];
+  const int n0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int k = k0 + i, n = n0 + threadIdx.x;
+    tile[i][threadIdx.x] = (k < K && n < N) ? src[(size_t)k * N + n] : 0.f;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int n = n0 + i, k = k0 + threadIdx.x;
+    if (n < N && k < K) {
+      const size_t row = interleave64 ? (size_t)(n / 64) * 128 + off + (n % 64) : (size_t)n;
+      dst[row * K + k] = from_f32<T>(tile[threadIdx.x][i]);
+    }
+  }
+}
+
+cudaError_t launch_pack_transpose(const float* src, int K, int N, void* dst, Dtype dt, int interleave64, int off,
+                                  cudaStream_t st) {
+  dim3 grid((N + 31) / 32, (K + 31) / 32), block(32, 8);
+  if (dt == DT_BF16)
+    pack_transpose_kernel<bf16><<<grid, block, 0, st>>>(src, K, N, (bf16*)dst, interleave64, off);
+  else
+    pack_transpose_kernel<float><<<grid, block, 0, st>>>(src, K, N, (float*)dst, interleave64, off);
+  return cudaGetLastError();
+}
+
+template <typename T>
+__global__ void convert_kernel(const float* __restrict__ src, size_t n, T* __restrict__ dst) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+    dst[i] = from_f32<T>(src[i]);
+}
+
+cudaError_t launch_convert(const float* src, size_t n, void* dst, Dtype dt, cudaStream_t st) {
+  const int blocks = (int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  if (n == 0) return cudaSuccess;
+  if (dt == DT_BF16)
+    convert_kernel<bf16><<<blocks, 256, 0, st>>>(src, n, (bf16*)dst);
+  else
+    convert_kernel<float><<<blocks, 256, 0, st>>>(src, n, (float*)dst);
+  return cudaGetLastError();
+}
+
+// ============================================================================ embedding
+
+// Sinusoidal embedding of a scalar (flow time or context offset): component
+// i < D/2 is sin(x w_i), i >= D/2 is cos(x w_{i-D/2}), w_i = 2 pi / p_i with
+// periods p_i geometric from 4e-3 to 4.  Angles in fp64: x w reaches ~1.6e3
+// rad, where a float32 angle would already be off by ~1e-4.
+template <typename T>
+__global__ void embed_kernel(const float* __restrict__ slot_times, int H, const float* __restrict__ delta, int D,
+                             T* __restrict__ E) {
+  const int r = blockIdx.x;
+  const double x = (r < H) ? (double)slot_times[r] : (double)delta[r - H];
+  const int half = D / 2;
+  for (int i = threadIdx.x; i < half; i += blockDim.x) {
+    const double period = 4e-3 * pow(1000.0, (double)i / (double)(half - 1));
+    const double ang = x * (6.283185307179586 / period);
+    double s, c;
+    sincos(ang, &s, &c);
+    E[(size_t)r * D + i] = from_f32<T>((float)s);
+    E[(size_t)r * D + half + i] = from_f32<T>((float)c);
+  }
+}
+
+cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, void* E, Dtype dt,
+                         cudaStream_t st) {
+  if (dt == DT_BF16)
+    embed_kernel<bf16><<<H + B, 128, 0, st>>>(slot_times, H, delta, D, (bf16*)E);
+  else
+    embed_kernel<float><<<H + B, 128, 0, st>>>(slot_times, H, delta, D, (float*)E);
+  return cudaGetLastError();
+}
+
+// ============================================================================ GEMM (SIMT)
+
+// 64x64 output tile, K step 32, 256 threads, 4x4 outputs per thread spread
+// with stride 16 so that shared-memory reads are broadcast-friendly.
+template <typename T, int EPI, typename TO>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, int lda, const T* __restrict__ W,
+                                                        int ldw, int M, int N, int K, TO* __restrict__ out, int ldo,
+                                                        const float* __restrict__ bias) {
+  __shared__ float As[32][64 + 4];
+  __shared__ float Ws[32][64 + 4];
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < K; k0 += 32) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int idx = threadIdx.x + 256 * i;
+      const int r = idx >> 5, kk = idx & 31;
+      const int m = m0 + r, n = n0 + r, k = k0 + kk;
+      As[kk][r] = (m < M && k < K) ? to_f32(A[(size_t)m * lda + k]) : 0.f;
+      Ws[kk][r] = (n < N && k < K) ? to_f32(W[(size_t)n * ldw + k]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int kk = 0; kk < 32; ++kk) {
+      float a[4], w[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) w[j] = Ws[kk][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], w[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int m = m0 + ty + 16 * i;
+    if (m >= M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int n = n0 + tx + 16 * j;
+      if (n >= N) continue;
+      float v = acc[i][j] + (bias ? bias[n] : 0.f);
+      if (EPI == EPI_STORE_SILU) v = silu_f(v);
+      if (EPI == EPI_ADD_F32)
+        ((float*)out)[(size_t)m * ldo + n] += v;
+      else
+        out[(size_t)m * ldo + n] = from_f32<TO>(v);
+    }
+  }
+}
+
+template <typename T>
+static cudaError_t gemm_simt_dispatch(const GemmArgs& g, cudaStream_t st) {
+  dim3 grid((g.N + 63) / 64, (g.M + 63) / 64);
+  const T* A = (const T*)g.A;
+  const T* W = (const T*)g.W;
+  if (g.epi == EPI_ADD_F32) {
+    gemm_simt_kernel<T, EPI_ADD_F32, float><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
+                                                                 g.ldo, g.bias);
+  } else if (g.out_dt == DT_BF16) {
+    if (g.epi == EPI_STORE_SILU)
+      gemm_simt_kernel<T, EPI_STORE_SILU, bf16><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K,
+                                                                     (bf16*)g.out, g.ldo, g.bias);
+    else
+      gemm_simt_kernel<T, EPI_STORE, bf16><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K, (bf16*)g.out,
+                                                                g.ldo, g.bias);
+  } else {
+    if (g.epi == EPI_STORE_SILU)
+      gemm_simt_kernel<T, EPI_STORE_SILU, float><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K,
+                                                                      (float*)g.out, g.ldo, g.bias);
+    else
+      gemm_simt_kernel<T, EPI_STORE, float><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
+                                                                 g.ldo, g.bias);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st) {
+  if (g.M <= 0 || g.N <= 0) return cudaSuccess;
+  return dt == DT_BF16 ? gemm_simt_dispatch<bf16>(g, st) : gemm_simt_dispatch<float>(g, st);
+}
+
+// ============================================================================ adaRMSNorm
+
+template <typename T>
+__global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a) {
+  __shared__ float red[32];
+  const int r = blockIdx.x;
+  const int D = a.D;
+  const int n_act = a.B * a.H;
+  T* Y = (T*)a.Y + (size_t)r * D;
+  if (r < n_act) {
+    const int b = r / a.H, j = r % a.H;
+    const float* x = a.x + (size_t)r * D;
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < D; c += blockDim.x) ss += x[c] * x[c];
+    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
+    const float* mt = a.modv + (size_t)j * a.mod_ld + a.off;
+    const float* md = a.modv + (size_t)(a.H + b) * a.mod_ld + a.off;
+    const float* mb = a.mod_b + a.off;
+    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+      const float sc = mt[c] + md[c] + mb[c];
+      const float sh = mt[D + c] + md[D + c] + mb[D + c];
+      Y[c] = from_f32<T>(x[c] * inv * (1.f + sc) + sh);
+    }
+  } else {
+    const T* z = (const T*)a.fop + (size_t)(r - n_act) * D;
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+      const float v = to_f32(z[c]);
+      ss += v * v;
+    }
+    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
+    for (int c = threadIdx.x; c < D; c += blockDim.x) Y[c] = from_f32<T>(to_f32(z[c]) * inv * (1.f + a.gamma[c]));
+  }
+}
+
+cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st) {
+  const int rows = a.B * a.H + (a.fop ? a.B * a.F : 0);
+  if (rows <= 0) return cudaSuccess;
+  if (dt == DT_BF16)
+    ada_norm_kernel<bf16><<<rows, 256, 0, st>>>(a);
+  else
+    ada_norm_kernel<float><<<rows, 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+// ============================================================================ in-proj
+
+__global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, const float* __restrict__ in_w,
+                               const float* __restrict__ in_b, float* __restrict__ x) {
+  const int r = blockIdx.x;
+  const float* a = buf + (size_t)r * A;
+  for (int c = threadIdx.x; c < D; c += blockDim.x) {
+    float acc = in_b[c];
+    for (int i = 0; i < A; ++i) acc = fmaf(a[i], in_w[(size_t)i * D + c], acc);
+    x[(size_t)r * D + c] = acc;
+  }
+}
+
+cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b, float* x,
+                           cudaStream_t st) {
+  if (BH <= 0) return cudaSuccess;
+  in_proj_kernel<<<BH, 256, 0, st>>>(buf, A, D, in_w, in_b, x);
+  return cudaGetLastError();
+}
+
+// ============================================================================ GeGLU
+
+template <typename T>
+__global__ void geglu_kernel(const float* __restrict__ GU, int M, int Fm, T* __restrict__ Hm) {
+  const size_t total = (size_t)M * Fm;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+    const int m = (int)(i / Fm), f = (int)(i % Fm);
+    const size_t base = (size_t)m * 2 * Fm + (size_t)(f / 64) * 128 + (f % 64);
+    Hm[i] = from_f32<T>(gelu_tanh_f(GU[base]) * GU[base + 64]);
+  }
+}
+
+cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cudaStream_t st) {
+  const size_t total = (size_t)M * Fm;
+  if (!total) return cudaSuccess;
+  const int blocks = (int)((total + 255) / 256 < 8192 ? (total + 255) / 256 : 8192);
+  if (dt == DT_BF16)
+    geglu_kernel<bf16><<<blocks, 256, 0, st>>>(GU, M, Fm, (bf16*)Hm);
+  else
+    geglu_kernel<float><<<blocks, 256, 0, st>>>(GU, M, Fm, (float*)Hm);
+  return cudaGetLastError();
+}
+
+// ============================================================================ attention (SIMT)
+
+// One CTA per (robot b, KV head g, tile of QT query rows).  Query row r of a
+// (b, g) pair is slot j = r / G of query head g*G + r % G.  Keys are visited
+// in chunks of KT: [0, P) the active context's prefix, [P, P+F) the FOP
+// tokens, [P+F, P+F+H) the action slots; online softmax in fp32.
+constexpr int ATT_QT = 16, ATT_KT = 32, ATT_THREADS = 256;
+
+template <typename T>
+__global__ void __launch_bounds__(ATT_THREADS) attention_simt_kernel(AttnArgs a) {
+  extern __shared__ float sm[];
+  const int hd = a.hd;
+  float* Qs = sm;                      // [QT][hd]
+  float* Ks = Qs + ATT_QT * hd;        // [KT][hd]
+  float* Vs = Ks + ATT_KT * hd;        // [KT][hd]
+  float* Ss = Vs + ATT_KT * hd;        // [QT][KT]
+  const int bg = blockIdx.x;
+  const int b = bg / a.Hkv, g = bg % a.Hkv;
+  const int G = a.Hq / a.Hkv;
+  const int nrows = a.H * G;
+  const int r0 = blockIdx.y * ATT_QT;
+  const int slot = a.ctx_state[0];
+  const int P = a.ctx_state[1];
+  if (P < 0 || P > a.Pmax) {
+    if (threadIdx.x == 0) raise_error(a.err, ERR_PREFIX_LEN);
+    return;
+  }
+  const T* qkv = (const T*)a.qkv;
+  const size_t ctx_off = ((((size_t)a.layer * a.Bmax + b) * a.Hkv + g) * (size_t)a.Pmax) * hd;
+  const T* pk = (const T*)(slot ? a.ctx_k1 : a.ctx_k0) + ctx_off;
+  const T* pv = (const T*)(slot ? a.ctx_v1 : a.ctx_v0) + ctx_off;
+  const int kofs = a.Hq * hd + g * hd, vofs = (a.Hq + a.Hkv) * hd + g * hd;
+  const int nk = P + a.F + a.H;
+  const float scale = rsqrtf((float)hd);
+
+  for (int i = threadIdx.x; i < ATT_QT * hd; i += ATT_THREADS) {
+    const int rr = i / hd, c = i % hd, r = r0 + rr;
+    float v = 0.f;
+    if (r < nrows) {
+      const int j = r / G, h = g * G + r % G;
+      v = to_f32(qkv[(size_t)(b * a.H + j) * a.ld_qkv + h * hd + c]);
+    }
+    Qs[i] = v * scale;
+  }
+  // thread layout for scores / softmax: 16 threads per query row
+  const int srow = threadIdx.x >> 4, slane = threadIdx.x & 15;
+  float m_run = -INFINITY, l_run = 0.f;
+  // output accumulators: row orow, columns ocol + 16*i
+  const int orow = threadIdx.x >> 4, ocol = threadIdx.x & 15;
+  float acc[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+  const int qrow_slot = (r0 + srow < nrows) ? (r0 + srow) / G : -1;
+
+  for (int k0 = 0; k0 < nk; k0 += ATT_KT) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < ATT_KT * hd; i += ATT_THREADS) {
+      const int kk = i / hd, c = i % hd, key = k0 + kk;
+      float kv = 0.f, vv = 0.f;
+      if (key < P) {
+        kv = to_f32(pk[(size_t)key * hd + c]);
+        vv = to_f32(pv[(size_t)key * hd + c]);
+      } else if (key < P + a.F) {
+        const size_t row = (size_t)(a.B * a.H + b * a.F + (key - P)) * a.ld_qkv;
+        kv = to_f32(qkv[row + kofs + c]);
+        vv = to_f32(qkv[row + vofs + c]);
+      } else if (key < nk) {
+        const size_t row = (size_t)(b * a.H + (key - P - a.F)) * a.ld_qkv;
+        kv = to_f32(qkv[row + kofs + c]);
+        vv = to_f32(qkv[row + vofs + c]);
+      }
+      Ks[i] = kv;
+      Vs[i] = vv;
+    }
+    __syncthreads();
+    // scores: row srow, keys slane and slane + 16
+    float s[2];
+#pragma unroll
+    for (int t = 0; t < 2; ++t) {
+      const int kk = slane + 16 * t, key = k0 + kk;
+      float d = 0.f;
+      for (int c = 0; c < hd; ++c) d = fmaf(Qs[srow * hd + c], Ks[kk * hd + c], d);
+      bool vis = key < nk;
+      if (a.mask_mode == 1 && key >= P + a.F && key < nk) vis = vis && (key - P - a.F == qrow_slot);
+      s[t] = vis ? d : -INFINITY;
+    }
+    float cmax = fmaxf(s[0], s[1]);
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) cmax = fmaxf(cmax, __shfl_xor_sync(0xffffffffu, cmax, o));
+    const float m_new = fmaxf(m_run, cmax);
+    const float corr = (m_new == -INFINITY) ? 1.f : __expf(m_run - m_new);
+    float psum = 0.f;
+#pragma unroll
+    for (int t = 0; t < 2; ++t) {
+      const float p = (s[t] == -INFINITY) ? 0.f : __expf(s[t] - m_new);
+      Ss[srow * ATT_KT + slane + 16 * t] = p;
+      psum += p;
+    }
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) psum += __shfl_xor_sync(0xffffffffu, psum, o);
+    l_run = l_run * corr + psum;
+    m_run = m_new;
+    __syncthreads();
+    // P V: orow == srow, so corr is this thread's own row correction
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int c = ocol + 16 * i;
+      if (c < hd) {
+        float v = acc[i] * corr;
+        for (int kk = 0; kk < ATT_KT; ++kk) v = fmaf(Ss[orow * ATT_KT + kk], Vs[kk * hd + c], v);
+        acc[i] = v;
+      }
+    }
+  }
+  const int r = r0 + orow;
+  if (r < nrows) {
+    const int j = r / G, h = g * G + r % G;
+    T* o = (T*)a.out + (size_t)(b * a.H + j) * a.ld_out + h * hd;
+    const float inv = 1.f / l_run;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int c = ocol + 16 * i;
+      if (c < hd) o[c] = from_f32<T>(acc[i] * inv);
+    }
+  }
+}
+
+cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st) {
+  if (a.hd > 256 || a.hd % 8) return cudaErrorInvalidValue;
+  const int G = a.Hq / a.Hkv;
+  dim3 grid(a.B * a.Hkv, (a.H * G + ATT_QT - 1) / ATT_QT);
+  const size_t smem = (size_t)(ATT_QT * a.hd + 2 * ATT_KT * a.hd + ATT_QT * ATT_KT) * sizeof(float);
+  if (dt == DT_BF16)
+    attention_simt_kernel<bf16><<<grid, ATT_THREADS, smem, st>>>(a);
+  else
+    attention_simt_kernel<float><<<grid, ATT_THREADS, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+// ============================================================================ tail
+
+// One CTA per robot: a'_j = a_j + dt_j v_j (Eq. 3), released = a'_0, buffer
+// slots shift forward, the last slot receives the Gaussian action of index
+// counters[b], and the counter advances.
+__global__ void tail_kernel(TailArgs a) {
+  extern __shared__ float sa[];   // [H][A]
+  const int b = blockIdx.x;
+  const int H = a.H, A = a.A;
+  float* buf = a.buffer + (size_t)b * H * A;
+  const float* v = a.vel + (size_t)b * H * A;
+  for (int i = threadIdx.x; i < H * A; i += blockDim.x) {
+    const int j = i / A;
+    const float t1 = a.slot_times[j];
+    const float t0 = j ? a.slot_times[j - 1] : 0.f;
+    const float dt = __fsub_rn(t1, t0);
+    sa[i] = fmaf(dt, v[i], buf[i]);
+    if (a.vel_out) a.vel_out[(size_t)b * H * A + i] = v[i];
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < H * A; i += blockDim.x) {
+    if (i < A) a.released[(size_t)b * A + i] = sa[i];
+    if (i < (H - 1) * A) buf[i] = sa[i + A];
+  }
+  const uint64_t n = a.counters[b];
+  const uint64_t seed = a.seeds[b];
+  for (int g = threadIdx.x; g < (A + 3) / 4; g += blockDim.x) {
+    float z[4];
+    action_noise4(seed, n, (uint32_t)g, z);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (4 * g + i < A) buf[(size_t)(H - 1) * A + 4 * g + i] = z[i];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) a.counters[b] = n + 1;
+}
+
+cudaError_t launch_tail(const TailArgs& a, cudaStream_t st) {
+  if (a.B <= 0) return cudaSuccess;
+  const size_t smem = (size_t)a.H * a.A * sizeof(float);
+  tail_kernel<<<a.B, 256, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t init_simt_kernels() {
+  const int att = (ATT_QT * 256 + 2 * ATT_KT * 256 + ATT_QT * ATT_KT) * (int)sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(attention_simt_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, att);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attention_simt_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, att);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tail_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * (int)sizeof(float));
+  return e;
+}
+
+__global__ void reset_kernel(float* __restrict__ buffer, const uint64_t* __restrict__ seeds,
+                             uint64_t* __restrict__ counters, int H, int A) {
+  const int b = blockIdx.x;
+  const int groups = (A + 3) / 4;
+  for (int i = threadIdx.x; i < H * groups; i += blockDim.x) {
+    const int j = i / groups, g = i % groups;
+    float z[4];
+    action_noise4(seeds[b], (uint64_t)j, (uint32_t)g, z);
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+      if (4 * g + t < A) buffer[((size_t)b * H + j) * A + 4 * g + t] = z[t];
+  }
+  if (threadIdx.x == 0) counters[b] = (uint64_t)H;
+}
+
+cudaError_t launch_reset(float* buffer, const uint64_t* seeds, uint64_t* counters, int B, int H, int A,
+                         cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  reset_kernel<<<B, 128, 0, st>>>(buffer, seeds, counters, H, A);
+  return cudaGetLastError();
+}
+
+__global__ void delay_kernel(unsigned long long ns) {
+  unsigned long long t0, t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  do {
+    __nanosleep(10000);
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  } while (t - t0 < ns);
+}
+
+cudaError_t launch_delay(unsigned long long ns, cudaStream_t st) {
+  delay_kernel<<<1, 1, 0, st>>>(ns);
+  return cudaGetLastError();
+}
+
+__global__ void flip_kernel(int* s, int slot, int len) {
+  s[0] = slot;
+  s[1] = len;
+}
+
+cudaError_t launch_flip(int* ctx_state, int slot, int prefix_len, cudaStream_t st) {
+  flip_kernel<<<1, 1, 0, st>>>(ctx_state, slot, prefix_len);
+  return cudaGetLastError();
+}
+
+}  // namespace ravel

@@ -1,0 +1,317 @@
+// Host runtime of the rolling action-expert step: owns the packed weights, the
+// double-buffered VLM context, activations, per-robot noise state and the
+// captured CUDA graph of one step, and implements the C ABI of ravel.h.
+#include <cuda_runtime.h>
+
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/ravel.h"
+#include "kernels.h"
+#include "step.h"
+
+using namespace ravel;
+
+namespace {
+
+const char* const kStatusText[] = {
+    "ok", "invalid argument", "shape outside the configuration", "out of memory", "CUDA error",
+    "no context set", "context swap already pending", "device error word raised", "device wait timed out",
+    "ravel_reset has not been called",
+};
+
+}  // namespace
+
+struct ravel_ctx {
+  StepPlan plan;               // sizes, device buffers, weights (step.h)
+  int device = 0;
+  // context double buffer
+  int active_host = 0;         // slot the device will use after pending flips
+  bool have_ctx = false;
+  bool swap_pending = false;
+  int pending_slot = 0, pending_len = 0;
+  bool any_step = false;
+  cudaEvent_t ev_step_done = nullptr, ev_ctx_ready = nullptr;
+  // rollout state
+  int batch = 0;
+  // graph
+  cudaStream_t cap_stream = nullptr;
+  cudaGraphExec_t gexec = nullptr;
+  StepIO graph_io{};
+  int graph_batch = -1;
+  int graph_kernels = 0;
+  // asynchronously mirrored device error word
+  int* err_host = nullptr;     // pinned
+  std::string last_error;
+};
+
+static ravel_status fail(ravel_t* r, ravel_status s, const std::string& msg) {
+  if (r) r->last_error = msg;
+  return s;
+}
+
+static ravel_status cuda_fail(ravel_t* r, cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  return fail(r, e == cudaErrorMemoryAllocation ? RAVEL_ENOMEM : RAVEL_ECUDA, m);
+}
+
+#define RV_CUDA(r, call, what)                         \
+  do {                                                 \
+    cudaError_t _e = (call);                           \
+    if (_e != cudaSuccess) return cuda_fail(r, _e, what); \
+  } while (0)
+
+extern "C" {
+
+const char* ravel_status_string(ravel_status s) {
+  int i = (int)s;
+  if (i < 0 || i >= (int)(sizeof(kStatusText) / sizeof(kStatusText[0]))) return "unknown status";
+  return kStatusText[i];
+}
+
+const char* ravel_last_error(const ravel_t* r) { return r ? r->last_error.c_str() : ""; }
+
+int ravel_step_kernel_count(const ravel_t* r) { return r ? r->graph_kernels : 0; }
+
+ravel_status ravel_create(const ravel_config* cfg, const ravel_weights* w, int device, ravel_t** out) {
+  if (!cfg || !w || !out) return RAVEL_EINVAL;
+  *out = nullptr;
+  std::string why;
+  if (!validate_config(*cfg, &why)) {
+    fprintf(stderr, "ravel_create: %s\n", why.c_str());
+    return RAVEL_ESHAPE;
+  }
+  ravel_t* r = new (std::nothrow) ravel_t();
+  if (!r) return RAVEL_ENOMEM;
+  r->device = device;
+  cudaError_t e = cudaSetDevice(device);
+  if (e != cudaSuccess) {
+    fprintf(stderr, "ravel_create: cudaSetDevice: %s\n", cudaGetErrorString(e));
+    delete r;
+    return RAVEL_ECUDA;
+  }
+  ravel_status s = plan_create(&r->plan, *cfg, *w, &r->last_error);
+  if (s == RAVEL_OK) {
+    if (cudaEventCreateWithFlags(&r->ev_step_done, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&r->ev_ctx_ready, cudaEventDisableTiming) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&r->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaHostAlloc((void**)&r->err_host, sizeof(int), cudaHostAllocDefault) != cudaSuccess) {
+      r->last_error = "event / stream / pinned allocation failed";
+      s = RAVEL_ECUDA;
+    } else {
+      *r->err_host = 0;
+    }
+  }
+  if (s != RAVEL_OK) {
+    fprintf(stderr, "ravel_create: %s\n", r->last_error.c_str());
+    ravel_destroy(r);
+    return s;
+  }
+  *out = r;
+  return RAVEL_OK;
+}
+
+void ravel_destroy(ravel_t* r) {
+  if (!r) return;
+  cudaSetDevice(r->device);
+  cudaDeviceSynchronize();
+  if (r->gexec) cudaGraphExecDestroy(r->gexec);
+  if (r->cap_stream) cudaStreamDestroy(r->cap_stream);
+  if (r->ev_step_done) cudaEventDestroy(r->ev_step_done);
+  if (r->ev_ctx_ready) cudaEventDestroy(r->ev_ctx_ready);
+  if (r->err_host) cudaFreeHost(r->err_host);
+  plan_destroy(&r->plan);
+  delete r;
+}
+
+ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* buffer, void* stream) {
+  if (!r || !seeds || !buffer) return fail(r, RAVEL_EINVAL, "reset: null argument");
+  if (batch < 1 || batch > r->plan.cfg.max_batch) return fail(r, RAVEL_ESHAPE, "reset: batch outside [1, max_batch]");
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  cudaStream_t st = (cudaStream_t)stream;
+  // seeds go through a synchronous copy: the host array may be freed on return
+  RV_CUDA(r, cudaStreamSynchronize(st), "reset: sync");
+  RV_CUDA(r, cudaMemcpy(r->plan.seeds, seeds, sizeof(uint64_t) * batch, cudaMemcpyHostToDevice), "reset: seeds");
+  RV_CUDA(r, launch_reset(buffer, r->plan.seeds, r->plan.counters, batch, r->plan.cfg.slots,
+                          r->plan.cfg.action_dim, st),
+          "reset kernel");
+  if (batch != r->batch) {
+    // contexts are laid out per robot: a new batch needs a new context
+    r->have_ctx = false;
+    r->swap_pending = false;
+  }
+  r->batch = batch;
+  return RAVEL_OK;
+}
+
+ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int prefix_len, void* side_stream) {
+  if (!r || !k || !v) return fail(r, RAVEL_EINVAL, "set_context: null argument");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "set_context: call ravel_reset first");
+  if (prefix_len < 1 || prefix_len > r->plan.cfg.max_prefix)
+    return fail(r, RAVEL_ESHAPE, "set_context: prefix_len outside [1, max_prefix]");
+  if (r->swap_pending) return fail(r, RAVEL_EBUSY, "set_context: previous context not yet consumed by a step");
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  cudaStream_t side = (cudaStream_t)side_stream;
+  const int target = r->have_ctx ? 1 - r->active_host : 0;
+  // the inactive slot was last read by steps already enqueued: wait for them
+  if (r->any_step) RV_CUDA(r, cudaStreamWaitEvent(side, r->ev_step_done, 0), "set_context: wait");
+  const StepPlan& p = r->plan;
+  const ravel_config& c = p.cfg;
+  const size_t es = p.esize;
+  const size_t row = (size_t)prefix_len * c.head_dim * es;        // one (l, b, g) block of the source
+  const size_t dpitch = (size_t)c.max_prefix * c.head_dim * es;  // the same block in the slot
+  const size_t per_layer_src = (size_t)r->batch * c.n_kv_heads;
+  for (int which = 0; which < 2; ++which) {
+    const char* src = (const char*)(which ? v : k);
+    char* dst = (char*)(which ? p.ctx_v[target] : p.ctx_k[target]);
+    for (int l = 0; l < c.layers; ++l) {
+      RV_CUDA(r,
+              cudaMemcpy2DAsync(dst + (size_t)l * c.max_batch * c.n_kv_heads * dpitch, dpitch,
+                                src + (size_t)l * per_layer_src * row, row, row, per_layer_src,
+                                cudaMemcpyDeviceToDevice, side),
+              "set_context: copy");
+    }
+  }
+  RV_CUDA(r, cudaEventRecord(r->ev_ctx_ready, side), "set_context: record");
+  r->swap_pending = true;
+  r->pending_slot = target;
+  r->pending_len = prefix_len;
+  r->have_ctx = true;
+  return RAVEL_OK;
+}
+
+static ravel_status check_device_errors(ravel_t* r) {
+  // the pinned mirror is written by an async copy after each step; reading a
+  // stale value only delays the report to a later call
+  const int bits = *(volatile int*)r->err_host;
+  if (bits) {
+    char buf[96];
+    snprintf(buf, sizeof buf, "device error word 0x%x", bits);
+    r->last_error = buf;
+    return (bits & ERR_TIMEOUT) ? RAVEL_ETIMEOUT : RAVEL_EDEVICE;
+  }
+  return RAVEL_OK;
+}
+
+ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                             const float* delta, float* released, float* velocity, void* stream) {
+  if (!r || !buffer || !slot_times || !delta || !released) return fail(r, RAVEL_EINVAL, "roll_step: null argument");
+  if (r->plan.cfg.fop_tokens > 0 && !obs_tokens) return fail(r, RAVEL_EINVAL, "roll_step: obs_tokens is null");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "roll_step: call ravel_reset first");
+  if (!r->have_ctx) return fail(r, RAVEL_ENOCONTEXT, "roll_step: no context set");
+  ravel_status s = check_device_errors(r);
+  if (s != RAVEL_OK) return s;
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  cudaStream_t st = (cudaStream_t)stream;
+  if (r->swap_pending) {
+    RV_CUDA(r, cudaStreamWaitEvent(st, r->ev_ctx_ready, 0), "roll_step: wait for context");
+    RV_CUDA(r, launch_flip(r->plan.ctx_state, r->pending_slot, r->pending_len, st), "roll_step: flip");
+    r->active_host = r->pending_slot;
+    r->swap_pending = false;
+  }
+  StepIO io{buffer, slot_times, obs_tokens, delta, released, velocity};
+  if (!r->gexec || r->graph_batch != r->batch || memcmp(&io, &r->graph_io, sizeof io) != 0) {
+    if (r->gexec) {
+      RV_CUDA(r, cudaStreamSynchronize(st), "roll_step: sync before re-capture");
+      cudaGraphExecDestroy(r->gexec);
+      r->gexec = nullptr;
+    }
+    cudaGraph_t graph = nullptr;
+    RV_CUDA(r, cudaStreamBeginCapture(r->cap_stream, cudaStreamCaptureModeThreadLocal), "capture begin");
+    int nk = 0;
+    cudaError_t e = enqueue_step(r->plan, r->batch, io, r->cap_stream, &nk);
+    cudaError_t e2 = cudaStreamEndCapture(r->cap_stream, &graph);
+    if (e != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      return cuda_fail(r, e, "roll_step: enqueue");
+    }
+    RV_CUDA(r, e2, "capture end");
+    e = cudaGraphInstantiateWithFlags(&r->gexec, graph, 0);
+    cudaGraphDestroy(graph);
+    RV_CUDA(r, e, "graph instantiate");
+    r->graph_io = io;
+    r->graph_batch = r->batch;
+    r->graph_kernels = nk;
+  }
+  RV_CUDA(r, cudaGraphLaunch(r->gexec, st), "graph launch");
+  RV_CUDA(r, cudaEventRecord(r->ev_step_done, st), "record step");
+  RV_CUDA(r, cudaMemcpyAsync(r->err_host, r->plan.err, sizeof(int), cudaMemcpyDeviceToHost, st), "error mirror");
+  r->any_step = true;
+  return RAVEL_OK;
+}
+
+const char* ravel_kernel_kind_name(int kind) { return kernel_kind_name(kind); }
+
+ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                                const float* delta, float* released, float* velocity, void* stream,
+                                float* launch_ms, int* launch_kind, int cap, int* n_launches) {
+  if (!r || !buffer || !slot_times || !delta || !released || !launch_ms || !launch_kind || !n_launches || cap < 0)
+    return fail(r, RAVEL_EINVAL, "profile_step: null argument");
+  if (r->plan.cfg.fop_tokens > 0 && !obs_tokens) return fail(r, RAVEL_EINVAL, "profile_step: obs_tokens is null");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "profile_step: call ravel_reset first");
+  if (!r->have_ctx) return fail(r, RAVEL_ENOCONTEXT, "profile_step: no context set");
+  ravel_status s = check_device_errors(r);
+  if (s != RAVEL_OK) return s;
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  cudaStream_t st = (cudaStream_t)stream;
+  if (r->swap_pending) {
+    RV_CUDA(r, cudaStreamWaitEvent(st, r->ev_ctx_ready, 0), "profile_step: wait for context");
+    RV_CUDA(r, launch_flip(r->plan.ctx_state, r->pending_slot, r->pending_len, st), "profile_step: flip");
+    r->active_host = r->pending_slot;
+    r->swap_pending = false;
+  }
+  // hold the stream for a few ms so that every launch below is queued before
+  // the first one starts: the events then time the kernels, not the host
+  RV_CUDA(r, launch_delay(5000000ull, st), "profile_step: delay");
+  cudaEvent_t start;
+  RV_CUDA(r, cudaEventCreate(&start), "profile_step: event");
+  LaunchTrace tr;
+  cudaError_t e = cudaEventRecord(start, st);
+  int nk = 0;
+  StepIO io{buffer, slot_times, obs_tokens, delta, released, velocity};
+  if (e == cudaSuccess) e = enqueue_step(r->plan, r->batch, io, st, &nk, &tr);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  int n = 0;
+  cudaEvent_t prev = start;
+  for (size_t i = 0; i < tr.events.size() && e == cudaSuccess; ++i) {
+    float ms = 0.f;
+    e = cudaEventElapsedTime(&ms, prev, tr.events[i]);
+    if (n < cap) {
+      launch_ms[n] = ms;
+      launch_kind[n] = tr.kinds[i];
+    }
+    ++n;
+    prev = tr.events[i];
+  }
+  for (cudaEvent_t ev : tr.events) cudaEventDestroy(ev);
+  cudaEventDestroy(start);
+  RV_CUDA(r, e, "profile_step");
+  *n_launches = n;
+  r->any_step = true;
+  RV_CUDA(r, cudaEventRecord(r->ev_step_done, st), "record step");
+  return RAVEL_OK;
+}
+
+ravel_status ravel_get_state(ravel_t* r, uint64_t* counters) {
+  if (!r || !counters) return fail(r, RAVEL_EINVAL, "get_state: null argument");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "get_state: call ravel_reset first");
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  RV_CUDA(r, cudaDeviceSynchronize(), "get_state: sync");
+  RV_CUDA(r, cudaMemcpy(counters, r->plan.counters, sizeof(uint64_t) * r->batch, cudaMemcpyDeviceToHost),
+          "get_state: copy");
+  return check_device_errors(r);
+}
+
+ravel_status ravel_set_state(ravel_t* r, const uint64_t* counters) {
+  if (!r || !counters) return fail(r, RAVEL_EINVAL, "set_state: null argument");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "set_state: call ravel_reset first");
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  RV_CUDA(r, cudaDeviceSynchronize(), "set_state: sync");
+  RV_CUDA(r, cudaMemcpy(r->plan.counters, counters, sizeof(uint64_t) * r->batch, cudaMemcpyHostToDevice),
+          "set_state: copy");
+  return RAVEL_OK;
+}
+
+}  // extern "C"

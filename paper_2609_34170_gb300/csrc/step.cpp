@@ -1,0 +1,264 @@
+// Step plan: allocation, weight packing and the kernel sequence of one
+// rolling action-expert step.
+#include "step.h"
+
+#include <cstdio>
+#include <algorithm>
+#include <cstring>
+
+namespace ravel {
+
+bool validate_config(const ravel_config& c, std::string* why) {
+  auto bad = [&](const char* m) {
+    *why = m;
+    return false;
+  };
+  if (c.layers < 1 || c.width < 4 || c.width % 2) return bad("layers >= 1 and an even width >= 4 are required");
+  if (c.n_q_heads < 1 || c.n_kv_heads < 1 || c.n_q_heads % c.n_kv_heads)
+    return bad("n_q_heads must be a positive multiple of n_kv_heads");
+  if (c.head_dim < 8 || c.head_dim > 256 || c.head_dim % 8) return bad("head_dim must be a multiple of 8 in [8, 256]");
+  if (c.mlp_dim < 64 || c.mlp_dim % 64) return bad("mlp_dim must be a positive multiple of 64");
+  if (c.slots < 1 || c.action_dim < 1 || (long)c.slots * c.action_dim > 16384)
+    return bad("slots >= 1, action_dim >= 1 and slots * action_dim <= 16384 are required");
+  if (c.max_prefix < 1 || c.fop_tokens < 0 || c.max_batch < 1) return bad("max_prefix, max_batch >= 1, fop_tokens >= 0");
+  if (c.dtype != RAVEL_FP32 && c.dtype != RAVEL_BF16) return bad("dtype must be RAVEL_FP32 or RAVEL_BF16");
+  if (c.mask_mode != RAVEL_MASK_FULL && c.mask_mode != RAVEL_MASK_SLOT_ISOLATED) return bad("unknown mask_mode");
+  return true;
+}
+
+static cudaError_t dalloc(StepPlan* p, void** ptr, size_t bytes) {
+  *ptr = nullptr;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(ptr, bytes);
+  if (e == cudaSuccess) {
+    p->allocs.push_back(*ptr);
+    e = cudaMemset(*ptr, 0, bytes);
+  }
+  return e;
+}
+
+void plan_destroy(StepPlan* p) {
+  for (void* a : p->allocs) cudaFree(a);
+  p->allocs.clear();
+}
+
+namespace {
+
+struct Packer {
+  StepPlan* p;
+  const ravel_weights* w;
+  float* staging;
+  cudaError_t err = cudaSuccess;
+
+  // device fp32 view of `n` floats at src (host or device)
+  const float* view(const float* src, size_t n) {
+    if (w->on_device) return src;
+    if (err == cudaSuccess) err = cudaMemcpy(staging, src, n * sizeof(float), cudaMemcpyHostToDevice);
+    return staging;
+  }
+  // dst = src^T ([K, N] -> [N, K]) in the plan's dtype
+  void transpose(const float* src, int K, int N, void* dst, int interleave = 0, int off = 0) {
+    const float* s = view(src, (size_t)K * N);
+    if (err == cudaSuccess) err = launch_pack_transpose(s, K, N, dst, p->dt, interleave, off, 0);
+    if (err == cudaSuccess) err = cudaDeviceSynchronize();
+  }
+  void copy_f32(const float* src, size_t n, float* dst) {
+    if (err != cudaSuccess) return;
+    err = cudaMemcpy(dst, src, n * sizeof(float), w->on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice);
+  }
+};
+
+}  // namespace
+
+ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights& w, std::string* errs) {
+  const ravel_weights* wp = &w;
+  const float* req[] = {w.t_w1, w.t_b1, w.t_w2, w.t_b2, w.d_w1, w.d_b1, w.d_w2, w.d_b2, w.mod_w, w.mod_b,
+                        w.in_w, w.in_b, w.fop_gamma, w.w_qkv, w.w_o, w.w_gate, w.w_up, w.w_down, w.out_w, w.out_b};
+  for (const float* q : req)
+    if (!q) {
+      *errs = "a weight pointer is null";
+      return RAVEL_EINVAL;
+    }
+  p->cfg = c;
+  p->dt = c.dtype == RAVEL_BF16 ? DT_BF16 : DT_F32;
+  p->esize = c.dtype == RAVEL_BF16 ? 2 : 4;
+  const size_t es = p->esize;
+  const int D = c.width, L = c.layers, H = c.slots, A = c.action_dim, F = c.fop_tokens, Fm = c.mlp_dim;
+  const int Bm = c.max_batch;
+  p->nqkv = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
+  p->qdim = c.n_q_heads * c.head_dim;
+  p->mod_dim = 4 * L * D + 2 * D;
+  const size_t DD = (size_t)D * D;
+
+  cudaError_t e = init_simt_kernels();
+#define AL(ptr, bytes)                                      \
+  do {                                                      \
+    if (e == cudaSuccess) e = dalloc(p, (void**)&(ptr), (bytes)); \
+  } while (0)
+  AL(p->t_w1, DD * es); AL(p->t_w2, DD * es); AL(p->d_w1, DD * es); AL(p->d_w2, DD * es);
+  AL(p->mod_w, (size_t)p->mod_dim * D * es);
+  AL(p->w_qkv, (size_t)L * p->nqkv * D * es);
+  AL(p->w_o, (size_t)L * D * p->qdim * es);
+  AL(p->w_gu, (size_t)L * 2 * Fm * D * es);
+  AL(p->w_down, (size_t)L * D * Fm * es);
+  AL(p->out_w, (size_t)A * D * es);
+  AL(p->t_b1, D * 4); AL(p->t_b2, D * 4); AL(p->d_b1, D * 4); AL(p->d_b2, D * 4);
+  AL(p->mod_b, (size_t)p->mod_dim * 4);
+  AL(p->in_w, (size_t)A * D * 4); AL(p->in_b, D * 4);
+  AL(p->fop_gamma, (size_t)L * D * 4);
+  AL(p->out_b, A * 4);
+  const size_t ctx_bytes = (size_t)L * Bm * c.n_kv_heads * c.max_prefix * c.head_dim * es;
+  for (int s = 0; s < 2; ++s) {
+    AL(p->ctx_k[s], ctx_bytes);
+    AL(p->ctx_v[s], ctx_bytes);
+  }
+  AL(p->ctx_state, 2 * sizeof(int));
+  const size_t rows_c = (size_t)H + Bm, rows_a = (size_t)Bm * H, rows_y = (size_t)Bm * (H + F);
+  AL(p->E, rows_c * D * es); AL(p->H1, rows_c * D * es); AL(p->HC, rows_c * D * es);
+  AL(p->modv, rows_c * p->mod_dim * 4);
+  AL(p->x, rows_a * D * 4);
+  AL(p->Y, rows_y * D * es);
+  AL(p->QKV, rows_y * p->nqkv * es);
+  AL(p->O, rows_a * p->qdim * es);
+  AL(p->GU, rows_a * 2 * Fm * 4);
+  AL(p->Hm, rows_a * Fm * es);
+  AL(p->V, rows_a * A * 4);
+  AL(p->seeds, Bm * sizeof(uint64_t));
+  AL(p->counters, Bm * sizeof(uint64_t));
+  AL(p->err, sizeof(int));
+#undef AL
+  if (e != cudaSuccess) {
+    *errs = std::string("allocation: ") + cudaGetErrorString(e);
+    plan_destroy(p);
+    return e == cudaErrorMemoryAllocation ? RAVEL_ENOMEM : RAVEL_ECUDA;
+  }
+
+  // staging for host weights: the largest single tensor slice packed at once
+  size_t stage = (size_t)D * p->mod_dim;
+  stage = std::max(stage, (size_t)D * p->nqkv);
+  stage = std::max(stage, (size_t)p->qdim * D);
+  stage = std::max(stage, (size_t)D * Fm);
+  float* staging = nullptr;
+  if (!w.on_device) {
+    e = cudaMalloc((void**)&staging, stage * sizeof(float));
+    if (e != cudaSuccess) {
+      *errs = "weight staging allocation failed";
+      plan_destroy(p);
+      return RAVEL_ENOMEM;
+    }
+  }
+  Packer pk{p, wp, staging};
+  pk.transpose(w.t_w1, D, D, p->t_w1);
+  pk.transpose(w.t_w2, D, D, p->t_w2);
+  pk.transpose(w.d_w1, D, D, p->d_w1);
+  pk.transpose(w.d_w2, D, D, p->d_w2);
+  pk.transpose(w.mod_w, D, p->mod_dim, p->mod_w);
+  for (int l = 0; l < L; ++l) {
+    pk.transpose(w.w_qkv + (size_t)l * D * p->nqkv, D, p->nqkv, (char*)p->w_qkv + (size_t)l * p->nqkv * D * es);
+    pk.transpose(w.w_o + (size_t)l * p->qdim * D, p->qdim, D, (char*)p->w_o + (size_t)l * D * p->qdim * es);
+    char* gu = (char*)p->w_gu + (size_t)l * 2 * Fm * D * es;
+    pk.transpose(w.w_gate + (size_t)l * D * Fm, D, Fm, gu, 1, 0);
+    pk.transpose(w.w_up + (size_t)l * D * Fm, D, Fm, gu, 1, 64);
+    pk.transpose(w.w_down + (size_t)l * Fm * D, Fm, D, (char*)p->w_down + (size_t)l * D * Fm * es);
+  }
+  pk.transpose(w.out_w, D, A, p->out_w);
+  pk.copy_f32(w.t_b1, D, p->t_b1);
+  pk.copy_f32(w.t_b2, D, p->t_b2);
+  pk.copy_f32(w.d_b1, D, p->d_b1);
+  pk.copy_f32(w.d_b2, D, p->d_b2);
+  pk.copy_f32(w.mod_b, p->mod_dim, p->mod_b);
+  pk.copy_f32(w.in_w, (size_t)A * D, p->in_w);
+  pk.copy_f32(w.in_b, D, p->in_b);
+  pk.copy_f32(w.fop_gamma, (size_t)L * D, p->fop_gamma);
+  pk.copy_f32(w.out_b, A, p->out_b);
+  if (pk.err == cudaSuccess) pk.err = cudaDeviceSynchronize();
+  if (staging) cudaFree(staging);
+  if (pk.err != cudaSuccess) {
+    *errs = std::string("weight packing: ") + cudaGetErrorString(pk.err);
+    plan_destroy(p);
+    return RAVEL_ECUDA;
+  }
+  return RAVEL_OK;
+}
+
+// ---------------------------------------------------------------------------- the step
+
+const char* kernel_kind_name(int k) {
+  static const char* const names[KK_COUNT] = {"embed", "gemm_cond", "gemm_mod", "in_proj", "norm", "gemm_qkv",
+                                              "attention", "gemm_o", "gemm_gate_up", "geglu", "gemm_down",
+                                              "gemm_out", "tail"};
+  return (k >= 0 && k < KK_COUNT) ? names[k] : "unknown";
+}
+
+cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_t st, int* n_kernels,
+                         LaunchTrace* trace) {
+  const ravel_config& c = p.cfg;
+  const int D = c.width, L = c.layers, H = c.slots, A = c.action_dim, F = c.fop_tokens, Fm = c.mlp_dim;
+  const size_t es = p.esize;
+  const Dtype dt = p.dt;
+  int nk = 0;
+  cudaError_t e = cudaSuccess;
+  auto mark = [&](int kind) {
+    if (!trace || e != cudaSuccess) return;
+    cudaEvent_t ev;
+    e = cudaEventCreate(&ev);
+    if (e != cudaSuccess) return;
+    trace->events.push_back(ev);
+    trace->kinds.push_back(kind);
+    e = cudaEventRecord(ev, st);
+  };
+#define RUN(kind, call)                 \
+  do {                                  \
+    if (e == cudaSuccess) {             \
+      e = (call);                       \
+      ++nk;                             \
+      mark(kind);                       \
+    }                                   \
+  } while (0)
+  auto gemm = [&](const void* Aop, int lda, const void* W, int M, int N, int K, Epi epi, void* out, int ldo,
+                  Dtype out_dt, const float* bias) {
+    GemmArgs g{Aop, lda, W, K, M, N, K, epi, out, ldo, out_dt, bias};
+    return launch_gemm_simt(g, dt, st);
+  };
+  auto rowp = [&](const void* base, size_t row, size_t ld) { return (const void*)((const char*)base + row * ld * es); };
+
+  // conditioning: embeddings, the two MLPs, modulation (App. A.1)
+  RUN(KK_EMBED, launch_embed(io.slot_times, H, io.delta, B, D, p.E, dt, st));
+  RUN(KK_GEMM_COND, gemm(p.E, D, p.t_w1, H, D, D, EPI_STORE_SILU, p.H1, D, dt, p.t_b1));
+  RUN(KK_GEMM_COND, gemm(rowp(p.E, H, D), D, p.d_w1, B, D, D, EPI_STORE_SILU, (void*)rowp(p.H1, H, D), D, dt, p.d_b1));
+  RUN(KK_GEMM_COND, gemm(p.H1, D, p.t_w2, H, D, D, EPI_STORE, p.HC, D, dt, p.t_b2));
+  RUN(KK_GEMM_COND, gemm(rowp(p.H1, H, D), D, p.d_w2, B, D, D, EPI_STORE, (void*)rowp(p.HC, H, D), D, dt, p.d_b2));
+  RUN(KK_GEMM_MOD, gemm(p.HC, D, p.mod_w, H + B, p.mod_dim, D, EPI_STORE, p.modv, p.mod_dim, DT_F32, nullptr));
+  // residual stream
+  RUN(KK_IN_PROJ, launch_in_proj(io.buffer, B * H, A, D, p.in_w, p.in_b, p.x, st));
+  const int BH = B * H, BY = B * (H + (io.obs ? F : 0));
+  for (int l = 0; l < L; ++l) {
+    NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, io.obs, F, p.fop_gamma + (size_t)l * D, p.Y};
+    RUN(KK_NORM, launch_ada_norm(n1, dt, st));
+    RUN(KK_GEMM_QKV, gemm(p.Y, D, (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es, BY, p.nqkv, D, EPI_STORE, p.QKV, p.nqkv,
+             dt, nullptr));
+    AttnArgs at{p.QKV, p.nqkv, p.ctx_k[0], p.ctx_k[1], p.ctx_v[0], p.ctx_v[1], p.ctx_state, l, c.max_batch,
+                c.max_prefix, B, H, io.obs ? F : 0, c.n_q_heads, c.n_kv_heads, c.head_dim, c.mask_mode, p.O, p.qdim,
+                p.err};
+    RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
+    RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x, D,
+             DT_F32, nullptr));
+    NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y};
+    RUN(KK_NORM, launch_ada_norm(n2, dt, st));
+    RUN(KK_GEMM_GATE_UP, gemm(p.Y, D, (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es, BH, 2 * Fm, D, EPI_STORE, p.GU, 2 * Fm,
+             DT_F32, nullptr));
+    RUN(KK_GEGLU, launch_geglu(p.GU, BH, Fm, p.Hm, dt, st));
+    RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D, DT_F32,
+             nullptr));
+  }
+  NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y};
+  RUN(KK_NORM, launch_ada_norm(nf, dt, st));
+  RUN(KK_GEMM_OUT, gemm(p.Y, D, p.out_w, BH, A, D, EPI_STORE, p.V, A, DT_F32, p.out_b));
+  TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A};
+  RUN(KK_TAIL, launch_tail(ta, st));
+#undef RUN
+  if (n_kernels) *n_kernels = nk;
+  return e;
+}
+
+}  // namespace ravel

@@ -1,0 +1,80 @@
+// The step plan: every device buffer of one handle and the kernel sequence of
+// one rolling step.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/ravel.h"
+#include "kernels.h"
+
+namespace ravel {
+
+// Caller-owned pointers of one ravel_roll_step call (captured into the graph).
+struct StepIO {
+  float* buffer;
+  const float* slot_times;
+  const void* obs;
+  const float* delta;
+  float* released;
+  float* velocity;
+};
+
+struct StepPlan {
+  ravel_config cfg{};
+  Dtype dt = DT_F32;
+  size_t esize = 4;
+  int nqkv = 0, qdim = 0, mod_dim = 0;
+  // packed weights, K-major [out][in] in dtype; biases / gains fp32
+  void *t_w1 = nullptr, *t_w2 = nullptr, *d_w1 = nullptr, *d_w2 = nullptr, *mod_w = nullptr;
+  void *w_qkv = nullptr, *w_o = nullptr, *w_gu = nullptr, *w_down = nullptr, *out_w = nullptr;
+  float *t_b1 = nullptr, *t_b2 = nullptr, *d_b1 = nullptr, *d_b2 = nullptr, *mod_b = nullptr;
+  float *in_w = nullptr, *in_b = nullptr, *fop_gamma = nullptr, *out_b = nullptr;
+  // VLM context double buffer [2] x [L][Bmax][Hkv][Pmax][hd] and its device state {active, len}
+  void* ctx_k[2] = {nullptr, nullptr};
+  void* ctx_v[2] = {nullptr, nullptr};
+  int* ctx_state = nullptr;
+  // activations
+  void* E = nullptr;      // [H+Bmax][D]  sinusoidal embeddings (times, then offsets)
+  void* H1 = nullptr;     // [H+Bmax][D]  first MLP layer (SiLU)
+  void* HC = nullptr;     // [H+Bmax][D]  MLP outputs h_t, h_delta
+  float* modv = nullptr;  // [H+Bmax][mod_dim]  h @ W_mod (bias added in the norms)
+  float* x = nullptr;     // [Bmax*H][D]  residual stream
+  void* Y = nullptr;      // [Bmax*(H+F)][D]  normed rows (actions, then FOP tokens)
+  void* QKV = nullptr;    // [Bmax*(H+F)][nqkv]
+  void* O = nullptr;      // [Bmax*H][Hq*hd]
+  float* GU = nullptr;    // [Bmax*H][2Fm]  interleaved gate/up (SIMT path)
+  void* Hm = nullptr;     // [Bmax*H][Fm]
+  float* V = nullptr;     // [Bmax*H][A]   velocity
+  uint64_t* seeds = nullptr;
+  uint64_t* counters = nullptr;
+  int* err = nullptr;
+  std::vector<void*> allocs;
+};
+
+bool validate_config(const ravel_config& c, std::string* why);
+ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights& w, std::string* err);
+void plan_destroy(StepPlan* p);
+
+// Kernel kinds of one step (per-launch profiling labels).
+enum KernelKind {
+  KK_EMBED = 0, KK_GEMM_COND, KK_GEMM_MOD, KK_IN_PROJ, KK_NORM, KK_GEMM_QKV, KK_ATTENTION, KK_GEMM_O,
+  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COUNT
+};
+const char* kernel_kind_name(int k);
+
+// Optional per-launch trace: an event recorded after every launch.
+struct LaunchTrace {
+  std::vector<cudaEvent_t> events;   // events[i] recorded after launch i
+  std::vector<int> kinds;
+};
+
+// Enqueue one rolling step for `B` robots on `st` (no synchronisation, graph
+// capture safe when trace == nullptr).  *n_kernels receives the number of
+// kernel launches.
+cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_t st, int* n_kernels,
+                         LaunchTrace* trace = nullptr);
+
+}  // namespace ravel
