@@ -169,6 +169,23 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
                                 const float* delta, float* released, float* velocity, void* stream,
                                 float* launch_ms, int* launch_kind, int cap, int* n_launches);
 
+/* One projection GEMM of the kind the step runs, through the step's own
+ * dispatcher (tcgen05 tensor cores for a RAVEL_BF16 handle whose operands
+ * are 16-byte aligned with K, lda, ldw multiples of 8; the fp32 SIMT kernel
+ * otherwise): a building block of ravel_roll_step exposed for kernel tests.
+ *   X   device [M, lda] activations of the handle's dtype, first K columns used
+ *   W   device [N, ldw] weights (K-major: row n holds output feature n)
+ *   epi 0: out = X W^T + bias            1: out = SiLU(X W^T + bias)
+ *       2: out += X W^T + bias (float32 out)
+ *       3: GeGLU (bf16 handle, N % 128 == 0): W rows in 128-row blocks of 64
+ *          gate rows then the 64 matching up rows; out[m][f] =
+ *          gelu_tanh(gate) * up for f < N/2 (bias ignored)
+ *   out device [M, ldo], out_dtype RAVEL_FP32 or RAVEL_BF16; bias device [N] or NULL
+ * Enqueued on `stream`; uses the handle's split-K workspace, so it must not
+ * overlap another call on the same handle. */
+ravel_status ravel_gemm(ravel_t* r, const void* X, int M, int K, int lda, const void* W, int N, int ldw, int epi,
+                        void* out, int ldo, int out_dtype, const float* bias, void* stream);
+
 /* Name of a kernel kind id of ravel_profile_step ("gemm_down", ...). */
 const char* ravel_kernel_kind_name(int kind);
 

@@ -69,6 +69,7 @@ def load(path: str | None = None):
         "ravel_step_kernel_count": (i, [vp]),
         "ravel_profile_step": (i, [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i, vp]),
         "ravel_kernel_kind_name": (C.c_char_p, [i]),
+        "ravel_gemm": (i, [vp, vp, i, i, i, vp, i, i, i, vp, i, i, vp, vp]),
         "ravel_status_string": (C.c_char_p, [i]),
         "ravel_last_error": (C.c_char_p, [vp]),
     }
@@ -175,6 +176,18 @@ def ravel_profile_step(h, buffer, slot_times, obs_tokens, delta, released, veloc
         _stream_ptr(stream), ms.ctypes.data, kinds.ctypes.data, cap, C.byref(n)), "ravel_profile_step")
     k = min(n.value, cap)
     return [(load().ravel_kernel_kind_name(int(kinds[i])).decode(), float(ms[i])) for i in range(k)]
+
+
+def ravel_gemm(h, X, W, epi: int, out, bias=None, K: int | None = None, stream=None):
+    """out (op)= X[:, :K] @ W[:, :K]^T (+ bias) on the device; see ravel.h."""
+    import torch
+    M, lda = X.shape
+    N, ldw = W.shape
+    K = lda if K is None else K
+    od = 1 if out.dtype == torch.bfloat16 else 0
+    _check(h, load().ravel_gemm(h, _dptr(X, name="X"), M, K, lda, _dptr(W, name="W"), N, ldw, epi,
+                                _dptr(out, name="out"), out.shape[1], od, _dptr(bias, torch.float32, "bias"),
+                                _stream_ptr(stream)), "ravel_gemm")
 
 
 def ravel_get_state(h, batch: int) -> np.ndarray:

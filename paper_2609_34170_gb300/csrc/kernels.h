@@ -34,7 +34,7 @@ cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int
                          cudaStream_t st);
 
 // ---- generic projection GEMM: out[m][n] = sum_k A[m][k] W[n][k] (W K-major) ----
-enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2 };
+enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2, EPI_GEGLU = 3 };
 struct GemmArgs {
   const void* A; int lda;       // [M][K] activations of dtype dt
   const void* W; int ldw;       // [N][K] weights of dtype dt
@@ -45,6 +45,18 @@ struct GemmArgs {
   const float* bias;            // [N] or null
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
+
+// tcgen05 / TMEM / TMA path (bf16 operands only).  EPI_GEGLU: W rows come in
+// 128-row blocks of 64 gate rows then the 64 matching up rows; out is bf16
+// [M][N/2] with out[m][f] = gelu_tanh(gate_f) * up_f.
+struct TcWorkspace {
+  float* ws; size_t ws_bytes;   // split-K partial tiles
+  int* counters; int n_counters;   // per-tile arrival counters, zero between launches
+  int* err;                     // device error word
+};
+cudaError_t init_tc_gemm();
+bool tc_gemm_supported(const GemmArgs& g);
+cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st);
 
 // ---- adaRMSNorm rows ---------------------------------------------------------
 // Action rows r < B*H (b = r / H, j = r % H):

@@ -244,6 +244,22 @@ ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times,
 
 const char* ravel_kernel_kind_name(int kind) { return kernel_kind_name(kind); }
 
+ravel_status ravel_gemm(ravel_t* r, const void* X, int M, int K, int lda, const void* W, int N, int ldw, int epi,
+                        void* out, int ldo, int out_dtype, const float* bias, void* stream) {
+  if (!r || !X || !W || !out) return fail(r, RAVEL_EINVAL, "gemm: null argument");
+  if (M < 0 || N < 1 || K < 1 || lda < K || ldw < K || epi < 0 || epi > 3 || (out_dtype != 0 && out_dtype != 1))
+    return fail(r, RAVEL_EINVAL, "gemm: bad sizes or mode");
+  if (epi == EPI_GEGLU && (r->plan.dt != DT_BF16 || N % 128 || out_dtype != 1 || ldo < N / 2))
+    return fail(r, RAVEL_EINVAL, "gemm: GeGLU needs bf16, N % 128 == 0 and a bf16 output");
+  if (epi != EPI_GEGLU && ldo < N) return fail(r, RAVEL_EINVAL, "gemm: ldo < N");
+  if (epi == EPI_ADD_F32 && out_dtype != 0) return fail(r, RAVEL_EINVAL, "gemm: accumulate needs a float32 output");
+  if (M == 0) return RAVEL_OK;
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  GemmArgs g{X, lda, W, ldw, M, N, K, (Epi)epi, out, ldo, out_dtype ? DT_BF16 : DT_F32, bias};
+  RV_CUDA(r, run_gemm(r->plan, g, (cudaStream_t)stream), "gemm");
+  return RAVEL_OK;
+}
+
 ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
                                 const float* delta, float* released, float* velocity, void* stream,
                                 float* launch_ms, int* launch_kind, int cap, int* n_launches) {

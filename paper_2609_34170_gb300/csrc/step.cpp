@@ -123,10 +123,24 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->GU, rows_a * 2 * Fm * 4);
   AL(p->Hm, rows_a * Fm * es);
   AL(p->V, rows_a * A * 4);
+  p->tcws.ws_bytes = (size_t)24 << 20;
+  p->tcws.n_counters = 4096;
+  AL(p->tcws.ws, p->tcws.ws_bytes);
+  AL(p->tcws.counters, p->tcws.n_counters * sizeof(int));
   AL(p->seeds, Bm * sizeof(uint64_t));
   AL(p->counters, Bm * sizeof(uint64_t));
   AL(p->err, sizeof(int));
 #undef AL
+  p->tcws.err = p->err;
+  if (e == cudaSuccess) {
+    int dev = 0;
+    e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  if (e == cudaSuccess && p->dt == DT_BF16) {
+    e = init_tc_gemm();
+    p->use_tc = (e == cudaSuccess);
+  }
   if (e != cudaSuccess) {
     *errs = std::string("allocation: ") + cudaGetErrorString(e);
     plan_destroy(p);
@@ -183,6 +197,12 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
 
 // ---------------------------------------------------------------------------- the step
 
+cudaError_t run_gemm(const StepPlan& p, const GemmArgs& g, cudaStream_t st) {
+  if (p.use_tc && tc_gemm_supported(g)) return launch_gemm_tc(g, p.tcws, p.num_sms, st);
+  if (g.epi == EPI_GEGLU) return cudaErrorNotSupported;
+  return launch_gemm_simt(g, p.dt, st);
+}
+
 const char* kernel_kind_name(int k) {
   static const char* const names[KK_COUNT] = {"embed", "gemm_cond", "gemm_mod", "in_proj", "norm", "gemm_qkv",
                                               "attention", "gemm_o", "gemm_gate_up", "geglu", "gemm_down",
@@ -218,7 +238,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   auto gemm = [&](const void* Aop, int lda, const void* W, int M, int N, int K, Epi epi, void* out, int ldo,
                   Dtype out_dt, const float* bias) {
     GemmArgs g{Aop, lda, W, K, M, N, K, epi, out, ldo, out_dt, bias};
-    return launch_gemm_simt(g, dt, st);
+    return run_gemm(p, g, st);
   };
   auto rowp = [&](const void* base, size_t row, size_t ld) { return (const void*)((const char*)base + row * ld * es); };
 
@@ -245,9 +265,14 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
              DT_F32, nullptr));
     NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y};
     RUN(KK_NORM, launch_ada_norm(n2, dt, st));
-    RUN(KK_GEMM_GATE_UP, gemm(p.Y, D, (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es, BH, 2 * Fm, D, EPI_STORE, p.GU, 2 * Fm,
-             DT_F32, nullptr));
-    RUN(KK_GEGLU, launch_geglu(p.GU, BH, Fm, p.Hm, dt, st));
+    const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
+    GemmArgs gu{p.Y, D, wgu, D, BH, 2 * Fm, D, EPI_GEGLU, p.Hm, Fm, dt, nullptr};
+    if (p.use_tc && tc_gemm_supported(gu)) {
+      RUN(KK_GEMM_GATE_UP, launch_gemm_tc(gu, p.tcws, p.num_sms, st));   // GeGLU fused in the epilogue
+    } else {
+      RUN(KK_GEMM_GATE_UP, gemm(p.Y, D, wgu, BH, 2 * Fm, D, EPI_STORE, p.GU, 2 * Fm, DT_F32, nullptr));
+      RUN(KK_GEGLU, launch_geglu(p.GU, BH, Fm, p.Hm, dt, st));
+    }
     RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D, DT_F32,
              nullptr));
   }

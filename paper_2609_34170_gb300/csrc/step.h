@@ -48,6 +48,9 @@ struct StepPlan {
   float* GU = nullptr;    // [Bmax*H][2Fm]  interleaved gate/up (SIMT path)
   void* Hm = nullptr;     // [Bmax*H][Fm]
   float* V = nullptr;     // [Bmax*H][A]   velocity
+  TcWorkspace tcws{};       // split-K workspace of the tensor-core GEMM
+  int num_sms = 0;
+  bool use_tc = false;      // bf16 projections on tcgen05
   uint64_t* seeds = nullptr;
   uint64_t* counters = nullptr;
   int* err = nullptr;
@@ -70,6 +73,10 @@ struct LaunchTrace {
   std::vector<cudaEvent_t> events;   // events[i] recorded after launch i
   std::vector<int> kinds;
 };
+
+// One projection GEMM through the step's dispatcher (tcgen05 for bf16 when
+// the shapes allow, SIMT otherwise).
+cudaError_t run_gemm(const StepPlan& p, const GemmArgs& g, cudaStream_t st);
 
 // Enqueue one rolling step for `B` robots on `st` (no synchronisation, graph
 // capture safe when trace == nullptr).  *n_kernels receives the number of
