@@ -186,6 +186,30 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
 ravel_status ravel_gemm(ravel_t* r, const void* X, int M, int K, int lda, const void* W, int N, int ldw, int epi,
                         void* out, int ldo, int out_dtype, const float* bias, void* stream);
 
+/* Allocation-free variant of ravel_gemm for callers that cannot allocate
+ * device memory (and so cannot create a handle): for example code running in
+ * another runtime's memory pool with raw allocation disabled, plugin hosts
+ * that forbid cudaMalloc, or control loops that must not touch the allocator
+ * after start-up.  The paper has no counterpart; this is a property of the
+ * library, not of the method.
+ * Same operation, arguments and epilogues as ravel_gemm, bf16 operands only
+ * (X and W bf16, 16-byte aligned, K, lda, ldw multiples of 8), on the
+ * current CUDA device.  It calls no cudaMalloc / cudaFree: its split-K
+ * scratch is one fixed device array inside the library (8 MiB of partial
+ * sums plus tile counters), held by every GPU that loads the library until
+ * the process exits.  The split plan is chosen to fit that array.  M, N, K
+ * above RAVEL_NOALLOC_MAX_M / _N / _K return RAVEL_ESHAPE; bad pointers or
+ * modes RAVEL_EINVAL.  The first call on a device resolves the array's device
+ * address (and the kernel set-up) for that device; make that first call
+ * before any stream capture.  Each call clears the scratch's counters on
+ * `stream` before the GEMM; every call shares the array, so calls that
+ * overlap on the GPU race and must be serialised by the caller. */
+#define RAVEL_NOALLOC_MAX_M 32768
+#define RAVEL_NOALLOC_MAX_N 262144
+#define RAVEL_NOALLOC_MAX_K 65536
+ravel_status ravel_gemm_noalloc(const void* X, int M, int K, int lda, const void* W, int N, int ldw, int epi,
+                                void* out, int ldo, int out_dtype, const float* bias, void* stream);
+
 /* Name of a kernel kind id of ravel_profile_step ("gemm_down", ...). */
 const char* ravel_kernel_kind_name(int kind);
 

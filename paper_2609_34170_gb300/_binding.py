@@ -70,6 +70,7 @@ def load(path: str | None = None):
         "ravel_profile_step": (i, [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i, vp]),
         "ravel_kernel_kind_name": (C.c_char_p, [i]),
         "ravel_gemm": (i, [vp, vp, i, i, i, vp, i, i, i, vp, i, i, vp, vp]),
+        "ravel_gemm_noalloc": (i, [vp, i, i, i, vp, i, i, i, vp, i, i, vp, vp]),
         "ravel_status_string": (C.c_char_p, [i]),
         "ravel_last_error": (C.c_char_p, [vp]),
     }
@@ -188,6 +189,19 @@ def ravel_gemm(h, X, W, epi: int, out, bias=None, K: int | None = None, stream=N
     _check(h, load().ravel_gemm(h, _dptr(X, name="X"), M, K, lda, _dptr(W, name="W"), N, ldw, epi,
                                 _dptr(out, name="out"), out.shape[1], od, _dptr(bias, torch.float32, "bias"),
                                 _stream_ptr(stream)), "ravel_gemm")
+
+
+def ravel_gemm_noalloc(X, W, epi: int, out, bias=None, K: int | None = None, stream=None):
+    """ravel_gemm without a handle and without device allocation (see ravel.h)."""
+    import torch
+    M, lda = X.shape
+    N, ldw = W.shape
+    K = lda if K is None else K
+    od = 1 if out.dtype == torch.bfloat16 else 0
+    _check(None, load().ravel_gemm_noalloc(_dptr(X, torch.bfloat16, "X"), M, K, lda, _dptr(W, torch.bfloat16, "W"),
+                                           N, ldw, epi, _dptr(out, name="out"), out.shape[1], od,
+                                           _dptr(bias, torch.float32, "bias"), _stream_ptr(stream)),
+           "ravel_gemm_noalloc")
 
 
 def ravel_get_state(h, batch: int) -> np.ndarray:
