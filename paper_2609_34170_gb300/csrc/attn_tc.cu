@@ -1,0 +1,533 @@
+// Grouped-query attention of the action slots on the 5th-generation tensor
+// cores (tcgen05 + TMEM + TMA), flash-attention style.
+//
+// One CTA owns a tile of up to 128 query rows of one (robot b, KV head g)
+// pair -- row r = t*G + hh is slot j0+t of query head g*G+hh -- and walks the
+// pair's keys in chunks of 64: first the active VLM context's prefix
+// (context slot, valid length read on the device), then the FOP tokens and
+// the H action slots of this step (the QKV buffer).  Per chunk:
+//   S = Q K^T        tcgen05.mma, M = 128 query rows, N = 64 keys, into TMEM
+//   P = exp(S - m)   softmax warps: TMEM -> registers -> bf16 P in shared memory
+//   O += P V         tcgen05.mma, M = 128, N = head dim, K = 64 keys, O in TMEM
+// Every operand is K-major with 128-byte swizzling; V is kept transposed
+// (keys contiguous) for that: the context's V is transposed when a context
+// is installed, and the step's own V by the QKV projection's epilogue.
+// The online softmax rescales O in TMEM only when a row's running maximum
+// grows by more than 2^8 (the kept maximum is exact for the final
+// normalisation, so this is not an approximation).
+// At batch 1 a (b, g) pair has only a few query tiles, so the key chunks are
+// split over grid.z and a combine kernel merges the partial (O, m, l).
+//
+// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator + MMA
+// issuer, warps 2..5 softmax / epilogue (warp w owns TMEM lanes 32*(w%4)..).
+// Every wait is bounded (ERR_TIMEOUT, then unwind).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "launch.h"
+#include "tc_common.cuh"
+
+namespace ravel {
+namespace {
+
+constexpr int AT_THREADS = 192;
+constexpr int AT_BM = 128;
+constexpr int AT_BKV = 64;
+constexpr int AT_SMEM_MAX = 227 * 1024;
+constexpr uint32_t AT_QBLK = AT_BM * 128;     // bytes of one 64-wide head-dim block of Q
+constexpr uint32_t AT_KBLK = AT_BKV * 128;    // bytes of one 64-wide head-dim block of a K chunk
+constexpr uint32_t AT_PBUF = AT_BM * 128;     // bytes of one P tile (128 rows x 64 keys bf16)
+
+struct AtParams {
+  int B, H, F, Hq, Hkv, G, hd, hdp;   // hdp: head dim rounded up to 16 (MMA N of P V)
+  int TQ, q_tiles;
+  int Pmax, n_pre, n_kv, splits;
+  int layer, Bmax, mask_mode;
+  int nblk, stages;
+  uint32_t vt_bytes;                  // bytes of one transposed-V chunk (hd rows x 128 B)
+  const int* ctx_state;
+  bf16* out;
+  int ld_out;
+  float* ws_o;
+  float* ws_ml;
+  int* err;
+  float scale_log2;                   // log2(e) / sqrt(hd)
+};
+
+struct AtMaps {
+  CUtensorMap q, k, vt, pk0, pk1, pv0, pv1;
+};
+
+__device__ __forceinline__ int chunk_count(const AtParams& p, int P, int c0, int c1) {
+  int n = 0;
+  for (int c = c0; c < c1; ++c)
+    if (!(c < p.n_pre && c * AT_BKV >= P)) ++n;
+  return n;
+}
+
+__global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_constant__ AtMaps maps, AtParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int S = p.stages;
+  const uint32_t k_bytes = (uint32_t)p.nblk * AT_KBLK;
+  const uint32_t stage_bytes = k_bytes + p.vt_bytes;   // both multiples of 1024
+  uint8_t* q_s = smem;
+  uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;
+  uint8_t* p_s = kv_s + (size_t)S * stage_bytes;
+  uint64_t* bars = (uint64_t*)(p_s + 2 * AT_PBUF);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;
+  uint64_t* kv_empty = kv_full + S;
+  uint64_t* s_full = kv_empty + S;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* pv_done = p_full + 2;
+  uint32_t* tmem_slot = (uint32_t*)(pv_done + 1);
+  int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] issued, [2] consumed
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x, bg = blockIdx.y, split = blockIdx.z;
+  const int b = bg / p.Hkv, g = bg % p.Hkv;
+  const int rows_per_robot = p.H + p.F;
+  const int slot = p.ctx_state[0];
+  const int P = p.ctx_state[1];
+  const int C = p.n_pre + p.n_kv;
+  const int c0 = (int)((long)split * C / p.splits), c1 = (int)((long)(split + 1) * C / p.splits);
+  const uint32_t ncols = (128 + p.hdp <= 256) ? 256u : 512u;
+  const int ctx_z = (p.layer * p.Bmax + b) * p.Hkv + g;
+
+  pdl_trigger();
+  if (P < 1 || P > p.Pmax) {   // uniform across the CTA: nothing allocated yet
+    pdl_wait();
+    if (threadIdx.x == 0) raise_error(p.err, ERR_PREFIX_LEN);
+    return;
+  }
+  const int n = chunk_count(p, P, c0, c1);
+  // the active context (slot, length and its prefix K/V) is fixed for the
+  // whole step, so the first prefix chunks are fetched before the wait on the
+  // previous kernel (the QKV projection)
+  int npre = 0, c_next = c0;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], 128);
+      mbar_init(&p_full[i], 128);
+    }
+    mbar_init(pv_done, 1);
+    flags[0] = flags[1] = flags[2] = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    uint64_t pol_kv;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_kv));
+    const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
+    const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
+    for (; c_next < c1 && c_next < p.n_pre && npre < S; ++c_next) {
+      if (c_next * AT_BKV >= P) continue;
+      uint8_t* ks = kv_s + (size_t)npre * stage_bytes;
+      mbar_expect_tx(&kv_full[npre], k_bytes + 128u * (uint32_t)p.hd);
+      for (int blk = 0; blk < p.nblk; ++blk)
+        tma_load_3d(pk, &kv_full[npre], ks + (size_t)blk * AT_KBLK, blk * 64, c_next * AT_BKV, ctx_z, pol_kv);
+      tma_load_3d(pv, &kv_full[npre], ks + k_bytes, c_next * AT_BKV, 0, ctx_z, pol_kv);
+      ++npre;
+    }
+  }
+  // rows of the Q tile that no query fills are zeroed (their scores are unused)
+  const int q_rows = p.TQ * p.G;
+  if (q_rows < AT_BM) {
+    for (int blk = 0; blk < p.nblk; ++blk) {
+      uint4* z = (uint4*)(q_s + (size_t)blk * AT_QBLK + (size_t)q_rows * 128);
+      for (int i = threadIdx.x; i < (AT_BM - q_rows) * 8; i += AT_THREADS) z[i] = make_uint4(0, 0, 0, 0);
+    }
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  pdl_wait();
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t o_col = 128;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint64_t pol_q, pol_kv;
+      asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_q));
+      asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_kv));
+      mbar_expect_tx(q_full, (uint32_t)p.nblk * 128u * (uint32_t)q_rows);
+      for (int blk = 0; blk < p.nblk; ++blk)
+        tma_load_3d(&maps.q, q_full, q_s + (size_t)blk * AT_QBLK, blk * 64, g * p.G, b * rows_per_robot + qt * p.TQ,
+                    pol_q);
+      const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
+      const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
+      int i = npre;
+      for (int c = c_next; c < c1; ++c) {
+        if (c < p.n_pre && c * AT_BKV >= P) continue;
+        const int s = i % S;
+        if (!mbar_wait(&kv_empty[s], ((uint32_t)(i / S) & 1u) ^ 1u)) {
+          flags[0] = 1;
+          break;
+        }
+        uint8_t* ks = kv_s + (size_t)s * stage_bytes;
+        uint8_t* vs = ks + k_bytes;
+        mbar_expect_tx(&kv_full[s], k_bytes + 128u * (uint32_t)p.hd);   // V box: hd rows x 64 keys
+        if (c < p.n_pre) {
+          for (int blk = 0; blk < p.nblk; ++blk)
+            tma_load_3d(pk, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, c * AT_BKV, ctx_z, pol_kv);
+          tma_load_3d(pv, &kv_full[s], vs, c * AT_BKV, 0, ctx_z, pol_kv);
+        } else {
+          const int cc = c - p.n_pre;
+          for (int blk = 0; blk < p.nblk; ++blk)
+            tma_load_3d(&maps.k, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, b * rows_per_robot + cc * AT_BKV,
+                        pol_q);
+          tma_load_3d(&maps.vt, &kv_full[s], vs, cc * AT_BKV, 0, b * p.Hkv + g, pol_q);
+        }
+        ++i;
+      }
+      flags[1] = i;
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc_s = idesc_bf16(AT_BM, AT_BKV);
+      const uint32_t idesc_o = idesc_bf16(AT_BM, p.hdp);
+      bool ok = mbar_wait(q_full, 0);
+      auto issue_s = [&](int j) -> bool {
+        const int s = j % S;
+        if (!mbar_wait(&kv_full[s], (uint32_t)(j / S) & 1u)) return false;
+        if (j >= 2 && !mbar_wait(&s_free[j & 1], (uint32_t)((j >> 1) - 1) & 1u)) return false;
+        tc_fence_after();
+        const uint8_t* ks = kv_s + (size_t)s * stage_bytes;
+        for (int blk = 0; blk < p.nblk; ++blk) {
+          const uint64_t ad = sw128_desc(smem_u32(q_s + (size_t)blk * AT_QBLK));
+          const uint64_t bd = sw128_desc(smem_u32(ks + (size_t)blk * AT_KBLK));
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(tmem + (uint32_t)(j & 1) * AT_BKV, ad + 2 * k, bd + 2 * k, idesc_s, (blk > 0 || k > 0) ? 1u : 0u);
+        }
+        umma_commit(&s_full[j & 1]);
+        return true;
+      };
+      int i = 0;
+      if (ok && n > 0) ok = issue_s(0);
+      for (; ok && i < n; ++i) {
+        if (i + 1 < n && !issue_s(i + 1)) {
+          ok = false;
+          break;
+        }
+        if (!mbar_wait(&p_full[i & 1], (uint32_t)(i >> 1) & 1u)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int s = i % S;
+        const uint64_t ad = sw128_desc(smem_u32(p_s + (size_t)(i & 1) * AT_PBUF));
+        const uint64_t bd = sw128_desc(smem_u32(kv_s + (size_t)s * stage_bytes + k_bytes));
+#pragma unroll
+        for (int k = 0; k < 4; ++k) umma_bf16(tmem + o_col, ad + 2 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
+        umma_commit(&kv_empty[s]);
+        umma_commit(pv_done);
+      }
+      if (!ok) flags[0] = 1;
+      flags[2] = i;
+    }
+  } else {
+    // softmax / epilogue: thread owns query row r (TMEM lane r)
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(q4 * 32) << 16);
+    const int t = r / p.G, hh = r % p.G;
+    const int j = qt * p.TQ + t;
+    const bool row_ok = (r < q_rows) && (j < p.H);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    int i = 0;
+    for (int c = c0; c < c1 && ok; ++c) {
+      if (c < p.n_pre && c * AT_BKV >= P) continue;
+      ok = __all_sync(0xffffffffu, mbar_wait(&s_full[i & 1], (uint32_t)(i >> 1) & 1u));
+      tc_fence_after();
+      float sc[64];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) tmem_ld16(lane_base + (uint32_t)(i & 1) * AT_BKV + 16 * q, sc + 16 * q);
+      tc_fence_before();
+      mbar_arrive(&s_free[i & 1]);
+      // key validity
+      float mx = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        bool v;
+        if (c < p.n_pre) {
+          v = c * AT_BKV + k < P;
+        } else {
+          const int kk = (c - p.n_pre) * AT_BKV + k;
+          v = kk < rows_per_robot;
+          if (p.mask_mode == 1 && kk < p.H) v = v && (kk == j);
+        }
+        sc[k] = v ? sc[k] * p.scale_log2 : -INFINITY;
+        mx = fmaxf(mx, sc[k]);
+      }
+      if (i > 0) {
+        ok = __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(i - 1) & 1u)) && ok;
+        tc_fence_after();
+      }
+      const float m_new = fmaxf(m_used, mx);
+      const bool need = m_new > m_used + 8.f;
+      if (i > 0 && __any_sync(0xffffffffu, need)) {
+        const float alpha = need ? exp2f(m_used - m_new) : 1.f;   // exp2(-inf) = 0
+        for (int cb = 0; cb < p.hdp; cb += 16) {
+          float o[16];
+          tmem_ld16(lane_base + o_col + cb, o);
+#pragma unroll
+          for (int q = 0; q < 16; ++q) o[q] *= alpha;
+          tmem_st16(lane_base + o_col + cb, o);
+        }
+        tmem_wait_st();
+        l *= alpha;
+      }
+      if (need) m_used = m_new;
+      const float base = (m_used == -INFINITY) ? 0.f : m_used;
+      uint8_t* prow = p_s + (size_t)(i & 1) * AT_PBUF + (size_t)r * 128;
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        uint32_t w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const bf16 lo = __float2bfloat16_rn(exp2f(sc[8 * ch + 2 * q] - base));
+          const bf16 hi = __float2bfloat16_rn(exp2f(sc[8 * ch + 2 * q + 1] - base));
+          l += __bfloat162float(lo) + __bfloat162float(hi);
+          w[q] = (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+        }
+        *(uint4*)(prow + ((ch ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_before();
+      mbar_arrive(&p_full[i & 1]);
+      ++i;
+    }
+    if (ok && n > 0) {
+      ok = __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(n - 1) & 1u));
+      tc_fence_after();
+    }
+    if (!ok && lane == 0) flags[0] = 1;
+    const int h = g * p.G + hh;
+    if (p.splits == 1) {
+      const float inv = (l > 0.f) ? 1.f / l : 0.f;
+      for (int cb = 0; cb < p.hdp; cb += 16) {
+        float o[16];
+        tmem_ld16(lane_base + o_col + cb, o);
+        if (row_ok && n > 0) {
+          bf16* dst = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)h * p.hd + cb;
+#pragma unroll
+          for (int q = 0; q < 16; ++q)
+            if (cb + q < p.hd) dst[q] = __float2bfloat16_rn(o[q] * inv);
+        }
+      }
+    } else {
+      // partial tile, column-major ([d][row]) so that a warp's stores are contiguous
+      const int cta = bg * gridDim.x + qt;
+      const size_t ti = (size_t)split * gridDim.x * gridDim.y + cta;
+      for (int cb = 0; cb < p.hdp; cb += 16) {
+        float o[16];
+        tmem_ld16(lane_base + o_col + cb, o);
+        float* dst = p.ws_o + (ti * p.hdp + cb) * AT_BM + r;
+#pragma unroll
+        for (int q = 0; q < 16; ++q) dst[(size_t)q * AT_BM] = (n > 0) ? o[q] : 0.f;
+      }
+      p.ws_ml[(ti * 2) * AT_BM + r] = (n > 0) ? m_used : -INFINITY;
+      p.ws_ml[(ti * 2 + 1) * AT_BM + r] = (n > 0) ? l : 0.f;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (flags[0]) {
+    if (threadIdx.x == 0) {
+      for (int i = flags[2]; i < flags[1]; ++i) mbar_wait(&kv_full[i % S], (uint32_t)(i / S) & 1u);
+      raise_error(p.err, ERR_TIMEOUT);
+    }
+    __syncthreads();
+  }
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
+  }
+}
+
+// Merge the split partials: O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
+// Block = (tile, 8 head-dim columns), thread = tile row; the column-major
+// partials make every load of a warp contiguous.
+__global__ void attn_combine_kernel(AtParams p, int nctas) {
+  pdl_trigger();
+  pdl_wait();
+  const int cta = blockIdx.x, d0 = blockIdx.y * 8, r = threadIdx.x;
+  const int qt = cta % p.q_tiles, bg = cta / p.q_tiles;
+  const int b = bg / p.Hkv, g = bg % p.Hkv;
+  const int t = r / p.G, hh = r % p.G;
+  const int j = qt * p.TQ + t;
+  if (r >= p.TQ * p.G || j >= p.H) return;
+  const int S = p.splits;   // <= 64
+  float w[64];
+  float M = -INFINITY;
+#pragma unroll 8
+  for (int s = 0; s < S; ++s) {
+    w[s] = p.ws_ml[(((size_t)s * nctas + cta) * 2) * AT_BM + r];
+    M = fmaxf(M, w[s]);
+  }
+  float L = 0.f;
+#pragma unroll 8
+  for (int s = 0; s < S; ++s) {
+    const float l = p.ws_ml[(((size_t)s * nctas + cta) * 2 + 1) * AT_BM + r];
+    w[s] = (w[s] == -INFINITY) ? 0.f : exp2f(w[s] - M);
+    L += w[s] * l;
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  float acc[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+  for (int s = 0; s < S; ++s) {
+    const float* src = p.ws_o + (((size_t)s * nctas + cta) * p.hdp + d0) * AT_BM + r;
+    float x[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) x[q] = (d0 + q < p.hdp) ? src[(size_t)q * AT_BM] : 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] += w[s] * x[q];
+  }
+  bf16* dst = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    if (d0 + q < p.hd) dst[d0 + q] = __float2bfloat16_rn(acc[q] * inv);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
+
+cudaError_t enc3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1_bytes,
+                 uint64_t s2_bytes, uint32_t b0, uint32_t b1, uint32_t b2) {
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {s1_bytes, s2_bytes};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+cudaError_t init_attention_tc() {
+  if (!g_enc) {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorSymbolNotFound;
+    g_enc = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  }
+  return cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM_MAX);
+}
+
+bool attention_tc_supported(int hd, int G) { return hd % 8 == 0 && hd <= 256 && G >= 1 && G <= 128; }
+
+cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
+  if (!g_enc) return cudaErrorInitializationError;
+  AtParams p{};
+  p.B = a.B; p.H = a.H; p.F = a.F; p.Hq = a.Hq; p.Hkv = a.Hkv; p.G = a.Hq / a.Hkv; p.hd = a.hd;
+  p.hdp = (a.hd + 15) / 16 * 16;
+  const int tq_max = AT_BM / p.G;
+  p.q_tiles = (a.H + tq_max - 1) / tq_max;
+  p.TQ = (a.H + p.q_tiles - 1) / p.q_tiles;
+  p.Pmax = a.Pmax;
+  p.n_pre = (a.Pmax + AT_BKV - 1) / AT_BKV;
+  p.n_kv = (a.H + a.F + AT_BKV - 1) / AT_BKV;
+  p.layer = a.layer; p.Bmax = a.Bmax; p.mask_mode = a.mask_mode;
+  p.nblk = (a.hd + 63) / 64;
+  p.vt_bytes = (uint32_t)((p.hdp * 128 + 1023) / 1024 * 1024);
+  p.ctx_state = a.ctx_state;
+  p.out = (bf16*)a.out; p.ld_out = a.ld_out;
+  p.err = a.err;
+  p.scale_log2 = 1.4426950408889634f / sqrtf((float)a.hd);
+  const int nctas = p.q_tiles * a.B * a.Hkv;
+  const int C = p.n_pre + p.n_kv;
+  // split the key chunks only when the (b, g, q-tile) grid leaves most SMs
+  // idle; about two chunks per split so S(i+1) overlaps the softmax of i
+  int splits = 1;
+  if (nctas * 2 <= a.num_sms) splits = std::min({(C + 1) / 2, std::max(1, a.num_sms / nctas), 64});
+  while (splits > 1 && (size_t)splits * nctas * AT_BM * (p.hdp + 2) * 4 > a.ws_bytes) --splits;
+  p.splits = splits;
+  p.ws_o = a.ws;
+  p.ws_ml = a.ws + (size_t)splits * nctas * AT_BM * p.hdp;
+  const uint32_t stage = (uint32_t)p.nblk * AT_KBLK + p.vt_bytes;
+  const size_t fixed = 1024 + (size_t)p.nblk * AT_QBLK + 2 * AT_PBUF + 256;
+  int stages = (int)std::min<size_t>(4, (AT_SMEM_MAX - fixed) / stage);
+  if (stages < 1) return cudaErrorInvalidConfiguration;
+  p.stages = stages;
+  const size_t smem = fixed + (size_t)stages * stage;
+
+  AtMaps m;
+  const int hd = a.hd, rpr = a.H + a.F;
+  const uint64_t rows = (uint64_t)a.B * rpr;
+  cudaError_t e = enc3(&m.q, a.qkv, hd, a.Hq, rows, (uint64_t)hd * 2, (uint64_t)a.ld_qkv * 2, 64, p.G, p.TQ);
+  if (e == cudaSuccess)
+    e = enc3(&m.k, (const bf16*)a.qkv + (size_t)a.Hq * hd, hd, a.Hkv, rows, (uint64_t)hd * 2, (uint64_t)a.ld_qkv * 2,
+             64, 1, AT_BKV);
+  if (e == cudaSuccess)
+    e = enc3(&m.vt, a.vt, rpr, hd, (uint64_t)a.B * a.Hkv, (uint64_t)a.kvp * 2, (uint64_t)hd * a.kvp * 2, AT_BKV, hd, 1);
+  const uint64_t zc = (uint64_t)(a.layers * a.Bmax * a.Hkv);
+  for (int s = 0; s < 2 && e == cudaSuccess; ++s) {
+    e = enc3(s ? &m.pk1 : &m.pk0, a.ctx_k[s], hd, a.Pmax, zc, (uint64_t)hd * 2, (uint64_t)a.Pmax * hd * 2, 64,
+             AT_BKV, 1);
+    if (e == cudaSuccess)
+      e = enc3(s ? &m.pv1 : &m.pv0, a.ctx_vt[s], a.Pmax, hd, zc, (uint64_t)a.pst * 2, (uint64_t)hd * a.pst * 2,
+               AT_BKV, hd, 1);
+  }
+  if (e != cudaSuccess) return e;
+  dim3 grid(p.q_tiles, a.B * a.Hkv, splits);
+  e = launch_kernel(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, 1, m, p);
+  if (a.n_launched) ++*a.n_launched;
+  if (e == cudaSuccess && splits > 1) {
+    e = launch_kernel(attn_combine_kernel, dim3(nctas, (p.hd + 7) / 8), dim3(AT_BM), 0, st, 1, p, nctas);
+    if (a.n_launched) ++*a.n_launched;
+  }
+  return e;
+}
+
+// Context V [L][B][Hkv][P][hd] -> slot Vt [L][Bmax][Hkv][hd][pst] (keys contiguous).
+__global__ void transpose_ctx_v_kernel(const bf16* __restrict__ src, bf16* __restrict__ dst, int B, int Bmax,
+                                       int Hkv, int P, int hd, int pst) {
+  __shared__ bf16 tile[32][33];
+  const int z = blockIdx.z;                 // (l * B + b) * Hkv + g
+  const int g = z % Hkv, lb = z / Hkv;
+  const int bb = lb % B, l = lb / B;
+  const bf16* s = src + (size_t)z * P * hd;
+  bf16* d = dst + ((size_t)(l * Bmax + bb) * Hkv + g) * hd * pst;
+  const int p0 = blockIdx.x * 32, d0 = blockIdx.y * 32;
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int pp = p0 + i, dd = d0 + threadIdx.x;
+    tile[i][threadIdx.x] = (pp < P && dd < hd) ? s[(size_t)pp * hd + dd] : __float2bfloat16_rn(0.f);
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int dd = d0 + i, pp = p0 + threadIdx.x;
+    if (dd < hd && pp < P) d[(size_t)dd * pst + pp] = tile[threadIdx.x][i];
+  }
+}
+
+cudaError_t launch_transpose_ctx_v(const void* src, void* dst, int L, int B, int Bmax, int Hkv, int P, int hd,
+                                   int pst, cudaStream_t st) {
+  dim3 grid((P + 31) / 32, (hd + 31) / 32, L * B * Hkv), block(32, 8);
+  transpose_ctx_v_kernel<<<grid, block, 0, st>>>((const bf16*)src, (bf16*)dst, B, Bmax, Hkv, P, hd, pst);
+  return cudaGetLastError();
+}
+
+}  // namespace ravel

@@ -48,6 +48,12 @@ __device__ __forceinline__ void raise_error(int* err, int bits) {
   if (err) atomicOr(err, bits);
 }
 
+// Programmatic Dependent Launch: let the next kernel in the stream start
+// launching, and wait until the previous kernel has completed and its memory
+// is visible (a no-op when the kernel was not launched programmatically).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + expf(-x)); }
 
 __device__ __forceinline__ float gelu_tanh_f(float g) {

@@ -94,6 +94,6 @@ extern "C" ravel_status ravel_gemm_noalloc(const void* X, int M, int K, int lda,
   // The split plan is chosen so that the partials fit the array (fewer
   // splits, or none, when they would not).
   TcWorkspace ws{(float*)s->scratch, kPartialBytes, (int*)zero, kCounters, (int*)zero + kCounters};
-  if (launch_gemm_tc(g, ws, s->num_sms, st) != cudaSuccess) return RAVEL_ECUDA;
+  if (launch_gemm_tc(g, ws, s->num_sms, st, /*cluster=*/false) != cudaSuccess) return RAVEL_ECUDA;
   return RAVEL_OK;
 }

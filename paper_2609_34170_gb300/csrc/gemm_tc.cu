@@ -26,6 +26,8 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "launch.h"
+#include "tc_common.cuh"
 
 namespace ravel {
 namespace {
@@ -34,13 +36,14 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
 constexpr int TC_THREADS = 192;
 constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;
-constexpr unsigned long long TC_TIMEOUT_NS = 1000000000ull;   // 1 s
 constexpr int TC_SMEM_BUDGET = 200 * 1024;                     // operand ring
 constexpr int TC_SMEM_MAX = 227 * 1024;
 
 struct TcParams {
   int M, N, K;
   int bn, stages, splits, num_kb;
+  int cluster_reduce;   // the grid.z splits of a tile form a cluster; 1: reduce through DSMEM, 2: through L2
+  uint32_t ring_bytes;  // operand ring (also holds the fp32 partial tile in cluster mode)
   int epi;          // Epi value, or EPI_GEGLU
   int out_bf16;
   void* out;
@@ -49,104 +52,37 @@ struct TcParams {
   float* ws;
   int* counters;
   int* err;
+  bf16* vt;
+  int v_col0, vt_hd, vt_tokens, vt_kvp, vt_hkv;
 };
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ unsigned long long globaltimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Wait for the phase of `parity` to complete; false after TC_TIMEOUT_NS.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const unsigned long long t0 = globaltimer();
-  while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer() - t0 > TC_TIMEOUT_NS) return false;
-  }
-  return true;
-}
-
-__device__ __forceinline__ void tma_load_2d(const CUtensorMap* map, uint64_t* bar, void* dst, int x, int y,
-                                            uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(policy)
-      : "memory");
-}
-
-// Shared-memory matrix descriptor of a K-major tile written by TMA with
-// 128-byte swizzling: rows of 128 bytes, 8-row groups 1024 bytes apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)1 << 16;                 // leading byte offset (unused for swizzled K-major)
-  d |= (uint64_t)(1024 >> 4) << 32;       // stride byte offset: next 8-row group
-  d |= (uint64_t)1 << 46;                 // descriptor version of tcgen05
-  d |= (uint64_t)2 << 61;                 // 128-byte swizzle
-  return d;
-}
-
-// Instruction descriptor of kind::f16 with bf16 A/B, fp32 D, both K-major.
-__device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
-}
-
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(acc));
-}
-
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-               : "memory");
-}
-
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float v[16]) {
-  uint32_t r[16];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
-      "%15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+// v[i] += sum over splits s = 0..S-1 (in order) of the partial at column
+// cc + i of split s; base points at this thread's row of split 0, column 0.
+// Up to 64 loads are in flight per batch; splits past S add exact zeros.
+template <int NC>
+__device__ __forceinline__ void reduce_splits_l2(const float* base, int S, int BN, int cc, float v[16]) {
+  constexpr int G = 64 / NC;
+  for (int s0 = 0; s0 < S; s0 += G) {
+    float x[G][NC];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+    for (int u = 0; u < G; ++u)
+#pragma unroll
+      for (int i = 0; i < NC; ++i)
+        x[u][i] = (s0 + u < S) ? __ldcg(base + ((size_t)(s0 + u) * BN + cc + i) * 128) : 0.f;
+#pragma unroll
+    for (int u = 0; u < G; ++u)
+#pragma unroll
+      for (int i = 0; i < NC; ++i) v[i] += x[u][i];
+  }
 }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// Apply the epilogue to 16 consecutive tokens m0..m0+15 of weight row n.
-// `xch` is the 64x16 exchange tile of the GeGLU epilogue.
+// Apply the epilogue to nc (<= 16) consecutive tokens m0.. of tile row r.
+// `xch` is the 64x16 exchange tile of the GeGLU epilogue (all 128 epilogue
+// threads must call this together in that mode).
 __device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile_n, int r, int m0, float v[16],
-                                               float* xch) {
+                                               float* xch, int nc = 16) {
   if (p.epi == EPI_GEGLU) {
     // rows 0..63 of the tile are gate features, rows 64..127 the matching up features
     if (r >= 64) {
@@ -161,7 +97,7 @@ __device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile_n, in
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int m = m0 + i;
-          if (m < p.M) o[(size_t)m * p.ldo + f] = __float2bfloat16_rn(gelu_tanh_f(v[i]) * xch[r * 17 + i]);
+          if (i < nc && m < p.M) o[(size_t)m * p.ldo + f] = __float2bfloat16_rn(gelu_tanh_f(v[i]) * xch[r * 17 + i]);
         }
       }
     }
@@ -171,15 +107,25 @@ __device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile_n, in
   const int n = tile_n * TC_BM + r;
   if (n >= p.N) return;
   const float b = p.bias ? p.bias[n] : 0.f;
+  if (p.epi == EPI_ADD_F32) {
+    // residual accumulate: all loads first, so their latencies overlap
+    float* o = (float*)p.out;
+    float old[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < nc && m0 + i < p.M) old[i] = o[(size_t)(m0 + i) * p.ldo + n];
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < nc && m0 + i < p.M) o[(size_t)(m0 + i) * p.ldo + n] = old[i] + (v[i] + b);
+    return;
+  }
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     const int m = m0 + i;
-    if (m >= p.M) continue;
+    if (i >= nc || m >= p.M) continue;
     float x = v[i] + b;
     const size_t idx = (size_t)m * p.ldo + n;
-    if (p.epi == EPI_ADD_F32) {
-      ((float*)p.out)[idx] += x;
-    } else {
+    {
       if (p.epi == EPI_STORE_SILU) x = silu_f(x);
       if (p.out_bf16)
         ((bf16*)p.out)[idx] = __float2bfloat16_rn(x);
@@ -187,9 +133,19 @@ __device__ __forceinline__ void apply_epilogue(const TcParams& p, int tile_n, in
         ((float*)p.out)[idx] = x;
     }
   }
+  if (p.vt && n >= p.v_col0) {
+    const int g = (n - p.v_col0) / p.vt_hd, d = (n - p.v_col0) % p.vt_hd;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int m = m0 + i;
+      if (i >= nc || m >= p.M) continue;
+      const int bb = m / p.vt_tokens, kk = m % p.vt_tokens;
+      p.vt[((size_t)(bb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp + kk] = __float2bfloat16_rn(v[i] + b);
+    }
+  }
 }
 
-__global__ void __launch_bounds__(TC_THREADS, 1)
+__global__ void __launch_bounds__(TC_THREADS, 2)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -197,7 +153,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const uint32_t b_bytes = (uint32_t)BN * TC_BK * 2;
   uint8_t* a_s = smem;
   uint8_t* b_s = smem + (size_t)S * TC_A_BYTES;
-  uint64_t* full = (uint64_t*)(b_s + (size_t)S * b_bytes);
+  uint64_t* full = (uint64_t*)(smem + p.ring_bytes);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
   uint32_t* tmem_slot = (uint32_t*)(accb + 1);
@@ -212,6 +168,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   uint32_t ncols = 32;
   while ((int)ncols < BN) ncols <<= 1;
 
+  pdl_trigger();
+  const int npre = nkb < S ? nkb : S;   // stages whose weight tiles are fetched before the dependency wait
+  uint64_t pol_w = 0, pol_x = 0;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
@@ -221,7 +180,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     flags[0] = flags[1] = flags[2] = flags[3] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // Weights never depend on earlier kernels: stream the first stages' weight
+    // tiles while the previous kernel is still finishing.
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&tmW) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&tmX) : "memory");
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
+    for (int i = 0; i < npre; ++i) {
+      mbar_expect_tx(&full[i], TC_A_BYTES + b_bytes);
+      tma_load_2d(&tmW, &full[i], a_s + (size_t)i * TC_A_BYTES, (kb0 + i) * TC_BK, tile_n * TC_BM, pol_w);
+    }
   }
+  // everything below may read what earlier kernels wrote; TMEM is taken only
+  // now, so a CTA waiting here never holds columns its predecessor needs
+  pdl_wait();
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"(ncols)
@@ -235,12 +207,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(&tmW) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(&tmX) : "memory");
-      uint64_t pol_w, pol_x;
-      asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
-      asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
-      int i = 0;
+      for (int i = 0; i < npre; ++i)
+        tma_load_2d(&tmX, &full[i], b_s + (size_t)i * b_bytes, (kb0 + i) * TC_BK, tile_m * BN, pol_x);
+      int i = npre;
       for (; i < nkb; ++i) {
         const int s = i % S;
         const uint32_t ph = (uint32_t)(i / S) & 1u;
@@ -286,7 +255,31 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
     const int m_base = tile_m * BN;
-    if (p.splits == 1) {
+    if (p.cluster_reduce == 2) {
+      // this split's fp32 partial tile to the workspace, column-major per tile
+      // ([col][row]) so a warp's stores and the later loads are contiguous
+      const size_t cl = (size_t)tile_m * gridDim.x + tile_n;
+      float* w = p.ws + ((cl * p.splits + split) * (size_t)BN) * TC_BM + r;
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        float v[16];
+        tmem_ld16(trow + c0, v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) __stcg(w + (size_t)(c0 + i) * TC_BM, v[i]);
+      }
+      __threadfence();
+    } else if (p.cluster_reduce) {
+      // this split's fp32 partial tile into its own shared memory (the drained
+      // operand ring), rows padded to BN + 4 floats against bank conflicts
+      float* part = (float*)smem;
+      const int ld = BN + 4;
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        float v[16];
+        tmem_ld16(trow + c0, v);
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq)
+          *(float4*)(part + (size_t)r * ld + c0 + 4 * qq) = make_float4(v[4 * qq], v[4 * qq + 1], v[4 * qq + 2], v[4 * qq + 3]);
+      }
+    } else if (p.splits == 1) {
       for (int c0 = 0; c0 < BN; c0 += 16) {
         float v[16];
         tmem_ld16(trow + c0, v);
@@ -336,6 +329,103 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     __syncthreads();
   }
+  if (p.cluster_reduce == 2) {
+    // Every split of this tile has written its partial to the workspace; the
+    // cluster barrier (release / acquire) makes them visible.  CTA rank q sums
+    // columns [q*BN/S, (q+1)*BN/S) over splits 0..S-1 in order (deterministic)
+    // with all loads of a chunk in flight together, and applies the epilogue.
+    cluster_sync();
+    if (warp >= 2) {
+      const int r = (warp & 3) * 32 + lane;
+      const int S = p.splits;
+      const int cpr = BN / S;
+      const int rank = (int)cluster_ctarank();
+      const size_t cl = (size_t)tile_m * gridDim.x + tile_n;
+      const float* base = p.ws + (cl * S * (size_t)BN + rank * cpr) * TC_BM + r;
+      for (int cc = 0; cc < cpr; cc += 16) {
+        const int nc = min(16, cpr - cc);
+        float v[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+        if (nc == 16) reduce_splits_l2<16>(base, S, BN, cc, v);
+        else if (nc == 8) reduce_splits_l2<8>(base, S, BN, cc, v);
+        else if (nc == 4) reduce_splits_l2<4>(base, S, BN, cc, v);
+        else
+          for (int i = 0; i < nc; ++i) {
+            float one[16] = {};
+            reduce_splits_l2<1>(base + (size_t)i * TC_BM, S, BN, cc, one);
+            v[i] = one[0];
+          }
+        apply_epilogue(p, tile_n, r, tile_m * BN + rank * cpr + cc, v, xch, nc);
+      }
+    }
+  } else if (p.cluster_reduce) {
+    // Every split of this tile holds its partial in shared memory.  CTA rank q
+    // of the cluster sums columns [q*BN/S, (q+1)*BN/S) over ranks 0..S-1 in
+    // order (deterministic) through distributed shared memory and applies the
+    // epilogue to them.  The second cluster barrier keeps every partial alive
+    // until all ranks have read it.
+    cluster_sync();
+    if (warp >= 2) {
+      const int r = (warp & 3) * 32 + lane;
+      const int S = p.splits;
+      const int cpr = BN / S;
+      const int rank = (int)cluster_ctarank();
+      const int ld = BN + 4;
+      const uint32_t mine = smem_u32((float*)smem + (size_t)r * ld + rank * cpr);
+      for (int cc = 0; cc < cpr; cc += 16) {
+        const int nc = min(16, cpr - cc);
+        float v[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+        // all remote loads of this chunk are in flight together (one DSMEM
+        // round trip), then summed in rank order
+        if ((nc & 3) == 0) {
+          const int n4 = nc >> 2;
+          const int rpb = 16 / n4;   // ranks per batch: at most 16 float4 in flight
+          for (int s0 = 0; s0 < S; s0 += rpb) {
+            float4 x[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              const int u = k / n4, qq = k % n4;
+              if (s0 + u < S) x[k] = ld_dsmem_f4(mapa_shared(mine + 4u * cc, (uint32_t)(s0 + u)) + 16u * qq);
+            }
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              const int u = k / n4, qq = k % n4;
+              if (s0 + u < S) {
+                v[4 * qq] += x[k].x; v[4 * qq + 1] += x[k].y; v[4 * qq + 2] += x[k].z; v[4 * qq + 3] += x[k].w;
+              }
+            }
+          }
+        } else {
+          // column counts that are not a multiple of 4 (narrow slices): scalar loads
+          for (int i0 = 0; i0 < nc; i0 += 4) {
+            for (int s0 = 0; s0 < S; s0 += 4) {
+              float x[4][4];
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                if (s0 + u >= S) break;
+                const uint32_t ra = mapa_shared(mine + 4u * (cc + i0), (uint32_t)(s0 + u));
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                  if (i0 + i < nc) x[u][i] = ld_dsmem_f32(ra + 4u * i);
+              }
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                if (s0 + u >= S) break;
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                  if (i0 + i < nc) v[i0 + i] += x[u][i];
+              }
+            }
+          }
+        }
+        apply_epilogue(p, tile_n, r, tile_m * BN + rank * cpr + cc, v, xch, nc);
+      }
+    }
+    cluster_sync();
+  }
   if (warp == 1) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
@@ -377,10 +467,31 @@ int pick_bn(int M) {
 
 }  // namespace
 
+int g_max_cluster = 8;   // largest power-of-two cluster the split-K reduction may use
+
 cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
+  e = cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
+  if (e != cudaSuccess) return e;
+  // clusters of 16 are beyond the portable limit: use them only if allowed
+  if (cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 1;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 16;
+    cfg.gridDim = dim3(1, 1, 16);
+    cfg.blockDim = dim3(TC_THREADS);
+    cfg.dynamicSmemBytes = TC_SMEM_MAX;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel, &cfg) == cudaSuccess && n > 0) g_max_cluster = 16;
+  }
+  cudaGetLastError();
+  return cudaSuccess;
 }
 
 bool tc_gemm_supported(const GemmArgs& g) {
@@ -391,7 +502,7 @@ bool tc_gemm_supported(const GemmArgs& g) {
   return g.M > 0 && g.N > 0 && g.K > 0;
 }
 
-cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st) {
+cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st, bool cluster) {
   if (!g_encode) return cudaErrorInitializationError;
   const int bn = pick_bn(g.M);
   const int tiles_n = (g.N + TC_BM - 1) / TC_BM;
@@ -400,21 +511,36 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const int tiles = tiles_n * tiles_m;
   int splits = 1;
   if (tiles < num_sms) splits = std::min(num_kb, std::max(1, num_sms / tiles));
-  while (splits > 1 && ((size_t)splits * tiles * bn * TC_BM * 4 > ws.ws_bytes || tiles > ws.n_counters)) --splits;
+  if (cluster) {
+    // the splits of a tile form one cluster: a power of two, at most the cluster
+    // limit, whose partials fit the workspace
+    int c = 1;
+    while (c * 2 <= std::min(splits, g_max_cluster) &&
+           (size_t)(c * 2) * tiles * bn * TC_BM * 4 <= ws.ws_bytes)
+      c *= 2;
+    splits = c;
+  } else {
+    while (splits > 1 && ((size_t)splits * tiles * bn * TC_BM * 4 > ws.ws_bytes || tiles > ws.n_counters)) --splits;
+  }
+  const bool cluster_reduce = cluster && splits > 1;
   const int stage_bytes = TC_A_BYTES + bn * TC_BK * 2;
   int stages = std::min(8, TC_SMEM_BUDGET / stage_bytes);
   stages = std::max(2, std::min(stages, std::max(2, (num_kb + splits - 1) / splits)));
-  // 1024 alignment slack + operand ring + barriers / TMEM slot / flags (+ slack) + GeGLU exchange tile
-  const size_t smem = 1024 + (size_t)stages * stage_bytes + (2 * stages + 1) * 8 + 128 + 64 * 17 * 4;
+  size_t ring = (size_t)stages * stage_bytes;
+  if (cluster_reduce) ring = std::max(ring, (size_t)TC_BM * (bn + 4) * 4);
+  ring = (ring + 1023) / 1024 * 1024;
+  // 1024 alignment slack + ring + barriers / TMEM slot / flags (+ slack) + GeGLU exchange tile
+  const size_t smem = 1024 + ring + (2 * stages + 1) * 8 + 128 + 64 * 17 * 4;
   CUtensorMap mw, mx;
   cudaError_t e = encode_2d(&mw, g.W, g.N, g.K, g.ldw, TC_BM);
   if (e == cudaSuccess) e = encode_2d(&mx, g.A, g.M, g.K, g.lda, bn);
   if (e != cudaSuccess) return e;
-  TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo,
-             g.bias, ws.ws, ws.counters, ws.err};
+  TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, cluster_reduce ? 2 : 0, (uint32_t)ring, (int)g.epi,
+             g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt, g.v_col0,
+             g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv};
   dim3 grid(tiles_n, tiles_m, splits);
-  tc_gemm_kernel<<<grid, TC_THREADS, smem, st>>>(mw, mx, p);
-  return cudaGetLastError();
+  return launch_kernel(tc_gemm_kernel, grid, dim3(TC_THREADS), smem, st, cluster_reduce ? (unsigned)splits : 1u, mw,
+                       mx, p);
 }
 
 }  // namespace ravel

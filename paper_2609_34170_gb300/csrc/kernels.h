@@ -29,9 +29,10 @@ cudaError_t launch_convert(const float* src, size_t n, void* dst, Dtype dt, cuda
 
 // ---- conditioning -------------------------------------------------------------
 // E[r][:] = sinusoidal(x_r) for r < H (x = slot_times[r]) and H <= r < H+B
-// (x = delta[r-H]); periods geometric from 4e-3 to 4; fp64 angles.
-cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, void* E, Dtype dt,
-                         cudaStream_t st);
+// (x = delta[r-H]); periods geometric from 4e-3 to 4; fp64 angles reduced mod 2 pi.
+// omega: device fp64 [D/2] angular frequencies 2 pi / p_i.
+cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, const double* omega,
+                         void* E, Dtype dt, cudaStream_t st);
 
 // ---- generic projection GEMM: out[m][n] = sum_k A[m][k] W[n][k] (W K-major) ----
 enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2, EPI_GEGLU = 3 };
@@ -43,6 +44,11 @@ struct GemmArgs {
   void* out; int ldo;           // EPI_STORE*: dtype `out_dt`; EPI_ADD_F32: float, += result
   Dtype out_dt;
   const float* bias;            // [N] or null
+  // optional second destination of the V columns (n >= v_col0), transposed:
+  // vt[((m / vt_tokens) * vt_hkv + g) * vt_hd + d][m % vt_tokens] with
+  // g = (n - v_col0) / vt_hd, d = (n - v_col0) % vt_hd, row pitch vt_kvp
+  void* vt = nullptr;
+  int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
 
@@ -56,18 +62,23 @@ struct TcWorkspace {
 };
 cudaError_t init_tc_gemm();
 bool tc_gemm_supported(const GemmArgs& g);
-cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st);
+// cluster = true: split-K partials are reduced through distributed shared
+// memory inside a thread-block cluster (no workspace); false: through the
+// workspace `ws` with a last-arriving-CTA fix-up.
+cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st,
+                           bool cluster = true);
 
 // ---- adaRMSNorm rows ---------------------------------------------------------
 // Action rows r < B*H (b = r / H, j = r % H):
 //   Y[r] = x[r] * rsqrt(mean(x[r]^2) + 1e-6) * (1 + sc) + sh,
 //   sc[c] = modv[j][off+c] + modv[H+b][off+c] + mod_b[off+c], sh likewise at off+D.
 // FOP rows B*H + b*F + f (when fop != null): Y = z * rsqrt(mean(z^2)+1e-6) * (1 + gamma).
+// Output row of action (b, j) is b*row_pitch + j, of FOP token (b, f) b*row_pitch + H + f.
 struct NormArgs {
   const float* x; int B, H, D;
   const float* modv; int mod_ld; const float* mod_b; int off;
   const void* fop; int F; const float* gamma;
-  void* Y;
+  void* Y; int row_pitch;
 };
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 
@@ -80,7 +91,7 @@ cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cud
 
 // ---- attention ---------------------------------------------------------------
 struct AttnArgs {
-  const void* qkv; int ld_qkv;      // rows: B*H action rows, then B*F FOP rows
+  const void* qkv; int ld_qkv;      // rows of robot b: b*(H+F) + [H action slots, F FOP tokens]
   const void* ctx_k0; const void* ctx_k1;   // the two context slots [L][Bmax][Hkv][Pmax][hd]
   const void* ctx_v0; const void* ctx_v1;
   const int* ctx_state;             // device: [0] active slot, [1] prefix length
@@ -91,6 +102,27 @@ struct AttnArgs {
   int* err;
 };
 cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st);
+
+// tcgen05 attention (bf16).  V operands transposed: the context slots hold
+// Vt [L][Bmax][Hkv][hd][pst]; the step's FOP/slot V is vt [B][Hkv][hd][kvp].
+struct AttnTcArgs {
+  const void* qkv; int ld_qkv;
+  const void* vt; int kvp;
+  const void* ctx_k[2]; const void* ctx_vt[2];
+  int layers, layer, Bmax, Pmax, pst;
+  const int* ctx_state;
+  int B, H, F, Hq, Hkv, hd, mask_mode;
+  void* out; int ld_out;
+  float* ws; size_t ws_bytes;
+  int* err; int num_sms;
+  int* n_launched = nullptr;   // optional: incremented by the number of kernels launched (1 or 2)
+};
+cudaError_t init_attention_tc();
+bool attention_tc_supported(int hd, int G);
+cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st);
+// bf16 context V [L][B][Hkv][P][hd] -> slot layout Vt [L][Bmax][Hkv][hd][pst]
+cudaError_t launch_transpose_ctx_v(const void* src, void* dst, int L, int B, int Bmax, int Hkv, int P, int hd,
+                                   int pst, cudaStream_t st);
 
 // ---- rolling tail: Euler, release, shift, append ------------------------------------
 struct TailArgs {

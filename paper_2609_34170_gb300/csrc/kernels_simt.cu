@@ -4,6 +4,7 @@
 // tail (Euler update, release, shift, Philox append).
 #include "common.cuh"
 #include "kernels.h"
+#include "launch.h"
 #include "noise.cuh"
 
 namespace ravel {
@@ -59,31 +60,34 @@ cudaError_t launch_convert(const float* src, size_t n, void* dst, Dtype dt, cuda
 
 // Sinusoidal embedding of a scalar (flow time or context offset): component
 // i < D/2 is sin(x w_i), i >= D/2 is cos(x w_{i-D/2}), w_i = 2 pi / p_i with
-// periods p_i geometric from 4e-3 to 4.  Angles in fp64: x w reaches ~1.6e3
-// rad, where a float32 angle would already be off by ~1e-4.
+// periods p_i geometric from 4e-3 to 4 (w_i precomputed in fp64).  x w
+// reaches ~1.6e3 rad, where a float32 product would already be off by ~1e-4:
+// the angle is formed and reduced modulo 2 pi in fp64, then sin / cos of the
+// reduced angle (|a| <= pi) in fp32.
 template <typename T>
 __global__ void embed_kernel(const float* __restrict__ slot_times, int H, const float* __restrict__ delta, int D,
-                             T* __restrict__ E) {
-  const int r = blockIdx.x;
+                             const double* __restrict__ omega, T* __restrict__ E) {
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.y;
   const double x = (r < H) ? (double)slot_times[r] : (double)delta[r - H];
   const int half = D / 2;
-  for (int i = threadIdx.x; i < half; i += blockDim.x) {
-    const double period = 4e-3 * pow(1000.0, (double)i / (double)(half - 1));
-    const double ang = x * (6.283185307179586 / period);
-    double s, c;
-    sincos(ang, &s, &c);
-    E[(size_t)r * D + i] = from_f32<T>((float)s);
-    E[(size_t)r * D + half + i] = from_f32<T>((float)c);
-  }
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= half) return;
+  const double ang = x * omega[i];
+  const double red = ang - 6.283185307179586 * rint(ang * 0.15915494309189535);
+  float s, c;
+  sincosf((float)red, &s, &c);
+  E[(size_t)r * D + i] = from_f32<T>(s);
+  E[(size_t)r * D + half + i] = from_f32<T>(c);
 }
 
-cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, void* E, Dtype dt,
-                         cudaStream_t st) {
+cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, const double* omega,
+                         void* E, Dtype dt, cudaStream_t st) {
+  dim3 grid((D / 2 + 127) / 128, H + B);
   if (dt == DT_BF16)
-    embed_kernel<bf16><<<H + B, 128, 0, st>>>(slot_times, H, delta, D, (bf16*)E);
-  else
-    embed_kernel<float><<<H + B, 128, 0, st>>>(slot_times, H, delta, D, (float*)E);
-  return cudaGetLastError();
+    return launch_kernel(embed_kernel<bf16>, grid, dim3(128), 0, st, 1, slot_times, H, delta, D, omega, (bf16*)E);
+  return launch_kernel(embed_kernel<float>, grid, dim3(128), 0, st, 1, slot_times, H, delta, D, omega, (float*)E);
 }
 
 // ============================================================================ GEMM (SIMT)
@@ -94,6 +98,8 @@ template <typename T, int EPI, typename TO>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, int lda, const T* __restrict__ W,
                                                         int ldw, int M, int N, int K, TO* __restrict__ out, int ldo,
                                                         const float* __restrict__ bias) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float As[32][64 + 4];
   __shared__ float Ws[32][64 + 4];
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
@@ -147,21 +153,21 @@ static cudaError_t gemm_simt_dispatch(const GemmArgs& g, cudaStream_t st) {
   const T* A = (const T*)g.A;
   const T* W = (const T*)g.W;
   if (g.epi == EPI_ADD_F32) {
-    gemm_simt_kernel<T, EPI_ADD_F32, float><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
+    launch_kernel(gemm_simt_kernel<T, EPI_ADD_F32, float>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
                                                                  g.ldo, g.bias);
   } else if (g.out_dt == DT_BF16) {
     if (g.epi == EPI_STORE_SILU)
-      gemm_simt_kernel<T, EPI_STORE_SILU, bf16><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K,
+      launch_kernel(gemm_simt_kernel<T, EPI_STORE_SILU, bf16>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K,
                                                                      (bf16*)g.out, g.ldo, g.bias);
     else
-      gemm_simt_kernel<T, EPI_STORE, bf16><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K, (bf16*)g.out,
+      launch_kernel(gemm_simt_kernel<T, EPI_STORE, bf16>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K, (bf16*)g.out,
                                                                 g.ldo, g.bias);
   } else {
     if (g.epi == EPI_STORE_SILU)
-      gemm_simt_kernel<T, EPI_STORE_SILU, float><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K,
+      launch_kernel(gemm_simt_kernel<T, EPI_STORE_SILU, float>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K,
                                                                       (float*)g.out, g.ldo, g.bias);
     else
-      gemm_simt_kernel<T, EPI_STORE, float><<<grid, 256, 0, st>>>(A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
+      launch_kernel(gemm_simt_kernel<T, EPI_STORE, float>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
                                                                  g.ldo, g.bias);
   }
   return cudaGetLastError();
@@ -176,11 +182,18 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st) {
 
 template <typename T>
 __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
   const int r = blockIdx.x;
   const int D = a.D;
   const int n_act = a.B * a.H;
-  T* Y = (T*)a.Y + (size_t)r * D;
+  size_t yrow;
+  if (r < n_act)
+    yrow = (size_t)(r / a.H) * a.row_pitch + r % a.H;
+  else
+    yrow = (size_t)((r - n_act) / a.F) * a.row_pitch + a.H + (r - n_act) % a.F;
+  T* Y = (T*)a.Y + yrow * D;
   if (r < n_act) {
     const int b = r / a.H, j = r % a.H;
     const float* x = a.x + (size_t)r * D;
@@ -210,37 +223,40 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a) {
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st) {
   const int rows = a.B * a.H + (a.fop ? a.B * a.F : 0);
   if (rows <= 0) return cudaSuccess;
-  if (dt == DT_BF16)
-    ada_norm_kernel<bf16><<<rows, 256, 0, st>>>(a);
-  else
-    ada_norm_kernel<float><<<rows, 256, 0, st>>>(a);
-  return cudaGetLastError();
+  if (dt == DT_BF16) return launch_kernel(ada_norm_kernel<bf16>, dim3(rows), dim3(256), 0, st, 1, a);
+  return launch_kernel(ada_norm_kernel<float>, dim3(rows), dim3(256), 0, st, 1, a);
 }
 
 // ============================================================================ in-proj
 
 __global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, const float* __restrict__ in_w,
                                const float* __restrict__ in_b, float* __restrict__ x) {
-  const int r = blockIdx.x;
-  const float* a = buf + (size_t)r * A;
-  for (int c = threadIdx.x; c < D; c += blockDim.x) {
-    float acc = in_b[c];
-    for (int i = 0; i < A; ++i) acc = fmaf(a[i], in_w[(size_t)i * D + c], acc);
-    x[(size_t)r * D + c] = acc;
-  }
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ float arow[];   // the action row of this slot
+  const int r = blockIdx.y;
+  for (int i = threadIdx.x; i < A; i += blockDim.x) arow[i] = buf[(size_t)r * A + i];
+  __syncthreads();
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= D) return;
+  float acc = in_b[c];
+  for (int i = 0; i < A; ++i) acc = fmaf(arow[i], in_w[(size_t)i * D + c], acc);
+  x[(size_t)r * D + c] = acc;
 }
 
 cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b, float* x,
                            cudaStream_t st) {
   if (BH <= 0) return cudaSuccess;
-  in_proj_kernel<<<BH, 256, 0, st>>>(buf, A, D, in_w, in_b, x);
-  return cudaGetLastError();
+  return launch_kernel(in_proj_kernel, dim3((D + 255) / 256, BH), dim3(256), A * sizeof(float), st, 1, buf, A, D,
+                       in_w, in_b, x);
 }
 
 // ============================================================================ GeGLU
 
 template <typename T>
 __global__ void geglu_kernel(const float* __restrict__ GU, int M, int Fm, T* __restrict__ Hm) {
+  pdl_trigger();
+  pdl_wait();
   const size_t total = (size_t)M * Fm;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
     const int m = (int)(i / Fm), f = (int)(i % Fm);
@@ -253,11 +269,8 @@ cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cud
   const size_t total = (size_t)M * Fm;
   if (!total) return cudaSuccess;
   const int blocks = (int)((total + 255) / 256 < 8192 ? (total + 255) / 256 : 8192);
-  if (dt == DT_BF16)
-    geglu_kernel<bf16><<<blocks, 256, 0, st>>>(GU, M, Fm, (bf16*)Hm);
-  else
-    geglu_kernel<float><<<blocks, 256, 0, st>>>(GU, M, Fm, (float*)Hm);
-  return cudaGetLastError();
+  if (dt == DT_BF16) return launch_kernel(geglu_kernel<bf16>, dim3(blocks), dim3(256), 0, st, 1, GU, M, Fm, (bf16*)Hm);
+  return launch_kernel(geglu_kernel<float>, dim3(blocks), dim3(256), 0, st, 1, GU, M, Fm, (float*)Hm);
 }
 
 // ============================================================================ attention (SIMT)
@@ -270,6 +283,8 @@ constexpr int ATT_QT = 16, ATT_KT = 32, ATT_THREADS = 256;
 
 template <typename T>
 __global__ void __launch_bounds__(ATT_THREADS) attention_simt_kernel(AttnArgs a) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ float sm[];
   const int hd = a.hd;
   float* Qs = sm;                      // [QT][hd]
@@ -293,6 +308,7 @@ __global__ void __launch_bounds__(ATT_THREADS) attention_simt_kernel(AttnArgs a)
   const T* pv = (const T*)(slot ? a.ctx_v1 : a.ctx_v0) + ctx_off;
   const int kofs = a.Hq * hd + g * hd, vofs = (a.Hq + a.Hkv) * hd + g * hd;
   const int nk = P + a.F + a.H;
+  const int rpr = a.H + a.F;   // QKV rows per robot: H action slots, then F FOP tokens
   const float scale = rsqrtf((float)hd);
 
   for (int i = threadIdx.x; i < ATT_QT * hd; i += ATT_THREADS) {
@@ -300,7 +316,7 @@ __global__ void __launch_bounds__(ATT_THREADS) attention_simt_kernel(AttnArgs a)
     float v = 0.f;
     if (r < nrows) {
       const int j = r / G, h = g * G + r % G;
-      v = to_f32(qkv[(size_t)(b * a.H + j) * a.ld_qkv + h * hd + c]);
+      v = to_f32(qkv[(size_t)(b * rpr + j) * a.ld_qkv + h * hd + c]);
     }
     Qs[i] = v * scale;
   }
@@ -323,11 +339,11 @@ __global__ void __launch_bounds__(ATT_THREADS) attention_simt_kernel(AttnArgs a)
         kv = to_f32(pk[(size_t)key * hd + c]);
         vv = to_f32(pv[(size_t)key * hd + c]);
       } else if (key < P + a.F) {
-        const size_t row = (size_t)(a.B * a.H + b * a.F + (key - P)) * a.ld_qkv;
+        const size_t row = (size_t)(b * rpr + a.H + (key - P)) * a.ld_qkv;
         kv = to_f32(qkv[row + kofs + c]);
         vv = to_f32(qkv[row + vofs + c]);
       } else if (key < nk) {
-        const size_t row = (size_t)(b * a.H + (key - P - a.F)) * a.ld_qkv;
+        const size_t row = (size_t)(b * rpr + (key - P - a.F)) * a.ld_qkv;
         kv = to_f32(qkv[row + kofs + c]);
         vv = to_f32(qkv[row + vofs + c]);
       }
@@ -392,10 +408,8 @@ cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st) 
   const int G = a.Hq / a.Hkv;
   dim3 grid(a.B * a.Hkv, (a.H * G + ATT_QT - 1) / ATT_QT);
   const size_t smem = (size_t)(ATT_QT * a.hd + 2 * ATT_KT * a.hd + ATT_QT * ATT_KT) * sizeof(float);
-  if (dt == DT_BF16)
-    attention_simt_kernel<bf16><<<grid, ATT_THREADS, smem, st>>>(a);
-  else
-    attention_simt_kernel<float><<<grid, ATT_THREADS, smem, st>>>(a);
+  if (dt == DT_BF16) return launch_kernel(attention_simt_kernel<bf16>, grid, dim3(ATT_THREADS), smem, st, 1, a);
+  return launch_kernel(attention_simt_kernel<float>, grid, dim3(ATT_THREADS), smem, st, 1, a);
   return cudaGetLastError();
 }
 
@@ -405,6 +419,8 @@ cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st) 
 // slots shift forward, the last slot receives the Gaussian action of index
 // counters[b], and the counter advances.
 __global__ void tail_kernel(TailArgs a) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ float sa[];   // [H][A]
   const int b = blockIdx.x;
   const int H = a.H, A = a.A;
@@ -439,8 +455,7 @@ __global__ void tail_kernel(TailArgs a) {
 cudaError_t launch_tail(const TailArgs& a, cudaStream_t st) {
   if (a.B <= 0) return cudaSuccess;
   const size_t smem = (size_t)a.H * a.A * sizeof(float);
-  tail_kernel<<<a.B, 256, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(tail_kernel, dim3(a.B), dim3(256), smem, st, 1, a);
 }
 
 cudaError_t init_simt_kernels() {

@@ -163,7 +163,13 @@ ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int pre
   const size_t row = (size_t)prefix_len * c.head_dim * es;        // one (l, b, g) block of the source
   const size_t dpitch = (size_t)c.max_prefix * c.head_dim * es;  // the same block in the slot
   const size_t per_layer_src = (size_t)r->batch * c.n_kv_heads;
-  for (int which = 0; which < 2; ++which) {
+  if (p.use_tc_attn) {
+    // the tensor-core attention reads V transposed (keys contiguous)
+    RV_CUDA(r, launch_transpose_ctx_v(v, p.ctx_v[target], c.layers, r->batch, c.max_batch, c.n_kv_heads, prefix_len,
+                                      c.head_dim, p.pst, side),
+            "set_context: transpose V");
+  }
+  for (int which = 0; which < (p.use_tc_attn ? 1 : 2); ++which) {
     const char* src = (const char*)(which ? v : k);
     char* dst = (char*)(which ? p.ctx_v[target] : p.ctx_k[target]);
     for (int l = 0; l < c.layers; ++l) {

@@ -2,8 +2,11 @@
 // rolling action-expert step.
 #include "step.h"
 
+#include "launch.h"
+
 #include <cstdio>
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 
 namespace ravel {
@@ -107,7 +110,8 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->in_w, (size_t)A * D * 4); AL(p->in_b, D * 4);
   AL(p->fop_gamma, (size_t)L * D * 4);
   AL(p->out_b, A * 4);
-  const size_t ctx_bytes = (size_t)L * Bm * c.n_kv_heads * c.max_prefix * c.head_dim * es;
+  p->pst = (c.max_prefix + 7) / 8 * 8;
+  const size_t ctx_bytes = (size_t)L * Bm * c.n_kv_heads * p->pst * c.head_dim * es;
   for (int s = 0; s < 2; ++s) {
     AL(p->ctx_k[s], ctx_bytes);
     AL(p->ctx_v[s], ctx_bytes);
@@ -115,6 +119,7 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->ctx_state, 2 * sizeof(int));
   const size_t rows_c = (size_t)H + Bm, rows_a = (size_t)Bm * H, rows_y = (size_t)Bm * (H + F);
   AL(p->E, rows_c * D * es); AL(p->H1, rows_c * D * es); AL(p->HC, rows_c * D * es);
+  AL(p->omega, (size_t)(D / 2) * sizeof(double));
   AL(p->modv, rows_c * p->mod_dim * 4);
   AL(p->x, rows_a * D * 4);
   AL(p->Y, rows_y * D * es);
@@ -123,6 +128,10 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->GU, rows_a * 2 * Fm * 4);
   AL(p->Hm, rows_a * Fm * es);
   AL(p->V, rows_a * A * 4);
+  p->kvp = (H + F + 7) / 8 * 8;
+  AL(p->Vt, (size_t)Bm * c.n_kv_heads * c.head_dim * p->kvp * es);
+  p->attn_ws_bytes = (size_t)32 << 20;
+  AL(p->attn_ws, p->attn_ws_bytes);
   p->tcws.ws_bytes = (size_t)24 << 20;
   p->tcws.n_counters = 4096;
   AL(p->tcws.ws, p->tcws.ws_bytes);
@@ -140,6 +149,8 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   if (e == cudaSuccess && p->dt == DT_BF16) {
     e = init_tc_gemm();
     p->use_tc = (e == cudaSuccess);
+    if (e == cudaSuccess) e = init_attention_tc();
+    p->use_tc_attn = (e == cudaSuccess) && attention_tc_supported(c.head_dim, c.n_q_heads / c.n_kv_heads);
   }
   if (e != cudaSuccess) {
     *errs = std::string("allocation: ") + cudaGetErrorString(e);
@@ -159,6 +170,18 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
       *errs = "weight staging allocation failed";
       plan_destroy(p);
       return RAVEL_ENOMEM;
+    }
+  }
+  {
+    // embedding frequencies w_i = 2 pi / p_i, periods geometric from 4e-3 (i = 0) to 4 (i = D/2 - 1)
+    std::vector<double> om(D / 2);
+    for (int i = 0; i < D / 2; ++i) om[i] = 6.283185307179586 / (4e-3 * std::pow(1000.0, (double)i / (double)(D / 2 - 1)));
+    e = cudaMemcpy(p->omega, om.data(), om.size() * sizeof(double), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+      *errs = "embedding table upload failed";
+      if (staging) cudaFree(staging);
+      plan_destroy(p);
+      return RAVEL_ECUDA;
     }
   }
   Packer pk{p, wp, staging};
@@ -243,7 +266,12 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   auto rowp = [&](const void* base, size_t row, size_t ld) { return (const void*)((const char*)base + row * ld * es); };
 
   // conditioning: embeddings, the two MLPs, modulation (App. A.1)
-  RUN(KK_EMBED, launch_embed(io.slot_times, H, io.delta, B, D, p.E, dt, st));
+  struct PdlScope {   // the step's kernels after the first may overlap their predecessors
+    ~PdlScope() { pdl_enabled() = false; }
+  } pdl_scope;
+  pdl_enabled() = false;
+  RUN(KK_EMBED, launch_embed(io.slot_times, H, io.delta, B, D, p.omega, p.E, dt, st));
+  pdl_enabled() = p.use_pdl && !trace;
   RUN(KK_GEMM_COND, gemm(p.E, D, p.t_w1, H, D, D, EPI_STORE_SILU, p.H1, D, dt, p.t_b1));
   RUN(KK_GEMM_COND, gemm(rowp(p.E, H, D), D, p.d_w1, B, D, D, EPI_STORE_SILU, (void*)rowp(p.H1, H, D), D, dt, p.d_b1));
   RUN(KK_GEMM_COND, gemm(p.H1, D, p.t_w2, H, D, D, EPI_STORE, p.HC, D, dt, p.t_b2));
@@ -251,19 +279,39 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   RUN(KK_GEMM_MOD, gemm(p.HC, D, p.mod_w, H + B, p.mod_dim, D, EPI_STORE, p.modv, p.mod_dim, DT_F32, nullptr));
   // residual stream
   RUN(KK_IN_PROJ, launch_in_proj(io.buffer, B * H, A, D, p.in_w, p.in_b, p.x, st));
-  const int BH = B * H, BY = B * (H + (io.obs ? F : 0));
+  const int FF = io.obs ? F : 0;      // FOP tokens present in this step
+  const int RPR = H + FF;              // normed / QKV rows per robot: H slots, then the FOP tokens
+  const int BH = B * H, BY = B * RPR;
   for (int l = 0; l < L; ++l) {
-    NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, io.obs, F, p.fop_gamma + (size_t)l * D, p.Y};
+    NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, io.obs, F, p.fop_gamma + (size_t)l * D, p.Y, RPR};
     RUN(KK_NORM, launch_ada_norm(n1, dt, st));
-    RUN(KK_GEMM_QKV, gemm(p.Y, D, (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es, BY, p.nqkv, D, EPI_STORE, p.QKV, p.nqkv,
-             dt, nullptr));
-    AttnArgs at{p.QKV, p.nqkv, p.ctx_k[0], p.ctx_k[1], p.ctx_v[0], p.ctx_v[1], p.ctx_state, l, c.max_batch,
-                c.max_prefix, B, H, io.obs ? F : 0, c.n_q_heads, c.n_kv_heads, c.head_dim, c.mask_mode, p.O, p.qdim,
-                p.err};
-    RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
+    const void* wqkv = (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es;
+    if (p.use_tc_attn) {
+      // QKV projection also writes V transposed (keys contiguous) for the tensor-core attention
+      GemmArgs gq{p.Y, D, wqkv, D, BY, p.nqkv, D, EPI_STORE, p.QKV, p.nqkv, dt, nullptr};
+      gq.vt = p.Vt;
+      gq.v_col0 = (c.n_q_heads + c.n_kv_heads) * c.head_dim;
+      gq.vt_hd = c.head_dim;
+      gq.vt_tokens = RPR;
+      gq.vt_kvp = p.kvp;
+      gq.vt_hkv = c.n_kv_heads;
+      RUN(KK_GEMM_QKV, run_gemm(p, gq, st));
+      AttnTcArgs at{p.QKV, p.nqkv, p.Vt, p.kvp, {p.ctx_k[0], p.ctx_k[1]}, {p.ctx_v[0], p.ctx_v[1]}, L, l,
+                    c.max_batch, c.max_prefix, p.pst, p.ctx_state, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim,
+                    c.mask_mode, p.O, p.qdim, p.attn_ws, p.attn_ws_bytes, p.err, p.num_sms};
+      int launched = 0;
+      at.n_launched = &launched;
+      RUN(KK_ATTENTION, launch_attention_tc(at, st));
+      nk += launched - 1;   // RUN counted one launch; a split attention adds its combine kernel
+    } else {
+      RUN(KK_GEMM_QKV, gemm(p.Y, D, wqkv, BY, p.nqkv, D, EPI_STORE, p.QKV, p.nqkv, dt, nullptr));
+      AttnArgs at{p.QKV, p.nqkv, p.ctx_k[0], p.ctx_k[1], p.ctx_v[0], p.ctx_v[1], p.ctx_state, l, c.max_batch,
+                  c.max_prefix, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim, c.mask_mode, p.O, p.qdim, p.err};
+      RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
+    }
     RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x, D,
              DT_F32, nullptr));
-    NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y};
+    NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y, H};
     RUN(KK_NORM, launch_ada_norm(n2, dt, st));
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
     GemmArgs gu{p.Y, D, wgu, D, BH, 2 * Fm, D, EPI_GEGLU, p.Hm, Fm, dt, nullptr};
@@ -276,7 +324,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D, DT_F32,
              nullptr));
   }
-  NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y};
+  NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y, H};
   RUN(KK_NORM, launch_ada_norm(nf, dt, st));
   RUN(KK_GEMM_OUT, gemm(p.Y, D, p.out_w, BH, A, D, EPI_STORE, p.V, A, DT_F32, p.out_b));
   TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A};

@@ -33,11 +33,14 @@ struct StepPlan {
   float *t_b1 = nullptr, *t_b2 = nullptr, *d_b1 = nullptr, *d_b2 = nullptr, *mod_b = nullptr;
   float *in_w = nullptr, *in_b = nullptr, *fop_gamma = nullptr, *out_b = nullptr;
   // VLM context double buffer [2] x [L][Bmax][Hkv][Pmax][hd] and its device state {active, len}
+  // (bf16 mode: ctx_v holds V transposed, [L][Bmax][Hkv][hd][pst], for the tensor-core attention)
   void* ctx_k[2] = {nullptr, nullptr};
   void* ctx_v[2] = {nullptr, nullptr};
+  int pst = 0;              // key pitch of the transposed context V (max_prefix rounded up to 8)
   int* ctx_state = nullptr;
   // activations
   void* E = nullptr;      // [H+Bmax][D]  sinusoidal embeddings (times, then offsets)
+  double* omega = nullptr;   // [D/2] angular frequencies of the embedding
   void* H1 = nullptr;     // [H+Bmax][D]  first MLP layer (SiLU)
   void* HC = nullptr;     // [H+Bmax][D]  MLP outputs h_t, h_delta
   float* modv = nullptr;  // [H+Bmax][mod_dim]  h @ W_mod (bias added in the norms)
@@ -48,6 +51,12 @@ struct StepPlan {
   float* GU = nullptr;    // [Bmax*H][2Fm]  interleaved gate/up (SIMT path)
   void* Hm = nullptr;     // [Bmax*H][Fm]
   float* V = nullptr;     // [Bmax*H][A]   velocity
+  void* Vt = nullptr;     // [Bmax][Hkv][hd][kvp]  transposed V of the FOP + slot keys (bf16 mode)
+  int kvp = 0;            // key pitch of Vt: (H + F) rounded up to 8
+  float* attn_ws = nullptr;  // split-KV partials of the tensor-core attention
+  size_t attn_ws_bytes = 0;
+  bool use_tc_attn = false;
+  bool use_pdl = true;      // Programmatic Dependent Launch between the step's kernels
   TcWorkspace tcws{};       // split-K workspace of the tensor-core GEMM
   int num_sms = 0;
   bool use_tc = false;      // bf16 projections on tcgen05
