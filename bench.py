@@ -38,6 +38,32 @@ import synth  # noqa: E402
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
+def csrc_sha() -> str:
+    """Hash of the CUDA sources: measured counters are valid only for the
+    kernels they were taken from."""
+    import glob
+    import hashlib
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2609_34170_gb300", "csrc", "*"))):
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(config: str, kind: str):
+    """DRAM bytes (read + write) per launch of `kind` from the committed ncu
+    capture, or None when absent or when the kernels changed since."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            t = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if t.get("csrc_sha") != csrc_sha():
+        return None
+    return t.get("bytes_per_launch", {}).get(config, {}).get(kind)
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -371,7 +397,8 @@ def main():
                           "frac_of_p50": step_roof_s * 1e6 / float(np.percentile(lat, 50) * 1e3),
                           "peaks": peak_src},
         "roofline": {"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                     "frac": (achieved / peak) if achieved else None, "traffic": None,
+                     "frac": (achieved / peak) if achieved else None,
+                     "traffic": measured_traffic(args.config, dom), "algorithmic_bytes": kb,
                      "launches_per_step": nlaunch, "avg_launch_us": avg_ms * 1e3,
                      "share_of_step": tot[dom] / grand, "peak_source": f"{peak_src} (MEASURED_PEAKS.json)"},
         "kernel_shares": {k: round(v / grand, 4) for k, v in sorted(tot.items(), key=lambda x: -x[1])},

@@ -85,8 +85,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   uint64_t* s_full = kv_empty + S;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
-  uint64_t* pv_done = p_full + 2;
-  uint32_t* tmem_slot = (uint32_t*)(pv_done + 1);
+  uint64_t* pv_done = p_full + 2;   // [2]: PV of chunk i completes pv_done[i & 1]
+  uint32_t* tmem_slot = (uint32_t*)(pv_done + 2);
   int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] issued, [2] consumed
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -123,7 +123,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       mbar_init(&s_free[i], 128);
       mbar_init(&p_full[i], 128);
     }
-    mbar_init(pv_done, 1);
+    mbar_init(&pv_done[0], 1);
+    mbar_init(&pv_done[1], 1);
     flags[0] = flags[1] = flags[2] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     uint64_t pol_kv;
@@ -199,6 +200,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       }
       flags[1] = i;
     }
+    __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc_s = idesc_bf16(AT_BM, AT_BKV);
@@ -238,11 +240,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
 #pragma unroll
         for (int k = 0; k < 4; ++k) umma_bf16(tmem + o_col, ad + 2 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
         umma_commit(&kv_empty[s]);
-        umma_commit(pv_done);
+        umma_commit(&pv_done[i & 1]);
       }
       if (!ok) flags[0] = 1;
       flags[2] = i;
     }
+    __syncwarp();
   } else {
     // softmax / epilogue: thread owns query row r (TMEM lane r)
     const int q4 = warp & 3;
@@ -251,40 +254,51 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     const int t = r / p.G, hh = r % p.G;
     const int j = qt * p.TQ + t;
     const bool row_ok = (r < q_rows) && (j < p.H);
-    float m_used = -INFINITY, l = 0.f;
+    float m_used = -INFINITY, l = 0.f;   // running max (log2 domain, scaled) and sum of P
     bool ok = true;
     int i = 0;
+    const float sl2 = p.scale_log2;
     for (int c = c0; c < c1 && ok; ++c) {
       if (c < p.n_pre && c * AT_BKV >= P) continue;
       ok = __all_sync(0xffffffffu, mbar_wait(&s_full[i & 1], (uint32_t)(i >> 1) & 1u));
       tc_fence_after();
       float sc[64];
+      {
+        uint32_t raw[64];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) tmem_ld16(lane_base + (uint32_t)(i & 1) * AT_BKV + 16 * q, sc + 16 * q);
+        for (int q = 0; q < 4; ++q) tmem_ld16_async(lane_base + (uint32_t)(i & 1) * AT_BKV + 16 * q, raw + 16 * q);
+        tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 64; ++k) sc[k] = __uint_as_float(raw[k]);
+      }
       tc_fence_before();
       mbar_arrive(&s_free[i & 1]);
-      // key validity
-      float mx = -INFINITY;
+      // keys of this chunk that exist (prefix shorter than the chunk, ragged
+      // FOP + slot chunk) and, in the slot-isolated test mode, that are visible
+      const int kk0 = (c < p.n_pre) ? c * AT_BKV : (c - p.n_pre) * AT_BKV;
+      const int kvalid = (c < p.n_pre) ? P - kk0 : rows_per_robot - kk0;
+      const bool iso = (p.mask_mode == 1) && (c >= p.n_pre) && (kk0 < p.H);
+      if (kvalid < AT_BKV || iso) {
 #pragma unroll
-      for (int k = 0; k < 64; ++k) {
-        bool v;
-        if (c < p.n_pre) {
-          v = c * AT_BKV + k < P;
-        } else {
-          const int kk = (c - p.n_pre) * AT_BKV + k;
-          v = kk < rows_per_robot;
-          if (p.mask_mode == 1 && kk < p.H) v = v && (kk == j);
+        for (int k = 0; k < 64; ++k) {
+          bool v = k < kvalid;
+          if (iso && kk0 + k < p.H) v = v && (kk0 + k == j);
+          if (!v) sc[k] = -INFINITY;
         }
-        sc[k] = v ? sc[k] * p.scale_log2 : -INFINITY;
-        mx = fmaxf(mx, sc[k]);
       }
-      if (i > 0) {
-        ok = __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(i - 1) & 1u)) && ok;
-        tc_fence_after();
-      }
+      float m8[8];
+#pragma unroll
+      for (int a = 0; a < 8; ++a)
+        m8[a] = fmaxf(fmaxf(fmaxf(sc[8 * a], sc[8 * a + 1]), fmaxf(sc[8 * a + 2], sc[8 * a + 3])),
+                      fmaxf(fmaxf(sc[8 * a + 4], sc[8 * a + 5]), fmaxf(sc[8 * a + 6], sc[8 * a + 7])));
+      const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                             fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7]))) * sl2;
       const float m_new = fmaxf(m_used, mx);
       const bool need = m_new > m_used + 8.f;
       if (i > 0 && __any_sync(0xffffffffu, need)) {
+        // O must hold PV of every earlier chunk before it is rescaled
+        ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(i - 1) & 1], (uint32_t)((i - 1) >> 1) & 1u)) && ok;
+        tc_fence_after();
         const float alpha = need ? exp2f(m_used - m_new) : 1.f;   // exp2(-inf) = 0
         for (int cb = 0; cb < p.hdp; cb += 16) {
           float o[16];
@@ -297,27 +311,33 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         l *= alpha;
       }
       if (need) m_used = m_new;
-      const float base = (m_used == -INFINITY) ? 0.f : m_used;
+      const float nb = (m_used == -INFINITY) ? 0.f : -m_used;
+      // the P buffer of this chunk was last read by PV of chunk i - 2
+      if (i >= 2) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[i & 1], (uint32_t)((i - 2) >> 1) & 1u)) && ok;
+        tc_fence_after();
+      }
       uint8_t* prow = p_s + (size_t)(i & 1) * AT_PBUF + (size_t)r * 128;
+      float ls[8];
 #pragma unroll
       for (int ch = 0; ch < 8; ++ch) {
+        float e[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) e[q] = fast_exp2(fmaf(sc[8 * ch + q], sl2, nb));
+        ls[ch] = ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
         uint32_t w[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const bf16 lo = __float2bfloat16_rn(exp2f(sc[8 * ch + 2 * q] - base));
-          const bf16 hi = __float2bfloat16_rn(exp2f(sc[8 * ch + 2 * q + 1] - base));
-          l += __bfloat162float(lo) + __bfloat162float(hi);
-          w[q] = (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
-        }
+        for (int q = 0; q < 4; ++q) w[q] = pack_bf16x2(e[2 * q], e[2 * q + 1]);
         *(uint4*)(prow + ((ch ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
       }
+      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
       mbar_arrive(&p_full[i & 1]);
       ++i;
     }
     if (ok && n > 0) {
-      ok = __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(n - 1) & 1u));
+      ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(n - 1) & 1], (uint32_t)((n - 1) >> 1) & 1u));
       tc_fence_after();
     }
     if (!ok && lane == 0) flags[0] = 1;

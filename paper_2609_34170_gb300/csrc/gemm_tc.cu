@@ -224,6 +224,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       }
       flags[2] = i;
     }
+    __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(TC_BM, BN);
@@ -246,6 +247,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       flags[3] = i;
       umma_commit(accb);   // arrives once every MMA issued above has completed
     }
+    __syncwarp();
   } else {
     // epilogue warps 2..5: TMEM lane quarter q = warp % 4, tile row r
     const int q = warp & 3;
