@@ -58,7 +58,7 @@ enum { RAVEL_MASK_FULL = 0, RAVEL_MASK_SLOT_ISOLATED = 1 };
 /* Shape of the expert and capacity of the handle. */
 typedef struct {
   int layers;       /* L */
-  int width;        /* D, even */
+  int width;        /* D, a multiple of 8, at most 4096 */
   int n_q_heads;    /* Hq, a multiple of n_kv_heads */
   int n_kv_heads;   /* Hkv */
   int head_dim;     /* hd, a multiple of 8, at most 256 */

@@ -16,7 +16,10 @@
 // grows by more than 2^8 (the kept maximum is exact for the final
 // normalisation, so this is not an approximation).
 // At batch 1 a (b, g) pair has only a few query tiles, so the key chunks are
-// split over grid.z and a combine kernel merges the partial (O, m, l).
+// split over grid.z; the splits of a query tile form a thread-block cluster,
+// publish their partial (O, m, l) through L2 and each rank merges a slice of
+// the head dimension after the cluster barrier.  The producer keeps the L2
+// warm a few prefix chunks ahead of its loads.
 //
 // Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator + MMA
 // issuer, warps 2..5 softmax / epilogue (warp w owns TMEM lanes 32*(w%4)..).
@@ -61,6 +64,22 @@ struct AtParams {
 struct AtMaps {
   CUtensorMap q, k, vt, pk0, pk1, pv0, pv1;
 };
+
+// The idx-th chunk this CTA processes (prefix chunks past the valid prefix
+// length are skipped), or -1.
+__device__ __forceinline__ int chunk_at(const AtParams& p, int P, int c0, int c1, int idx) {
+  const int pre_end = min(min(c1, p.n_pre), (P + AT_BKV - 1) / AT_BKV);
+  const int npre = max(0, pre_end - c0);
+  if (idx < npre) return c0 + idx;
+  const int c = max(c0, p.n_pre) + (idx - npre);
+  return c < c1 ? c : -1;
+}
+
+__device__ __forceinline__ void prefetch_l2_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(map), "r"(x), "r"(y),
+               "r"(z)
+               : "memory");
+}
 
 __device__ __forceinline__ int chunk_count(const AtParams& p, int P, int c0, int c1) {
   int n = 0;
@@ -140,6 +159,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       tma_load_3d(pv, &kv_full[npre], ks + k_bytes, c_next * AT_BKV, 0, ctx_z, pol_kv);
       ++npre;
     }
+    // and warm L2 with the prefix chunks that will refill those stages
+    for (int k = 0; k < S; ++k) {
+      const int c = chunk_at(p, P, c0, c1, npre + k);
+      if (c < 0 || c >= p.n_pre) break;
+      for (int blk = 0; blk < p.nblk; ++blk) prefetch_l2_3d(pk, blk * 64, c * AT_BKV, ctx_z);
+      prefetch_l2_3d(pv, c * AT_BKV, 0, ctx_z);
+    }
   }
   // rows of the Q tile that no query fills are zeroed (their scores are unused)
   const int q_rows = p.TQ * p.G;
@@ -195,6 +221,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
             tma_load_3d(&maps.k, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, b * rows_per_robot + cc * AT_BKV,
                         pol_q);
           tma_load_3d(&maps.vt, &kv_full[s], vs, cc * AT_BKV, 0, b * p.Hkv + g, pol_q);
+        }
+        {   // keep the L2 warm S chunks ahead of the loads (prefix chunks only)
+          const int cf = chunk_at(p, P, c0, c1, i + 2 * S);
+          if (cf >= 0 && cf < p.n_pre) {
+            for (int blk = 0; blk < p.nblk; ++blk) prefetch_l2_3d(pk, blk * 64, cf * AT_BKV, ctx_z);
+            prefetch_l2_3d(pv, cf * AT_BKV, 0, ctx_z);
+          }
         }
         ++i;
       }
@@ -355,18 +388,22 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         }
       }
     } else {
-      // partial tile, column-major ([d][row]) so that a warp's stores are contiguous
-      const int cta = bg * gridDim.x + qt;
-      const size_t ti = (size_t)split * gridDim.x * gridDim.y + cta;
+      // unnormalised partial O as [ti][d/4][row][4] (a warp stores one
+      // contiguous 512-byte run per 4 columns), plus this split's (m, l)
+      const size_t ti = ((size_t)bg * gridDim.x + qt) * p.splits + split;
+      float* dst = p.ws_o + ti * (size_t)(p.hdp / 4) * 512 + (size_t)r * 4;
       for (int cb = 0; cb < p.hdp; cb += 16) {
         float o[16];
         tmem_ld16(lane_base + o_col + cb, o);
-        float* dst = p.ws_o + (ti * p.hdp + cb) * AT_BM + r;
 #pragma unroll
-        for (int q = 0; q < 16; ++q) dst[(size_t)q * AT_BM] = (n > 0) ? o[q] : 0.f;
+        for (int q = 0; q < 4; ++q)
+          __stcg((float4*)(dst + (size_t)(cb / 4 + q) * 512),
+                 (n > 0) ? make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3])
+                         : make_float4(0.f, 0.f, 0.f, 0.f));
       }
-      p.ws_ml[(ti * 2) * AT_BM + r] = (n > 0) ? m_used : -INFINITY;
-      p.ws_ml[(ti * 2 + 1) * AT_BM + r] = (n > 0) ? l : 0.f;
+      __stcg(p.ws_ml + (ti * 2) * AT_BM + r, (n > 0) ? m_used : -INFINITY);
+      __stcg(p.ws_ml + (ti * 2 + 1) * AT_BM + r, (n > 0) ? l : 0.f);
+      __threadfence();
     }
   }
   tc_fence_before();
@@ -378,58 +415,77 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
     __syncthreads();
   }
+  if (p.splits > 1) {
+    // The key splits of this query tile form a cluster: once every split has
+    // published its (O, m, l), rank q merges head-dim columns
+    // [q*hdp/S, (q+1)*hdp/S):  O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
+    cluster_sync();
+    if (warp >= 2) {
+      const int r = (warp & 3) * 32 + lane;
+      const int Sp = p.splits;
+      const int cps = p.hdp / Sp;   // a multiple of 4
+      const int rank = (int)cluster_ctarank();
+      const size_t t0 = ((size_t)bg * gridDim.x + qt) * Sp;
+      float wgt[16];
+      float M = -INFINITY, L = 0.f;
+#pragma unroll
+      for (int s2 = 0; s2 < 16; ++s2) {
+        wgt[s2] = (s2 < Sp) ? __ldcg(p.ws_ml + ((t0 + s2) * 2) * AT_BM + r) : -INFINITY;
+        M = fmaxf(M, wgt[s2]);
+      }
+#pragma unroll
+      for (int s2 = 0; s2 < 16; ++s2) {
+        const float l_s = (s2 < Sp) ? __ldcg(p.ws_ml + ((t0 + s2) * 2 + 1) * AT_BM + r) : 0.f;
+        wgt[s2] = (wgt[s2] == -INFINITY) ? 0.f : exp2f(wgt[s2] - M);
+        L += wgt[s2] * l_s;
+      }
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      const int t = r / p.G, hh = r % p.G;
+      const int j = qt * p.TQ + t;
+      const bool row_ok = (r < p.TQ * p.G) && (j < p.H);
+      bf16* orow = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
+      for (int c4 = rank * cps / 4; c4 < (rank + 1) * cps / 4; c4 += 4) {
+        float4 acc[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int s2 = 0; s2 < Sp; ++s2) {
+          const float* src = p.ws_o + (t0 + s2) * (size_t)(p.hdp / 4) * 512 + (size_t)r * 4;
+          float4 x[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            x[k] = (c4 + k < (rank + 1) * cps / 4) ? __ldcg((const float4*)(src + (size_t)(c4 + k) * 512))
+                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+          const float w = wgt[s2 < 16 ? s2 : 15];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            acc[k].x += w * x[k].x;
+            acc[k].y += w * x[k].y;
+            acc[k].z += w * x[k].z;
+            acc[k].w += w * x[k].w;
+          }
+        }
+        if (row_ok) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int d = 4 * (c4 + k);
+            if (c4 + k >= (rank + 1) * cps / 4) break;
+            const float o4[4] = {acc[k].x * inv, acc[k].y * inv, acc[k].z * inv, acc[k].w * inv};
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              if (d + e < p.hd) orow[d + e] = __float2bfloat16_rn(o4[e]);
+          }
+        }
+      }
+    }
+  }
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
   }
 }
 
-// Merge the split partials: O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
-// Block = (tile, 8 head-dim columns), thread = tile row; the column-major
-// partials make every load of a warp contiguous.
-__global__ void attn_combine_kernel(AtParams p, int nctas) {
-  pdl_trigger();
-  pdl_wait();
-  const int cta = blockIdx.x, d0 = blockIdx.y * 8, r = threadIdx.x;
-  const int qt = cta % p.q_tiles, bg = cta / p.q_tiles;
-  const int b = bg / p.Hkv, g = bg % p.Hkv;
-  const int t = r / p.G, hh = r % p.G;
-  const int j = qt * p.TQ + t;
-  if (r >= p.TQ * p.G || j >= p.H) return;
-  const int S = p.splits;   // <= 64
-  float w[64];
-  float M = -INFINITY;
-#pragma unroll 8
-  for (int s = 0; s < S; ++s) {
-    w[s] = p.ws_ml[(((size_t)s * nctas + cta) * 2) * AT_BM + r];
-    M = fmaxf(M, w[s]);
-  }
-  float L = 0.f;
-#pragma unroll 8
-  for (int s = 0; s < S; ++s) {
-    const float l = p.ws_ml[(((size_t)s * nctas + cta) * 2 + 1) * AT_BM + r];
-    w[s] = (w[s] == -INFINITY) ? 0.f : exp2f(w[s] - M);
-    L += w[s] * l;
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  float acc[8];
-#pragma unroll
-  for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const float* src = p.ws_o + (((size_t)s * nctas + cta) * p.hdp + d0) * AT_BM + r;
-    float x[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) x[q] = (d0 + q < p.hdp) ? src[(size_t)q * AT_BM] : 0.f;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] += w[s] * x[q];
-  }
-  bf16* dst = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
-#pragma unroll
-  for (int q = 0; q < 8; ++q)
-    if (d0 + q < p.hd) dst[d0 + q] = __float2bfloat16_rn(acc[q] * inv);
-}
-
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
+int g_attn_max_cluster = 8;   // largest power-of-two cluster of key splits
 
 cudaError_t enc3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1_bytes,
                  uint64_t s2_bytes, uint32_t b0, uint32_t b1, uint32_t b2) {
@@ -454,7 +510,25 @@ cudaError_t init_attention_tc() {
     if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorSymbolNotFound;
     g_enc = (PFN_cuTensorMapEncodeTiled_v12000)fn;
   }
-  return cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM_MAX);
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM_MAX);
+  if (e != cudaSuccess) return e;
+  if (cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 1;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 16;
+    cfg.gridDim = dim3(1, 1, 16);
+    cfg.blockDim = dim3(AT_THREADS);
+    cfg.dynamicSmemBytes = AT_SMEM_MAX;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg) == cudaSuccess && n > 0) g_attn_max_cluster = 16;
+  }
+  cudaGetLastError();
+  return cudaSuccess;
 }
 
 bool attention_tc_supported(int hd, int G) { return hd % 8 == 0 && hd <= 256 && G >= 1 && G <= 128; }
@@ -481,9 +555,15 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   const int C = p.n_pre + p.n_kv;
   // split the key chunks only when the (b, g, q-tile) grid leaves most SMs
   // idle; about two chunks per split so S(i+1) overlaps the softmax of i
+  // the splits of a query tile form one cluster (power of two, <= 16) whose
+  // head-dim slices are multiples of 4 columns
   int splits = 1;
-  if (nctas * 2 <= a.num_sms) splits = std::min({(C + 1) / 2, std::max(1, a.num_sms / nctas), 64});
-  while (splits > 1 && (size_t)splits * nctas * AT_BM * (p.hdp + 2) * 4 > a.ws_bytes) --splits;
+  if (nctas * 2 <= a.num_sms) {
+    const int cap = std::min({(C + 1) / 2, std::max(1, a.num_sms / nctas), g_attn_max_cluster});
+    while (splits * 2 <= cap && (p.hdp / (splits * 2)) % 4 == 0 &&
+           (size_t)(splits * 2) * nctas * AT_BM * (p.hdp + 2) * 4 <= a.ws_bytes)
+      splits *= 2;
+  }
   p.splits = splits;
   p.ws_o = a.ws;
   p.ws_ml = a.ws + (size_t)splits * nctas * AT_BM * p.hdp;
@@ -513,12 +593,8 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   }
   if (e != cudaSuccess) return e;
   dim3 grid(p.q_tiles, a.B * a.Hkv, splits);
-  e = launch_kernel(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, 1, m, p);
+  e = launch_kernel(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, (unsigned)splits, m, p);
   if (a.n_launched) ++*a.n_launched;
-  if (e == cudaSuccess && splits > 1) {
-    e = launch_kernel(attn_combine_kernel, dim3(nctas, (p.hd + 7) / 8), dim3(AT_BM), 0, st, 1, p, nctas);
-    if (a.n_launched) ++*a.n_launched;
-  }
   return e;
 }
 

@@ -180,11 +180,27 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st) {
 
 // ============================================================================ adaRMSNorm
 
+__device__ __forceinline__ float4 ld4(const float* p) { return *(const float4*)p; }
+__device__ __forceinline__ float4 add3(float4 a, float4 b, float4 c) {
+  return make_float4(a.x + b.x + c.x, a.y + b.y + c.y, a.z + b.z + c.z, a.w + b.w + c.w);
+}
+__device__ __forceinline__ void st4(float* p, float4 v) { *(float4*)p = v; }
+__device__ __forceinline__ void st4(bf16* p, float4 v) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *(uint32_t*)&lo;
+  u.y = *(uint32_t*)&hi;
+  *(uint2*)p = u;
+}
+
+// One row per block.  Every load of the row (x, and for action rows the six
+// modulation vectors) is issued before the reduction, so the row costs one
+// memory round trip; D % 4 == 0 and D <= 4096 (4 float4 per thread).
 template <typename T>
 __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a) {
   pdl_trigger();
-  pdl_wait();
   __shared__ float red[32];
+  constexpr int G = 4;
   const int r = blockIdx.x;
   const int D = a.D;
   const int n_act = a.B * a.H;
@@ -194,29 +210,57 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a) {
   else
     yrow = (size_t)((r - n_act) / a.F) * a.row_pitch + a.H + (r - n_act) % a.F;
   T* Y = (T*)a.Y + yrow * D;
+  pdl_wait();
   if (r < n_act) {
     const int b = r / a.H, j = r % a.H;
     const float* x = a.x + (size_t)r * D;
-    float ss = 0.f;
-    for (int c = threadIdx.x; c < D; c += blockDim.x) ss += x[c] * x[c];
-    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
     const float* mt = a.modv + (size_t)j * a.mod_ld + a.off;
     const float* md = a.modv + (size_t)(a.H + b) * a.mod_ld + a.off;
     const float* mb = a.mod_b + a.off;
-    for (int c = threadIdx.x; c < D; c += blockDim.x) {
-      const float sc = mt[c] + md[c] + mb[c];
-      const float sh = mt[D + c] + md[D + c] + mb[D + c];
-      Y[c] = from_f32<T>(x[c] * inv * (1.f + sc) + sh);
+    float4 xv[G], sc[G], sh[G];
+    float ss = 0.f;
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int c = 4 * (threadIdx.x + 256 * g);
+      if (c < D) {
+        xv[g] = ld4(x + c);
+        sc[g] = add3(ld4(mt + c), ld4(md + c), ld4(mb + c));
+        sh[g] = add3(ld4(mt + D + c), ld4(md + D + c), ld4(mb + D + c));
+        ss += xv[g].x * xv[g].x + xv[g].y * xv[g].y + xv[g].z * xv[g].z + xv[g].w * xv[g].w;
+      }
+    }
+    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int c = 4 * (threadIdx.x + 256 * g);
+      if (c < D)
+        st4(Y + c, make_float4(xv[g].x * inv * (1.f + sc[g].x) + sh[g].x, xv[g].y * inv * (1.f + sc[g].y) + sh[g].y,
+                               xv[g].z * inv * (1.f + sc[g].z) + sh[g].z, xv[g].w * inv * (1.f + sc[g].w) + sh[g].w));
     }
   } else {
     const T* z = (const T*)a.fop + (size_t)(r - n_act) * D;
+    float zv[4 * G], gm[4 * G];
     float ss = 0.f;
-    for (int c = threadIdx.x; c < D; c += blockDim.x) {
-      const float v = to_f32(z[c]);
-      ss += v * v;
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int c = 4 * (threadIdx.x + 256 * g);
+      if (c < D) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          zv[4 * g + q] = to_f32(z[c + q]);
+          gm[4 * g + q] = a.gamma[c + q];
+          ss += zv[4 * g + q] * zv[4 * g + q];
+        }
+      }
     }
     const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
-    for (int c = threadIdx.x; c < D; c += blockDim.x) Y[c] = from_f32<T>(to_f32(z[c]) * inv * (1.f + a.gamma[c]));
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int c = 4 * (threadIdx.x + 256 * g);
+      if (c < D)
+        st4(Y + c, make_float4(zv[4 * g] * inv * (1.f + gm[4 * g]), zv[4 * g + 1] * inv * (1.f + gm[4 * g + 1]),
+                               zv[4 * g + 2] * inv * (1.f + gm[4 * g + 2]), zv[4 * g + 3] * inv * (1.f + gm[4 * g + 3])));
+    }
   }
 }
 

@@ -16,7 +16,8 @@ bool validate_config(const ravel_config& c, std::string* why) {
     *why = m;
     return false;
   };
-  if (c.layers < 1 || c.width < 4 || c.width % 2) return bad("layers >= 1 and an even width >= 4 are required");
+  if (c.layers < 1 || c.width < 8 || c.width % 8 || c.width > 4096)
+    return bad("layers >= 1 and a width that is a multiple of 8 in [8, 4096] are required");
   if (c.n_q_heads < 1 || c.n_kv_heads < 1 || c.n_q_heads % c.n_kv_heads)
     return bad("n_q_heads must be a positive multiple of n_kv_heads");
   if (c.head_dim < 8 || c.head_dim > 256 || c.head_dim % 8) return bad("head_dim must be a multiple of 8 in [8, 256]");
