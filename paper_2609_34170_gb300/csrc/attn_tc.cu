@@ -51,6 +51,7 @@ struct AtParams {
   int Pmax, n_pre, n_kv, splits;
   int layer, Bmax, mask_mode;
   int nblk, stages;
+  int mc;                             // query tiles of a (b, g) pair sharing each K/V chunk by multicast (1 = none)
   uint32_t vt_bytes;                  // bytes of one transposed-V chunk (hd rows x 128 B)
   const int* ctx_state;
   bf16* out;
@@ -63,6 +64,7 @@ struct AtParams {
 
 struct AtMaps {
   CUtensorMap q, k, vt, pk0, pk1, pv0, pv1;
+  CUtensorMap vts, pvs0, pvs1;   // V^T boxes of hd/mc rows (multicast slices)
 };
 
 // The idx-th chunk this CTA processes (prefix chunks past the valid prefix
@@ -135,7 +137,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     mbar_init(q_full, 1);
     for (int s = 0; s < S; ++s) {
       mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&kv_empty[s], p.mc);   // released by the PV commit of every CTA sharing the chunk
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
@@ -146,17 +148,45 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     mbar_init(&pv_done[1], 1);
     flags[0] = flags[1] = flags[2] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  // with multicast, every CTA's barriers must exist before a peer targets them
+  if (p.mc > 1) cluster_sync();
+  const int mrank = (p.mc > 1) ? (int)cluster_ctarank() : 0;
+  const uint16_t mmask = (uint16_t)((1u << p.mc) - 1u);
+  const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
+  const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
+  const CUtensorMap* pvs = slot ? &maps.pvs1 : &maps.pvs0;
+  // K and V^T of chunk c into stage s: all of it, or (multicast) this CTA's
+  // share -- head-dim blocks rank, rank+mc, .. of K and V^T rows
+  // [rank*hd/mc, (rank+1)*hd/mc) -- sent to every CTA of the cluster
+  auto load_chunk = [&](int c, int s, uint64_t pol) {
+    uint8_t* ks = kv_s + (size_t)s * stage_bytes;
+    mbar_expect_tx(&kv_full[s], k_bytes + 128u * (uint32_t)p.hd);   // the whole chunk, whoever sends it
+    const bool pre = c < p.n_pre;
+    const int cc = c - p.n_pre;
+    const CUtensorMap* km = pre ? pk : &maps.k;
+    const int ky = pre ? c * AT_BKV : g, kz = pre ? ctx_z : b * rows_per_robot + cc * AT_BKV;
+    const int vx = (pre ? c : cc) * AT_BKV, vz = pre ? ctx_z : b * p.Hkv + g;
+    if (p.mc == 1) {
+      for (int blk = 0; blk < p.nblk; ++blk)
+        if (pre) tma_load_3d(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, pol);
+        else tma_load_3d(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, kz, pol);
+      tma_load_3d(pre ? pv : &maps.vt, &kv_full[s], ks + k_bytes, vx, 0, vz, pol);
+    } else {
+      for (int blk = mrank; blk < p.nblk; blk += p.mc)
+        if (pre) tma_load_3d_mc(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, mmask, pol);
+        else tma_load_3d_mc(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, kz, mmask, pol);
+      const int rows = p.hd / p.mc;
+      tma_load_3d_mc(pre ? pvs : &maps.vts, &kv_full[s], ks + k_bytes + (size_t)mrank * rows * 128, vx, mrank * rows,
+                     vz, mmask, pol);
+    }
+  };
+  if (threadIdx.x == 0) {
     uint64_t pol_kv;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_kv));
-    const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
-    const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
     for (; c_next < c1 && c_next < p.n_pre && npre < S; ++c_next) {
       if (c_next * AT_BKV >= P) continue;
-      uint8_t* ks = kv_s + (size_t)npre * stage_bytes;
-      mbar_expect_tx(&kv_full[npre], k_bytes + 128u * (uint32_t)p.hd);
-      for (int blk = 0; blk < p.nblk; ++blk)
-        tma_load_3d(pk, &kv_full[npre], ks + (size_t)blk * AT_KBLK, blk * 64, c_next * AT_BKV, ctx_z, pol_kv);
-      tma_load_3d(pv, &kv_full[npre], ks + k_bytes, c_next * AT_BKV, 0, ctx_z, pol_kv);
+      load_chunk(c_next, npre, pol_kv);
       ++npre;
     }
     // and warm L2 with the prefix chunks that will refill those stages
@@ -198,8 +228,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       for (int blk = 0; blk < p.nblk; ++blk)
         tma_load_3d(&maps.q, q_full, q_s + (size_t)blk * AT_QBLK, blk * 64, g * p.G, b * rows_per_robot + qt * p.TQ,
                     pol_q);
-      const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
-      const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
       int i = npre;
       for (int c = c_next; c < c1; ++c) {
         if (c < p.n_pre && c * AT_BKV >= P) continue;
@@ -208,20 +236,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           flags[0] = 1;
           break;
         }
-        uint8_t* ks = kv_s + (size_t)s * stage_bytes;
-        uint8_t* vs = ks + k_bytes;
-        mbar_expect_tx(&kv_full[s], k_bytes + 128u * (uint32_t)p.hd);   // V box: hd rows x 64 keys
-        if (c < p.n_pre) {
-          for (int blk = 0; blk < p.nblk; ++blk)
-            tma_load_3d(pk, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, c * AT_BKV, ctx_z, pol_kv);
-          tma_load_3d(pv, &kv_full[s], vs, c * AT_BKV, 0, ctx_z, pol_kv);
-        } else {
-          const int cc = c - p.n_pre;
-          for (int blk = 0; blk < p.nblk; ++blk)
-            tma_load_3d(&maps.k, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, b * rows_per_robot + cc * AT_BKV,
-                        pol_q);
-          tma_load_3d(&maps.vt, &kv_full[s], vs, cc * AT_BKV, 0, b * p.Hkv + g, pol_q);
-        }
+        load_chunk(c, s, c < p.n_pre ? pol_kv : pol_q);
         {   // keep the L2 warm S chunks ahead of the loads (prefix chunks only)
           const int cf = chunk_at(p, P, c0, c1, i + 2 * S);
           if (cf >= 0 && cf < p.n_pre) {
@@ -239,44 +254,55 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       const uint32_t idesc_s = idesc_bf16(AT_BM, AT_BKV);
       const uint32_t idesc_o = idesc_bf16(AT_BM, p.hdp);
       bool ok = mbar_wait(q_full, 0);
-      auto issue_s = [&](int j) -> bool {
-        const int s = j % S;
-        if (!mbar_wait(&kv_full[s], (uint32_t)(j / S) & 1u)) return false;
-        if (j >= 2 && !mbar_wait(&s_free[j & 1], (uint32_t)((j >> 1) - 1) & 1u)) return false;
-        tc_fence_after();
-        const uint8_t* ks = kv_s + (size_t)s * stage_bytes;
-        for (int blk = 0; blk < p.nblk; ++blk) {
-          const uint64_t ad = sw128_desc(smem_u32(q_s + (size_t)blk * AT_QBLK));
-          const uint64_t bd = sw128_desc(smem_u32(ks + (size_t)blk * AT_KBLK));
+      // Issue S of the next chunk and PV of the oldest chunk whose P is ready,
+      // whichever can go: PV(i) never waits for chunk i+1's K/V (that would
+      // chain every chunk's load behind the previous PV).  S runs at most one
+      // chunk ahead of PV (two S buffers in TMEM).
+      int ns = 0, i = 0;   // next S, next PV
+      unsigned long long t_last = globaltimer();
+      while (ok && i < n) {
+        bool progress = false;
+        if (ns < n && ns <= i + 1) {
+          const int s = ns % S;
+          if (mbar_test_wait(&kv_full[s], (uint32_t)(ns / S) & 1u) &&
+              (ns < 2 || mbar_test_wait(&s_free[ns & 1], (uint32_t)((ns >> 1) - 1) & 1u))) {
+            tc_fence_after();
+            const uint8_t* ks = kv_s + (size_t)s * stage_bytes;
+            for (int blk = 0; blk < p.nblk; ++blk) {
+              const uint64_t ad = sw128_desc(smem_u32(q_s + (size_t)blk * AT_QBLK));
+              const uint64_t bd = sw128_desc(smem_u32(ks + (size_t)blk * AT_KBLK));
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                umma_bf16(tmem + (uint32_t)(ns & 1) * AT_BKV, ad + 2 * k, bd + 2 * k, idesc_s,
+                          (blk > 0 || k > 0) ? 1u : 0u);
+            }
+            umma_commit(&s_full[ns & 1]);
+            ++ns;
+            progress = true;
+          }
+        }
+        if (i < ns && mbar_test_wait(&p_full[i & 1], (uint32_t)(i >> 1) & 1u)) {
+          tc_fence_after();
+          const int s = i % S;
+          const uint64_t ad = sw128_desc(smem_u32(p_s + (size_t)(i & 1) * AT_PBUF));
+          const uint64_t bd = sw128_desc(smem_u32(kv_s + (size_t)s * stage_bytes + k_bytes));
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_bf16(tmem + (uint32_t)(j & 1) * AT_BKV, ad + 2 * k, bd + 2 * k, idesc_s, (blk > 0 || k > 0) ? 1u : 0u);
+            umma_bf16(tmem + o_col, ad + 2 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
+          if (p.mc > 1) umma_commit_mc(&kv_empty[s], mmask);
+          else umma_commit(&kv_empty[s]);
+          umma_commit(&pv_done[i & 1]);
+          ++i;
+          progress = true;
         }
-        umma_commit(&s_full[j & 1]);
-        return true;
-      };
-      int i = 0;
-      if (ok && n > 0) ok = issue_s(0);
-      for (; ok && i < n; ++i) {
-        if (i + 1 < n && !issue_s(i + 1)) {
+        if (progress) {
+          t_last = globaltimer();
+        } else if (globaltimer() - t_last > kTcTimeoutNs) {
           ok = false;
-          break;
         }
-        if (!mbar_wait(&p_full[i & 1], (uint32_t)(i >> 1) & 1u)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const int s = i % S;
-        const uint64_t ad = sw128_desc(smem_u32(p_s + (size_t)(i & 1) * AT_PBUF));
-        const uint64_t bd = sw128_desc(smem_u32(kv_s + (size_t)s * stage_bytes + k_bytes));
-#pragma unroll
-        for (int k = 0; k < 4; ++k) umma_bf16(tmem + o_col, ad + 2 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
-        umma_commit(&kv_empty[s]);
-        umma_commit(&pv_done[i & 1]);
       }
       if (!ok) flags[0] = 1;
-      flags[2] = i;
+      flags[2] = ns;   // chunks whose K/V arrival was consumed
     }
     __syncwarp();
   } else {
@@ -482,6 +508,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
   }
+  // no CTA leaves while a peer may still multicast into it or arrive on its barriers
+  if (p.mc > 1) cluster_sync();
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
@@ -565,6 +593,10 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
       splits *= 2;
   }
   p.splits = splits;
+  // query tiles of a (b, g) pair share K/V chunks by multicast (clusters along x)
+  p.mc = 1;
+  if (splits == 1 && (p.q_tiles == 2 || p.q_tiles == 4) && p.nblk % p.q_tiles == 0 && (a.hd / p.q_tiles) % 8 == 0)
+    p.mc = p.q_tiles;
   p.ws_o = a.ws;
   p.ws_ml = a.ws + (size_t)splits * nctas * AT_BM * p.hdp;
   const uint32_t stage = (uint32_t)p.nblk * AT_KBLK + p.vt_bytes;
@@ -591,9 +623,16 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
       e = enc3(s ? &m.pv1 : &m.pv0, a.ctx_vt[s], a.Pmax, hd, zc, (uint64_t)a.pst * 2, (uint64_t)hd * a.pst * 2,
                AT_BKV, hd, 1);
   }
+  const uint32_t vrows = (uint32_t)(hd / p.mc);
+  if (e == cudaSuccess)
+    e = enc3(&m.vts, a.vt, rpr, hd, (uint64_t)a.B * a.Hkv, (uint64_t)a.kvp * 2, (uint64_t)hd * a.kvp * 2, AT_BKV,
+             vrows, 1);
+  for (int s = 0; s < 2 && e == cudaSuccess; ++s)
+    e = enc3(s ? &m.pvs1 : &m.pvs0, a.ctx_vt[s], a.Pmax, hd, zc, (uint64_t)a.pst * 2, (uint64_t)hd * a.pst * 2,
+             AT_BKV, vrows, 1);
   if (e != cudaSuccess) return e;
   dim3 grid(p.q_tiles, a.B * a.Hkv, splits);
-  e = launch_kernel(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, (unsigned)splits, m, p);
+  e = launch_kernel_cluster(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, dim3(p.mc, 1, splits), m, p);
   if (a.n_launched) ++*a.n_launched;
   return e;
 }

@@ -91,6 +91,32 @@ __device__ __forceinline__ bool work_item(const TcParams& p, int i, int& tn, int
   return true;
 }
 
+// dst[k] = bf16(vals[k] + add) for k < n (n <= 16), with 2-, 4-, 8- or
+// 16-byte stores as alignment allows.
+__device__ __forceinline__ void store_bf16_run(bf16* dst, const float* vals, int n, float add) {
+  int k = 0;
+  while (k < n) {
+    const uintptr_t a = (uintptr_t)(dst + k);
+    if ((a & 15) == 0 && n - k >= 8) {
+      *(uint4*)(dst + k) = make_uint4(pack_bf16x2(vals[k] + add, vals[k + 1] + add),
+                                      pack_bf16x2(vals[k + 2] + add, vals[k + 3] + add),
+                                      pack_bf16x2(vals[k + 4] + add, vals[k + 5] + add),
+                                      pack_bf16x2(vals[k + 6] + add, vals[k + 7] + add));
+      k += 8;
+    } else if ((a & 7) == 0 && n - k >= 4) {
+      *(uint2*)(dst + k) = make_uint2(pack_bf16x2(vals[k] + add, vals[k + 1] + add),
+                                      pack_bf16x2(vals[k + 2] + add, vals[k + 3] + add));
+      k += 4;
+    } else if ((a & 3) == 0 && n - k >= 2) {
+      *(uint32_t*)(dst + k) = pack_bf16x2(vals[k] + add, vals[k + 1] + add);
+      k += 2;
+    } else {
+      dst[k] = __float2bfloat16_rn(vals[k] + add);
+      k += 1;
+    }
+  }
+}
+
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 // v[4g + e] += sum over splits s = 0..S-1 (in order) of the partial of this
@@ -130,15 +156,21 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
 #pragma unroll
   for (int i = 0; i < 16; ++i) stage[i * STG_LD + r] = v[i];
   if (p.vt) {
+    // this thread's feature is one row d of V^T: its tokens m0.. are
+    // consecutive keys of at most two robots -> vectorised runs
     const int n = tile_n * TC_BM + r;
     if (n >= p.v_col0 && n < p.N) {
       const float bb = p.bias ? p.bias[n] : 0.f;
       const int g = (n - p.v_col0) / p.vt_hd, d = (n - p.v_col0) % p.vt_hd;
-      for (int i = 0; i < nc; ++i) {
+      const int nv = min(nc, p.M - m0);
+      int i = 0;
+      while (i < nv) {
         const int m = m0 + i;
-        if (m >= p.M) break;
         const int rb = m / p.vt_tokens, kk = m % p.vt_tokens;
-        p.vt[((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp + kk] = __float2bfloat16_rn(v[i] + bb);
+        const int run = min(nv - i, p.vt_tokens - kk);
+        bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp + kk;
+        store_bf16_run(dst, v + i, run, bb);
+        i += run;
       }
     }
   }
@@ -483,11 +515,25 @@ cudaError_t encode_2d(CUtensorMap* m, const void* base, int rows, int cols, int 
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-int pick_bn(int M) {
+// Token-tile width: the smallest of 32/64/96/128 that holds M; beyond 128
+// tokens, the multiple of 16 in [128, 256] whose tile count fills whole waves
+// of the SMs best (per-CTA work ~ waves x BN), larger BN on ties.
+int pick_bn(int M, int tiles_n, int num_sms) {
   const int cands[] = {32, 64, 96, 128};
   for (int c : cands)
     if (M <= c) return c;
-  return 256;
+  int best = 256;
+  long best_cost = -1;
+  for (int bn = 256; bn >= 128; bn -= 16) {
+    const long tiles = (long)tiles_n * ((M + bn - 1) / bn);
+    const long waves = (tiles + num_sms - 1) / num_sms;
+    const long cost = waves * bn;
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
 }
 
 int g_max_cluster = 8;   // largest power-of-two cluster the split-K reduction may use
@@ -529,8 +575,8 @@ bool tc_gemm_supported(const GemmArgs& g) {
 
 cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st, bool cluster) {
   if (!g_encode) return cudaErrorInitializationError;
-  const int bn = pick_bn(g.M);
   const int tiles_n = (g.N + TC_BM - 1) / TC_BM;
+  const int bn = pick_bn(g.M, tiles_n, num_sms);
   const int tiles_m = (g.M + bn - 1) / bn;
   const int num_kb = (g.K + TC_BK - 1) / TC_BK;
   const int tiles = tiles_n * tiles_m;
