@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
-  __syncthreads();
+  cta_sync();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t o_col = 128;
@@ -310,9 +310,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(q4 * 32) << 16);
-    const int t = r / p.G, hh = r % p.G;
+    const int t = r / p.G;
     const int j = qt * p.TQ + t;
-    const bool row_ok = (r < q_rows) && (j < p.H);
     float m_used = -INFINITY, l = 0.f;   // running max (log2 domain, scaled) and sum of P
     bool ok = true;
     int i = 0;
@@ -400,18 +399,40 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       tc_fence_after();
     }
     if (!ok && lane == 0) flags[0] = 1;
-    const int h = g * p.G + hh;
     if (p.splits == 1) {
-      const float inv = (l > 0.f) ? 1.f / l : 0.f;
-      for (int cb = 0; cb < p.hdp; cb += 16) {
-        float o[16];
-        tmem_ld16(lane_base + o_col + cb, o);
-        if (row_ok && n > 0) {
-          bf16* dst = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)h * p.hd + cb;
+      // O / l as bf16, staged row by row in the K/V stages (every chunk has
+      // been consumed and every MMA has completed, so nothing writes there
+      // any more), then stored by whole rows: a warp writes one output row of
+      // hd values per instruction instead of one value per lane.  16-byte
+      // column blocks are XOR-swizzled by row so that neither side conflicts.
+      const float inv = (l > 0.f && n > 0) ? 1.f / l : 0.f;
+      const int rbytes = (2 * p.hdp + 127) & ~127;   // whole 128-byte swizzle spans
+      uint8_t* srow = kv_s + (size_t)r * rbytes;
+      for (int cb = 0; cb < p.hdp; cb += 32) {
+        uint32_t raw[32];
+        tmem_ld16_async(lane_base + o_col + cb, raw);
+        tmem_ld16_async(lane_base + o_col + cb + 16, raw + 16);
+        tmem_wait_ld();
 #pragma unroll
-          for (int q = 0; q < 16; ++q)
-            if (cb + q < p.hd) dst[q] = __float2bfloat16_rn(o[q] * inv);
+        for (int q = 0; q < 4; ++q) {
+          uint4 w;
+          w.x = pack_bf16x2(__uint_as_float(raw[8 * q]) * inv, __uint_as_float(raw[8 * q + 1]) * inv);
+          w.y = pack_bf16x2(__uint_as_float(raw[8 * q + 2]) * inv, __uint_as_float(raw[8 * q + 3]) * inv);
+          w.z = pack_bf16x2(__uint_as_float(raw[8 * q + 4]) * inv, __uint_as_float(raw[8 * q + 5]) * inv);
+          w.w = pack_bf16x2(__uint_as_float(raw[8 * q + 6]) * inv, __uint_as_float(raw[8 * q + 7]) * inv);
+          const int blk = cb / 8 + q;
+          *(uint4*)(srow + ((blk ^ (r & 7)) << 4)) = w;
         }
+      }
+      __syncwarp();
+      const int nblk16 = p.hd / 8;   // 16-byte blocks of one output row
+      for (int rr = q4 * 32; rr < q4 * 32 + 32; ++rr) {
+        const int tt = rr / p.G, jj = qt * p.TQ + tt;
+        if (rr >= q_rows || jj >= p.H) break;   // rows are in token order
+        const uint8_t* sr = kv_s + (size_t)rr * rbytes;
+        bf16* dst = p.out + (size_t)(b * p.H + jj) * p.ld_out + (size_t)(g * p.G + rr % p.G) * p.hd;
+        for (int blk = lane; blk < nblk16; blk += 32)
+          *(uint4*)(dst + 8 * blk) = *(const uint4*)(sr + ((blk ^ (rr & 7)) << 4));
       }
     } else {
       // unnormalised partial O as [ti][d/4][row][4] (a warp stores one
@@ -433,13 +454,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
   }
   tc_fence_before();
-  __syncthreads();
+  cta_sync();
   if (flags[0]) {
     if (threadIdx.x == 0) {
       for (int i = flags[2]; i < flags[1]; ++i) mbar_wait(&kv_full[i % S], (uint32_t)(i / S) & 1u);
       raise_error(p.err, ERR_TIMEOUT);
     }
-    __syncthreads();
+    cta_sync();
   }
   if (p.splits > 1) {
     // The key splits of this query tile form a cluster: once every split has
@@ -474,14 +495,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         float4 acc[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s2 = 0; s2 < Sp; ++s2) {
+#pragma unroll
+        for (int s2 = 0; s2 < 16; ++s2) {
+          if (s2 >= Sp) break;
           const float* src = p.ws_o + (t0 + s2) * (size_t)(p.hdp / 4) * 512 + (size_t)r * 4;
           float4 x[4];
 #pragma unroll
           for (int k = 0; k < 4; ++k)
             x[k] = (c4 + k < (rank + 1) * cps / 4) ? __ldcg((const float4*)(src + (size_t)(c4 + k) * 512))
                                                    : make_float4(0.f, 0.f, 0.f, 0.f);
-          const float w = wgt[s2 < 16 ? s2 : 15];
+          const float w = wgt[s2];
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             acc[k].x += w * x[k].x;
@@ -603,6 +626,10 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   const size_t fixed = 1024 + (size_t)p.nblk * AT_QBLK + 2 * AT_PBUF + 256;
   int stages = (int)std::min<size_t>(4, (AT_SMEM_MAX - fixed) / stage);
   if (stages < 1) return cudaErrorInvalidConfiguration;
+  // the epilogue stages 128 bf16 rows of O in the K/V stages and stores them
+  // with 16-byte writes
+  if ((size_t)AT_BM * (size_t)((2 * p.hdp + 127) & ~127) > (size_t)stages * stage) return cudaErrorInvalidConfiguration;
+  if (a.ld_out % 8 != 0 || ((uintptr_t)a.out & 15u) != 0) return cudaErrorMisalignedAddress;
   p.stages = stages;
   const size_t smem = fixed + (size_t)stages * stage;
 
@@ -651,7 +678,7 @@ __global__ void transpose_ctx_v_kernel(const bf16* __restrict__ src, bf16* __res
     const int pp = p0 + i, dd = d0 + threadIdx.x;
     tile[i][threadIdx.x] = (pp < P && dd < hd) ? s[(size_t)pp * hd + dd] : __float2bfloat16_rn(0.f);
   }
-  __syncthreads();
+  cta_sync();
   for (int i = threadIdx.y; i < 32; i += blockDim.y) {
     const int dd = d0 + i, pp = p0 + threadIdx.x;
     if (dd < hd && pp < P) d[(size_t)dd * pst + pp] = tile[threadIdx.x][i];

@@ -302,7 +302,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
-  __syncthreads();
+  cta_sync();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
@@ -447,14 +447,14 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     }
   }
   tc_fence_before();
-  __syncthreads();
+  cta_sync();
   if (flags[0]) {
     // unwind: wait (bounded) for the copies this CTA issued but never consumed
     if (threadIdx.x == 0) {
       for (int i = flags[3]; i < flags[2]; ++i) mbar_wait(&full[i % S], (uint32_t)(i / S) & 1u);
       raise_error(p.err, ERR_TIMEOUT);
     }
-    __syncthreads();
+    cta_sync();
   }
   if (p.reduce == RED_L2_CLUSTER && p.splits > 1) {
     // Every split of this tile has written its partial; the cluster barrier

@@ -199,7 +199,17 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 }
 
 // All threads of all CTAs of the cluster; release / acquire of shared memory.
+// CTA-wide barrier.  bar.sync is a warp-aligned instruction: a warp that
+// reaches it with some lanes still inside a single-lane branch is counted
+// early and puts every later phase of the barrier out of step, so each warp
+// reconverges first.
+__device__ __forceinline__ void cta_sync() {
+  __syncwarp();
+  __syncthreads();
+}
+
 __device__ __forceinline__ void cluster_sync() {
+  __syncwarp();
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
