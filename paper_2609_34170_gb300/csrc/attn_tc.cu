@@ -77,17 +77,46 @@ __device__ __forceinline__ int chunk_at(const AtParams& p, int P, int c0, int c1
   return c < c1 ? c : -1;
 }
 
-__device__ __forceinline__ void prefetch_l2_3d(const CUtensorMap* map, int x, int y, int z) {
-  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(map), "r"(x), "r"(y),
-               "r"(z)
-               : "memory");
-}
 
 __device__ __forceinline__ int chunk_count(const AtParams& p, int P, int c0, int c1) {
   int n = 0;
   for (int c = c0; c < c1; ++c)
     if (!(c < p.n_pre && c * AT_BKV >= P)) ++n;
   return n;
+}
+
+// Rows of the split-KV combine: out = sum_s wgt[s] * O_s * inv over float4
+// columns [c4b, c4e) of this thread's row, the SP partials of a column batch
+// loaded together (one L2 round trip per batch).  src0 points at split 0 of
+// the row; splits are sstride floats apart, float4 columns 512.
+template <int SP>
+__device__ __forceinline__ void combine_slice(const float* src0, size_t sstride, int c4b, int c4e, const float* wgt,
+                                              float inv, bf16* orow, int hd, bool row_ok) {
+  constexpr int KC = 32 / SP;
+  for (int c4 = c4b; c4 < c4e; c4 += KC) {
+    float4 x[SP][KC];
+#pragma unroll
+    for (int s2 = 0; s2 < SP; ++s2)
+#pragma unroll
+      for (int k = 0; k < KC; ++k)
+        x[s2][k] = (c4 + k < c4e) ? __ldcg((const float4*)(src0 + (size_t)s2 * sstride + (size_t)(c4 + k) * 512))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < KC; ++k) {
+      const int d = 4 * (c4 + k);
+      if (c4 + k >= c4e || d >= hd) break;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int s2 = 0; s2 < SP; ++s2) {
+        acc.x += wgt[s2] * x[s2][k].x;
+        acc.y += wgt[s2] * x[s2][k].y;
+        acc.z += wgt[s2] * x[s2][k].z;
+        acc.w += wgt[s2] * x[s2][k].w;
+      }
+      if (row_ok)   // hd % 8 == 0 and d % 4 == 0: all four columns exist; 8-byte aligned
+        *(uint2*)(orow + d) = make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+    }
+  }
 }
 
 __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_constant__ AtMaps maps, AtParams p) {
@@ -439,14 +468,20 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       // contiguous 512-byte run per 4 columns), plus this split's (m, l)
       const size_t ti = ((size_t)bg * gridDim.x + qt) * p.splits + split;
       float* dst = p.ws_o + ti * (size_t)(p.hdp / 4) * 512 + (size_t)r * 4;
-      for (int cb = 0; cb < p.hdp; cb += 16) {
-        float o[16];
-        tmem_ld16(lane_base + o_col + cb, o);
+      for (int cb = 0; cb < p.hdp; cb += 64) {   // up to four TMEM loads in flight, one wait
+        const int nq = min(4, (p.hdp - cb) / 16);
+        uint32_t raw[64];
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-          __stcg((float4*)(dst + (size_t)(cb / 4 + q) * 512),
-                 (n > 0) ? make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3])
-                         : make_float4(0.f, 0.f, 0.f, 0.f));
+          if (q < nq) tmem_ld16_async(lane_base + o_col + cb + 16 * q, raw + 16 * q);
+        tmem_wait_ld();
+#pragma unroll
+        for (int q = 0; q < 16; ++q)
+          if (q < 4 * nq)
+            __stcg((float4*)(dst + (size_t)(cb / 4 + q) * 512),
+                   (n > 0) ? make_float4(__uint_as_float(raw[4 * q]), __uint_as_float(raw[4 * q + 1]),
+                                         __uint_as_float(raw[4 * q + 2]), __uint_as_float(raw[4 * q + 3]))
+                           : make_float4(0.f, 0.f, 0.f, 0.f));
       }
       __stcg(p.ws_ml + (ti * 2) * AT_BM + r, (n > 0) ? m_used : -INFINITY);
       __stcg(p.ws_ml + (ti * 2 + 1) * AT_BM + r, (n > 0) ? l : 0.f);
@@ -491,39 +526,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       const int j = qt * p.TQ + t;
       const bool row_ok = (r < p.TQ * p.G) && (j < p.H);
       bf16* orow = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
-      for (int c4 = rank * cps / 4; c4 < (rank + 1) * cps / 4; c4 += 4) {
-        float4 acc[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int s2 = 0; s2 < 16; ++s2) {
-          if (s2 >= Sp) break;
-          const float* src = p.ws_o + (t0 + s2) * (size_t)(p.hdp / 4) * 512 + (size_t)r * 4;
-          float4 x[4];
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            x[k] = (c4 + k < (rank + 1) * cps / 4) ? __ldcg((const float4*)(src + (size_t)(c4 + k) * 512))
-                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-          const float w = wgt[s2];
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            acc[k].x += w * x[k].x;
-            acc[k].y += w * x[k].y;
-            acc[k].z += w * x[k].z;
-            acc[k].w += w * x[k].w;
-          }
-        }
-        if (row_ok) {
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const int d = 4 * (c4 + k);
-            if (c4 + k >= (rank + 1) * cps / 4) break;
-            const float o4[4] = {acc[k].x * inv, acc[k].y * inv, acc[k].z * inv, acc[k].w * inv};
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-              if (d + e < p.hd) orow[d + e] = __float2bfloat16_rn(o4[e]);
-          }
-        }
+      const float* src0 = p.ws_o + t0 * (size_t)(p.hdp / 4) * 512 + (size_t)r * 4;
+      const size_t sstride = (size_t)(p.hdp / 4) * 512;
+      const int c4b = rank * cps / 4, c4e = (rank + 1) * cps / 4;
+      switch (Sp) {
+        case 2: combine_slice<2>(src0, sstride, c4b, c4e, wgt, inv, orow, p.hd, row_ok); break;
+        case 4: combine_slice<4>(src0, sstride, c4b, c4e, wgt, inv, orow, p.hd, row_ok); break;
+        case 8: combine_slice<8>(src0, sstride, c4b, c4e, wgt, inv, orow, p.hd, row_ok); break;
+        default: combine_slice<16>(src0, sstride, c4b, c4e, wgt, inv, orow, p.hd, row_ok); break;
       }
     }
   }

@@ -22,16 +22,20 @@
 //    MMAs of the next;
 //  * few tiles: the K dimension is split over grid.z.  The splits of a tile
 //    form a thread-block cluster; each writes its fp32 partial to L2, the
-//    cluster barrier publishes them, and rank q sums a column slice over the
+//    cluster barrier publishes them, and rank q sums a token slice over the
 //    splits in order (deterministic) and applies the epilogue;
 //  * workspace mode (no cluster, for callers that bring their own scratch):
 //    the last split to arrive (per-tile counter) sums all partials.
-// The epilogue stages each 16-token chunk in shared memory so that global
-// stores are 16-byte row segments written by all 128 epilogue threads.
+// Epilogue: a chunk of tokens is written into a shared-memory box in the
+// output layout and leaves through one TMA store (or a TMA reduce-add for the
+// residual-stream epilogue), double-buffered so that the epilogue threads
+// never wait on global memory; the workspace mode (and unaligned outputs)
+// store from the threads instead.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstring>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -47,8 +51,10 @@ constexpr int TC_THREADS = 192;
 constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;
 constexpr int TC_SMEM_BUDGET = 200 * 1024;   // operand ring
 constexpr int TC_SMEM_MAX = 227 * 1024;
-constexpr int STG_LD = 132;                  // staging pitch (floats): 16 tokens x 128 tile rows
+constexpr int TC_RING_SPLIT = 128 * 1024;    // operand ring of a split-K launch
+constexpr int STG_LD = 132;                  // SIMT staging pitch (floats): 16 tokens x 128 tile rows
 constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
+constexpr uint32_t XCH_BYTES = STG_BYTES;        // GeGLU transpose tile (TMA epilogue)
 
 enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2 };
 
@@ -69,6 +75,12 @@ struct TcParams {
   int* err;
   bf16* vt;
   int v_col0, vt_hd, vt_tokens, vt_kvp, vt_hkv;
+  int tma_out;          // outputs leave through TMA boxes
+  int box_m;            // tokens per epilogue chunk (= rows of a TMA output box)
+  uint32_t box_bytes;   // bytes of one TMA output box (1024-aligned)
+  uint32_t stg_off;     // SIMT transpose tile, or two TMA output boxes
+  uint32_t xch_off;     // GeGLU exchange
+  uint32_t bar_off;     // mbarriers, TMEM slot, flags
 };
 
 // The i-th work item of this CTA: a tile (tn, tm) and split sp.  With splits
@@ -89,32 +101,6 @@ __device__ __forceinline__ bool work_item(const TcParams& p, int i, int& tn, int
   tn = t / p.tiles_m;
   sp = 0;
   return true;
-}
-
-// dst[k] = bf16(vals[k] + add) for k < n (n <= 16), with 2-, 4-, 8- or
-// 16-byte stores as alignment allows.
-__device__ __forceinline__ void store_bf16_run(bf16* dst, const float* vals, int n, float add) {
-  int k = 0;
-  while (k < n) {
-    const uintptr_t a = (uintptr_t)(dst + k);
-    if ((a & 15) == 0 && n - k >= 8) {
-      *(uint4*)(dst + k) = make_uint4(pack_bf16x2(vals[k] + add, vals[k + 1] + add),
-                                      pack_bf16x2(vals[k + 2] + add, vals[k + 3] + add),
-                                      pack_bf16x2(vals[k + 4] + add, vals[k + 5] + add),
-                                      pack_bf16x2(vals[k + 6] + add, vals[k + 7] + add));
-      k += 8;
-    } else if ((a & 7) == 0 && n - k >= 4) {
-      *(uint2*)(dst + k) = make_uint2(pack_bf16x2(vals[k] + add, vals[k + 1] + add),
-                                      pack_bf16x2(vals[k + 2] + add, vals[k + 3] + add));
-      k += 4;
-    } else if ((a & 3) == 0 && n - k >= 2) {
-      *(uint32_t*)(dst + k) = pack_bf16x2(vals[k] + add, vals[k + 1] + add);
-      k += 2;
-    } else {
-      dst[k] = __float2bfloat16_rn(vals[k] + add);
-      k += 1;
-    }
-  }
 }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -146,6 +132,28 @@ __device__ __forceinline__ void reduce_splits_l2(const float* b0, int S, size_t 
   }
 }
 
+// V^T side output of the QKV projection for tokens m0 .. m0+nv-1 of this
+// thread's tile row: token m -> (robot m / T, key m % T).
+__device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, int nv, int r, const float v[16]) {
+  const int n = tile_n * TC_BM + r;
+  if (n < p.v_col0 || n >= p.N) return;
+  const float bb = p.bias ? p.bias[n] : 0.f;
+  const int g = (n - p.v_col0) / p.vt_hd, d = (n - p.v_col0) % p.vt_hd;
+  int rb = m0 / p.vt_tokens, kk = m0 % p.vt_tokens;
+  bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    if (i < nv) {
+      dst[kk] = __float2bfloat16_rn(v[i] + bb);
+      if (++kk == p.vt_tokens) {
+        kk = 0;
+        ++rb;
+        dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
+      }
+    }
+  }
+}
+
 // Epilogue of tokens m0 .. m0+nc-1 (nc <= 16) of tile row block tile_n: v[i]
 // is this thread's tile row r at token m0+i.  All 128 epilogue threads call it
 // together.  The chunk is transposed through `stage` so that each thread then
@@ -155,25 +163,7 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
                                                const float v[16], float* stage) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) stage[i * STG_LD + r] = v[i];
-  if (p.vt) {
-    // this thread's feature is one row d of V^T: its tokens m0.. are
-    // consecutive keys of at most two robots -> vectorised runs
-    const int n = tile_n * TC_BM + r;
-    if (n >= p.v_col0 && n < p.N) {
-      const float bb = p.bias ? p.bias[n] : 0.f;
-      const int g = (n - p.v_col0) / p.vt_hd, d = (n - p.v_col0) % p.vt_hd;
-      const int nv = min(nc, p.M - m0);
-      int i = 0;
-      while (i < nv) {
-        const int m = m0 + i;
-        const int rb = m / p.vt_tokens, kk = m % p.vt_tokens;
-        const int run = min(nv - i, p.vt_tokens - kk);
-        bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp + kk;
-        store_bf16_run(dst, v + i, run, bb);
-        i += run;
-      }
-    }
-  }
+  if (p.vt) store_vt(p, tile_n, m0, min(nc, p.M - m0), r, v);
   epi_bar();
   const int c = r >> 3, fg = r & 7;
   const int m = m0 + c;
@@ -184,7 +174,11 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
       const int f0 = tile_n * 64 + fg * 8, nf = p.N / 2;
       float o[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) o[q] = gelu_tanh_f(srow[fg * 8 + q]) * srow[64 + fg * 8 + q];
+      for (int q = 0; q < 8; ++q) {
+        const int ng = tile_n * TC_BM + fg * 8 + q;   // gate row; its up row is ng + 64
+        const float bg = p.bias ? p.bias[ng] : 0.f, bu = p.bias ? p.bias[ng + 64] : 0.f;
+        o[q] = gelu_tanh_f(srow[fg * 8 + q] + bg) * (srow[64 + fg * 8 + q] + bu);
+      }
       bf16* dst = (bf16*)p.out + (size_t)m * p.ldo + f0;
       if (f0 + 8 <= nf && ((uintptr_t)dst & 15) == 0) {
         *(uint4*)dst = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
@@ -243,21 +237,87 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
   epi_bar();
 }
 
+// TMA epilogue of tokens m0 .. m0+box_m-1 of tile row block tile_n: v[i] is
+// this thread's tile row r at token m0+i, brow its bias.  All 128 epilogue
+// threads call it together.  The chunk is written into output box `ebuf` in
+// shared memory (token-major, as the output), and thread 64 sends the box
+// with one TMA store (EPI_ADD_F32: TMA reduce-add into the residual stream);
+// rows past M and columns past N are clipped by the tensor map.
+__device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* tmO, int tile_n, int m0, int r,
+                                             const float v[16], float brow, uint8_t* boxes, float* xch, int& ebuf) {
+  const int bm = p.box_m;
+  if (p.vt) store_vt(p, tile_n, m0, min(bm, p.M - m0), r, v);
+  // the box written two chunks ago must have been read by its TMA store
+  if (threadIdx.x == 64) bulk_wait_read<1>();
+  epi_bar();
+  uint8_t* box = boxes + (size_t)ebuf * p.box_bytes;
+  if (p.epi == EPI_GEGLU) {
+    // tile rows 0..63 are gate features, 64..127 the matching up features:
+    // transpose through xch so that every thread then forms 8 outputs of one
+    // token (the GELUs spread over all 128 threads)
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < bm) xch[i * STG_LD + r] = v[i] + brow;
+    epi_bar();
+    const int c = r >> 3, fg = r & 7;
+    if (c < bm) {
+      const float4* g4 = (const float4*)(xch + c * STG_LD + fg * 8);
+      const float4* u4 = (const float4*)(xch + c * STG_LD + 64 + fg * 8);
+      const float4 ga = g4[0], gb = g4[1], ua = u4[0], ub = u4[1];
+      *(uint4*)((bf16*)box + c * 64 + fg * 8) =
+          make_uint4(pack_bf16x2(gelu_tanh_f(ga.x) * ua.x, gelu_tanh_f(ga.y) * ua.y),
+                     pack_bf16x2(gelu_tanh_f(ga.z) * ua.z, gelu_tanh_f(ga.w) * ua.w),
+                     pack_bf16x2(gelu_tanh_f(gb.x) * ub.x, gelu_tanh_f(gb.y) * ub.y),
+                     pack_bf16x2(gelu_tanh_f(gb.z) * ub.z, gelu_tanh_f(gb.w) * ub.w));
+    }
+  } else if (p.out_bf16) {
+    bf16* o = (bf16*)box;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float x = v[i] + brow;
+      if (p.epi == EPI_STORE_SILU) x = silu_f(x);
+      if (i < bm) o[i * TC_BM + r] = __float2bfloat16_rn(x);
+    }
+  } else {
+    float* o = (float*)box;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float x = v[i] + brow;
+      if (p.epi == EPI_STORE_SILU) x = silu_f(x);
+      if (i < bm) o[i * TC_BM + r] = x;
+    }
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  epi_bar();
+  if (threadIdx.x == 64) {
+    if (p.epi == EPI_ADD_F32) tma_reduce_add_2d(tmO, box, tile_n * TC_BM, m0);
+    else tma_store_2d(tmO, box, p.epi == EPI_GEGLU ? tile_n * 64 : tile_n * TC_BM, m0);
+    bulk_commit();
+  }
+  ebuf ^= 1;
+}
+
+// RED = p.reduce, fixed per instantiation so that each reduction mode gets
+// its own register allocation.
+template <int RED>
 __global__ void __launch_bounds__(TC_THREADS, 2)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, TcParams p) {
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                   const __grid_constant__ CUtensorMap tmO, TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int BN = p.bn, S = p.stages;
   const uint32_t b_bytes = (uint32_t)BN * TC_BK * 2;
   uint8_t* a_s = smem;
   uint8_t* b_s = smem + (size_t)S * TC_A_BYTES;
-  uint64_t* full = (uint64_t*)(smem + p.ring_bytes);
+  uint8_t* stg_raw = smem + p.stg_off;
+  float* stage = (float*)stg_raw;
+  float* xch = (float*)(smem + p.xch_off);
+  uint64_t* full = (uint64_t*)(smem + p.bar_off);
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;      // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
   uint32_t* tmem_slot = (uint32_t*)(acc_empty + 2);
   int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] last split, [2] issued, [3] consumed
-  float* stage = (float*)(((uintptr_t)(flags + 4) + 15) & ~(uintptr_t)15);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t ncols = (p.splits > 1) ? p.acc_cols : 2 * p.acc_cols;
@@ -266,6 +326,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   const int kb0_first = (int)((long)sp0 * p.num_kb / p.splits);
   const int kb1_first = (int)((long)(sp0 + 1) * p.num_kb / p.splits);
   const int npre = has_work ? min(S, kb1_first - kb0_first) : 0;
+  const int cpr = BN / p.splits;   // tokens of the slice each split rank owns (a multiple of 4)
 
   pdl_trigger();
   uint64_t pol_w = 0, pol_x = 0;
@@ -285,12 +346,17 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     // tiles while the previous kernel is still finishing.
     asm volatile("prefetch.tensormap [%0];" ::"l"(&tmW) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(&tmX) : "memory");
+    if (p.tma_out) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
     for (int i = 0; i < npre; ++i) {
       mbar_expect_tx(&full[i], TC_A_BYTES + b_bytes);
       tma_load_2d(&tmW, &full[i], a_s + (size_t)i * TC_A_BYTES, (kb0_first + i) * TC_BK, tn0 * TC_BM, pol_w);
     }
+    // a split CTA has one short K range: the rest of its weight slice goes
+    // to L2 now, so that after the wait every operand load is an L2 hit
+    if (p.splits > 1)
+      for (int kb = kb0_first + npre; kb < kb1_first; ++kb) prefetch_l2_2d(&tmW, kb * TC_BK, tn0 * TC_BM);
   }
   // everything below may read what earlier kernels wrote; TMEM is taken only
   // now, so a CTA waiting here never holds columns its predecessor needs
@@ -372,6 +438,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     // epilogue warps 2..5: TMEM lane quarter q = warp % 4, tile row r
     const int q = warp & 3;
     const int r = q * 32 + lane;
+    int ebuf = 0;   // TMA output box in use
     int tn, tm, sp;
     for (int i = 0; work_item(p, i, tn, tm, sp); ++i) {
       const int b = i & 1;
@@ -383,28 +450,53 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       tc_fence_after();
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)b * p.acc_cols;
       const int m_base = tm * BN;
-      if (p.splits == 1) {
+      const int n = tn * TC_BM + r;
+      const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
+      if constexpr (RED == RED_NONE) {
+        // 16-token chunks; the TMEM load of chunk c+1 is in flight while chunk
+        // c goes out
+        uint32_t nxt[16];
+        tmem_ld16_async(trow, nxt);
+        tmem_wait_ld();
+        tmem_reg_fence16(nxt);
         for (int c0 = 0; c0 < BN; c0 += 16) {
           float v[16];
-          tmem_ld16(trow + c0, v);
-          if (c0 + 16 >= BN) {   // accumulator drained: the MMA warp may reuse it
+#pragma unroll
+          for (int k = 0; k < 16; ++k) v[k] = __uint_as_float(nxt[k]);
+          const bool more = c0 + 16 < BN;
+          if (more) {
+            tmem_ld16_async(trow + c0 + 16, nxt);
+          } else {   // accumulator drained: the MMA warp may reuse it
             tc_fence_before();
             mbar_arrive(&acc_empty[b]);
           }
-          epilogue_chunk(p, tn, m_base + c0, 16, r, v, stage);
+          if (p.tma_out) epilogue_tma(p, &tmO, tn, m_base + c0, r, v, brow, stg_raw, xch, ebuf);
+          else epilogue_chunk(p, tn, m_base + c0, 16, r, v, stage);
+          if (more) {
+            tmem_wait_ld();
+            tmem_reg_fence16(nxt);
+          }
         }
-      } else if (p.reduce == RED_L2_CLUSTER) {
+      } else if constexpr (RED == RED_L2_CLUSTER) {
         // this split's fp32 partial to the workspace as [col/4][row][4]: each
         // thread stores float4 of 4 consecutive columns, a warp one 512-byte run
         const size_t cl = (size_t)tm * gridDim.x + tn;
         float* w = p.ws + ((cl * p.splits + sp) * (size_t)(BN / 4)) * (TC_BM * 4) + (size_t)r * 4;
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          float v[16];
-          tmem_ld16(trow + c0, v);
+        for (int c0 = 0; c0 < BN; c0 += 64) {   // up to four TMEM loads in flight, one wait
+          const int nq = min(4, (BN - c0) / 16);   // BN is a multiple of 16
+          uint32_t raw[64];
 #pragma unroll
           for (int qq = 0; qq < 4; ++qq)
-            __stcg((float4*)(w + (size_t)(c0 / 4 + qq) * (TC_BM * 4)),
-                   make_float4(v[4 * qq], v[4 * qq + 1], v[4 * qq + 2], v[4 * qq + 3]));
+            if (qq < nq) tmem_ld16_async(trow + c0 + 16 * qq, raw + 16 * qq);
+          tmem_wait_ld();
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) tmem_reg_fence16(raw + 16 * qq);
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq)
+            if (qq < 4 * nq)
+              __stcg((float4*)(w + (size_t)(c0 / 4 + qq) * (TC_BM * 4)),
+                     make_float4(__uint_as_float(raw[4 * qq]), __uint_as_float(raw[4 * qq + 1]),
+                                 __uint_as_float(raw[4 * qq + 2]), __uint_as_float(raw[4 * qq + 3])));
         }
         __threadfence();
       } else {
@@ -445,6 +537,8 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         }
       }
     }
+    // every TMA output box has been written to global memory
+    if (p.tma_out && threadIdx.x == 64) bulk_wait<0>();
   }
   tc_fence_before();
   cta_sync();
@@ -456,7 +550,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     }
     cta_sync();
   }
-  if (p.reduce == RED_L2_CLUSTER && p.splits > 1) {
+  if constexpr (RED == RED_L2_CLUSTER) {
     // Every split of this tile has written its partial; the cluster barrier
     // (release / acquire) makes them visible.  Rank q sums columns
     // [q*BN/S, (q+1)*BN/S) over the splits in order and applies the epilogue.
@@ -464,23 +558,27 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     if (warp >= 2) {
       const int r = (warp & 3) * 32 + lane;
       const int Sp = p.splits;
-      const int cpr = BN / Sp;   // a multiple of 4
       const int rank = (int)cluster_ctarank();
       const size_t cl = (size_t)tm0 * gridDim.x + tn0;
       const float* base = p.ws + (cl * Sp * (size_t)(BN / 4) + rank * cpr / 4) * (TC_BM * 4) + (size_t)r * 4;
       const size_t sstride = (size_t)(BN / 4) * (TC_BM * 4);
-      for (int cc = 0; cc < cpr; cc += 16) {
-        const int nc = min(16, cpr - cc);
+      const int n = tn0 * TC_BM + r;
+      const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
+      int ebuf = 0;
+      for (int cc = 0; cc < cpr; cc += p.box_m) {
+        const int nc = p.box_m;
         float v[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) v[k] = 0.f;
         const float* b0 = base + (size_t)(cc / 4) * (TC_BM * 4);
         if (nc == 16) reduce_splits_l2<4>(b0, Sp, sstride, v);
-        else if (nc == 12) reduce_splits_l2<3>(b0, Sp, sstride, v);
         else if (nc == 8) reduce_splits_l2<2>(b0, Sp, sstride, v);
         else reduce_splits_l2<1>(b0, Sp, sstride, v);
-        epilogue_chunk(p, tn0, tm0 * BN + rank * cpr + cc, nc, r, v, stage);
+        const int m0 = tm0 * BN + rank * cpr + cc;
+        if (p.tma_out) epilogue_tma(p, &tmO, tn0, m0, r, v, brow, stg_raw, xch, ebuf);
+        else epilogue_chunk(p, tn0, m0, nc, r, v, stage);
       }
+      if (p.tma_out && threadIdx.x == 64) bulk_wait<0>();
     }
   }
   if (warp == 1) {
@@ -515,6 +613,20 @@ cudaError_t encode_2d(CUtensorMap* m, const void* base, int rows, int cols, int 
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// 2D map over a row-major output [rows][cols] (row stride ld elements) for
+// TMA stores: box = box_cols x box_rows, no swizzle (the box is dense in
+// shared memory), writes past the extents clipped.
+cudaError_t encode_out(CUtensorMap* m, void* base, int rows, int cols, int ld, bool bf, int box_cols, int box_rows) {
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * (bf ? 2 : 4)};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 // Token-tile width: the smallest of 32/64/96/128 that holds M; beyond 128
 // tokens, the multiple of 16 in [128, 256] whose tile count fills whole waves
 // of the SMs best (per-CTA work ~ waves x BN), larger BN on ties.
@@ -543,10 +655,16 @@ int g_max_cluster = 8;   // largest power-of-two cluster the split-K reduction m
 cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
-  if (e != cudaSuccess) return e;
+  const void* kernels[] = {(const void*)tc_gemm_kernel<RED_NONE>, (const void*)tc_gemm_kernel<RED_L2_CLUSTER>,
+                           (const void*)tc_gemm_kernel<RED_WORKSPACE>};
+  for (const void* k : kernels) {
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
+    if (e != cudaSuccess) return e;
+  }
   // clusters of 16 are beyond the portable limit: use them only if allowed
-  if (cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+  bool big = true;
+  for (const void* k : kernels) big = big && cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+  if (big) {
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
@@ -559,7 +677,7 @@ cudaError_t init_tc_gemm() {
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel, &cfg) == cudaSuccess && n > 0) g_max_cluster = 16;
+    if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel<RED_L2_CLUSTER>, &cfg) == cudaSuccess && n > 0) g_max_cluster = 16;
   }
   cudaGetLastError();
   return cudaSuccess;
@@ -582,6 +700,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const int tiles = tiles_n * tiles_m;
   int splits = 1;
   if (tiles < num_sms) splits = std::min(num_kb, std::max(1, num_sms / tiles));
+  if (g.max_splits > 0) splits = std::min(splits, g.max_splits);
   if (cluster) {
     // the splits of a tile form one cluster: a power of two, at most the cluster
     // limit, whose partials fit the workspace and whose column slices are
@@ -594,7 +713,8 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   } else {
     while (splits > 1 && ((size_t)splits * tiles * bn * TC_BM * 4 > ws.ws_bytes || tiles > ws.n_counters)) --splits;
   }
-  const int reduce = splits == 1 ? RED_NONE : (cluster ? RED_L2_CLUSTER : RED_WORKSPACE);
+  int reduce = splits == 1 ? RED_NONE : (cluster ? RED_L2_CLUSTER : RED_WORKSPACE);
+  const int cpr = bn / splits;   // a multiple of 4 whenever the splits form a cluster
   uint32_t acc_cols = 32;
   while ((int)acc_cols < bn) acc_cols <<= 1;
   const int stage_bytes = TC_A_BYTES + bn * TC_BK * 2;
@@ -602,20 +722,44 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const int grid_ctas = splits > 1 ? tiles * splits : std::min(tiles, num_sms);
   const int items = splits > 1 ? 1 : (tiles + grid_ctas - 1) / grid_ctas;
   int stages = std::min(8, TC_SMEM_BUDGET / stage_bytes);
+  // a split-K launch is latency-bound: enough stages for its whole (short) K
+  // range when that fits, so that no operand load waits for a freed stage
+  if (splits > 1) stages = std::min(stages, std::max(2, TC_RING_SPLIT / stage_bytes));
   stages = std::max(2, std::min(stages, std::max(2, kb_per_item * items)));
   const size_t ring = ((size_t)stages * stage_bytes + 1023) / 1024 * 1024;
-  // alignment slack + ring + barriers / TMEM slot / flags + staging tile (+ slack)
-  const size_t smem = 1024 + ring + (2 * stages + 4) * 8 + 32 + 16 + STG_BYTES + 64;
-  CUtensorMap mw, mx;
+  // outputs through TMA boxes when the output rows are 16-byte aligned
+  const bool out_bf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
+  const int es = out_bf ? 2 : 4;
+  const bool tma_out = reduce != RED_WORKSPACE && ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * es) % 16 == 0;
+  const int box_m = splits == 1 ? 16 : (cpr % 16 == 0 ? 16 : (cpr % 8 == 0 ? 8 : 4));
+  const uint32_t box_bytes =
+      (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
+  const size_t stg_bytes = tma_out ? 2 * (size_t)box_bytes : (STG_BYTES + 1023) / 1024 * 1024;
+  const size_t xch_bytes = (tma_out && g.epi == EPI_GEGLU) ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
+  const uint32_t stg_off = (uint32_t)ring;
+  const uint32_t xch_off = stg_off + (uint32_t)stg_bytes;
+  const uint32_t bar_off = xch_off + (uint32_t)xch_bytes;
+  const size_t smem = 1024 + bar_off + (size_t)(2 * stages + 4) * 8 + 4 + 16 + 64;
+  CUtensorMap mw, mx, mo;
+  memset(&mo, 0, sizeof(mo));
   cudaError_t e = encode_2d(&mw, g.W, g.N, g.K, g.ldw, TC_BM);
   if (e == cudaSuccess) e = encode_2d(&mx, g.A, g.M, g.K, g.lda, bn);
+  if (e == cudaSuccess && tma_out)
+    e = encode_out(&mo, g.out, g.M, g.epi == EPI_GEGLU ? g.N / 2 : g.N, g.ldo, out_bf,
+                   g.epi == EPI_GEGLU ? 64 : TC_BM, box_m);
   if (e != cudaSuccess) return e;
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
-             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv};
+             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
+             bar_off};
   const dim3 grid = splits > 1 ? dim3(tiles_n, tiles_m, splits) : dim3(grid_ctas);
-  return launch_kernel(tc_gemm_kernel, grid, dim3(TC_THREADS), smem, st,
-                       reduce == RED_L2_CLUSTER ? (unsigned)splits : 1u, mw, mx, p);
+  const dim3 block(TC_THREADS);
+  switch (reduce) {
+    case RED_NONE: return launch_kernel(tc_gemm_kernel<RED_NONE>, grid, block, smem, st, 1u, mw, mx, mo, p);
+    case RED_L2_CLUSTER:
+      return launch_kernel(tc_gemm_kernel<RED_L2_CLUSTER>, grid, block, smem, st, (unsigned)splits, mw, mx, mo, p);
+    default: return launch_kernel(tc_gemm_kernel<RED_WORKSPACE>, grid, block, smem, st, 1u, mw, mx, mo, p);
+  }
 }
 
 }  // namespace ravel

@@ -49,6 +49,7 @@ struct GemmArgs {
   // g = (n - v_col0) / vt_hd, d = (n - v_col0) % vt_hd, row pitch vt_kvp
   void* vt = nullptr;
   int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
+  int max_splits = 0;           // tcgen05 path: cap on the split-K factor (0: chosen from the shape)
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
 

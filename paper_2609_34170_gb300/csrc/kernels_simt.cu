@@ -2,6 +2,8 @@
 // adaRMSNorm, action in-projection, generic projection GEMM (fp32 FFMA; the
 // exact path of fp32 mode), GeGLU, grouped-query attention, and the rolling
 // tail (Euler update, release, shift, Philox append).
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "launch.h"
@@ -193,82 +195,171 @@ __device__ __forceinline__ void st4(bf16* p, float4 v) {
   *(uint2*)p = u;
 }
 
-// One row per block.  Every load of the row (x, and for action rows the six
-// modulation vectors) is issued before the reduction, so the row costs one
-// memory round trip; D % 4 == 0 and D <= 4096 (4 float4 per thread).
-template <typename T>
-__global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a) {
+__device__ __forceinline__ float4 add2(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float4 ld4(const bf16* p) {
+  const uint2 u = *(const uint2*)p;
+  const __nv_bfloat162 lo = *(const __nv_bfloat162*)&u.x, hi = *(const __nv_bfloat162*)&u.y;
+  return make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
+}
+
+// adaRMSNorm over a block of rows of one robot (Sec. 3.1, Eq. 2):
+//   action row (b, j):  y = x * rsqrt(mean(x^2) + eps) * (1 + scale) + shift,
+//                       (scale, shift) = M_t[j] + M_delta[b] + bias  (the
+//                       modulation is linear in the two embeddings)
+//   FOP row (b, f):     y = z * rsqrt(mean(z^2) + eps) * (1 + gamma)
+// A thread owns columns 4*tid + 1024*g (g < G) of every row of the block, so
+// the per-robot part M_delta[b] + bias (or gamma) is read once per block and
+// kept in registers; rows go through in batches of R with one barrier each
+// (the batch's row sums are reduced through a double-buffered table).
+template <typename T, int G>
+__global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, int nb_act, int rb_fop, int nb_fop) {
+  constexpr int R = (G >= 4) ? 1 : 4 / G;
+  __shared__ float red[2][R][8];
   pdl_trigger();
-  __shared__ float red[32];
-  constexpr int G = 4;
-  const int r = blockIdx.x;
-  const int D = a.D;
-  const int n_act = a.B * a.H;
-  size_t yrow;
-  if (r < n_act)
-    yrow = (size_t)(r / a.H) * a.row_pitch + r % a.H;
-  else
-    yrow = (size_t)((r - n_act) / a.F) * a.row_pitch + a.H + (r - n_act) % a.F;
-  T* Y = (T*)a.Y + yrow * D;
-  pdl_wait();
-  if (r < n_act) {
-    const int b = r / a.H, j = r % a.H;
-    const float* x = a.x + (size_t)r * D;
-    const float* mt = a.modv + (size_t)j * a.mod_ld + a.off;
-    const float* md = a.modv + (size_t)(a.H + b) * a.mod_ld + a.off;
-    const float* mb = a.mod_b + a.off;
-    float4 xv[G], sc[G], sh[G];
-    float ss = 0.f;
+  const int D = a.D, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int blk = blockIdx.x;
+  const bool act = blk < a.B * nb_act;
+  int b, j0, j1;
+  if (act) {
+    b = blk / nb_act;
+    j0 = (blk % nb_act) * rb_act;
+    j1 = min(a.H, j0 + rb_act);
+  } else {
+    blk -= a.B * nb_act;
+    b = blk / nb_fop;
+    j0 = (blk % nb_fop) * rb_fop;
+    j1 = min(a.F, j0 + rb_fop);
+  }
+  float4 csc[G], csh[G];   // action: bias (+ M_delta[b] after the wait); FOP: gamma
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int c = 4 * (threadIdx.x + 256 * g);
-      if (c < D) {
-        xv[g] = ld4(x + c);
-        sc[g] = add3(ld4(mt + c), ld4(md + c), ld4(mb + c));
-        sh[g] = add3(ld4(mt + D + c), ld4(md + D + c), ld4(mb + D + c));
-        ss += xv[g].x * xv[g].x + xv[g].y * xv[g].y + xv[g].z * xv[g].z + xv[g].w * xv[g].w;
+  for (int g = 0; g < G; ++g) {
+    const int c = 4 * threadIdx.x + 1024 * g;
+    csc[g] = csh[g] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c < D) {   // weights: independent of the earlier kernels
+      if (act) {
+        csc[g] = ld4(a.mod_b + a.off + c);
+        csh[g] = ld4(a.mod_b + a.off + D + c);
+      } else {
+        csc[g] = ld4(a.gamma + c);
       }
     }
-    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
+  }
+  pdl_wait();
+  const float* md = a.modv + (size_t)(a.H + b) * a.mod_ld + a.off;
+  int buf = 0;
+  for (int j = j0; j < j1; j += R, buf ^= 1) {
+    float4 xv[R][G], ts[R][G], th[R][G];
+    float ss[R];
+    if (act && j == j0) {   // M_delta[b] joins the first batch's loads (one round trip)
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int c = 4 * (threadIdx.x + 256 * g);
-      if (c < D)
-        st4(Y + c, make_float4(xv[g].x * inv * (1.f + sc[g].x) + sh[g].x, xv[g].y * inv * (1.f + sc[g].y) + sh[g].y,
-                               xv[g].z * inv * (1.f + sc[g].z) + sh[g].z, xv[g].w * inv * (1.f + sc[g].w) + sh[g].w));
-    }
-  } else {
-    const T* z = (const T*)a.fop + (size_t)(r - n_act) * D;
-    float zv[4 * G], gm[4 * G];
-    float ss = 0.f;
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int c = 4 * (threadIdx.x + 256 * g);
-      if (c < D) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          zv[4 * g + q] = to_f32(z[c + q]);
-          gm[4 * g + q] = a.gamma[c + q];
-          ss += zv[4 * g + q] * zv[4 * g + q];
+      for (int g = 0; g < G; ++g) {
+        const int c = 4 * threadIdx.x + 1024 * g;
+        if (c < D) {
+          csc[g] = add2(csc[g], ld4(md + c));
+          csh[g] = add2(csh[g], ld4(md + D + c));
         }
       }
     }
-    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int c = 4 * (threadIdx.x + 256 * g);
-      if (c < D)
-        st4(Y + c, make_float4(zv[4 * g] * inv * (1.f + gm[4 * g]), zv[4 * g + 1] * inv * (1.f + gm[4 * g + 1]),
-                               zv[4 * g + 2] * inv * (1.f + gm[4 * g + 2]), zv[4 * g + 3] * inv * (1.f + gm[4 * g + 3])));
+    for (int rr = 0; rr < R; ++rr) {
+      ss[rr] = 0.f;
+      const int jj = j + rr;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const int c = 4 * threadIdx.x + 1024 * g;
+        xv[rr][g] = ts[rr][g] = th[rr][g] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (jj < j1 && c < D) {
+          if (act) {
+            xv[rr][g] = ld4(a.x + (size_t)(b * a.H + jj) * D + c);
+            const float* mt = a.modv + (size_t)jj * a.mod_ld + a.off;
+            ts[rr][g] = ld4(mt + c);
+            th[rr][g] = ld4(mt + D + c);
+          } else {
+            xv[rr][g] = ld4((const T*)a.fop + (size_t)(b * a.F + jj) * D + c);
+          }
+        }
+      }
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+        ss[rr] += xv[rr][g].x * xv[rr][g].x + xv[rr][g].y * xv[rr][g].y + xv[rr][g].z * xv[rr][g].z +
+                  xv[rr][g].w * xv[rr][g].w;
+    }
+#pragma unroll
+    for (int rr = 0; rr < R; ++rr) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ss[rr] += __shfl_xor_sync(0xffffffffu, ss[rr], o);
+      if (lane == 0) red[buf][rr][warp] = ss[rr];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int rr = 0; rr < R; ++rr) {
+      const int jj = j + rr;
+      float tot = 0.f;
+#pragma unroll
+      for (int w = 0; w < 8; ++w) tot += red[buf][rr][w];
+      const float inv = rsqrtf(tot / (float)D + 1e-6f);
+      if (jj >= j1) continue;
+      T* Y = (T*)a.Y + ((size_t)b * a.row_pitch + (act ? jj : a.H + jj)) * D;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const int c = 4 * threadIdx.x + 1024 * g;
+        if (c >= D) continue;
+        const float4 x = xv[rr][g];
+        if (act) {
+          const float4 sc = add2(csc[g], ts[rr][g]), sh = add2(csh[g], th[rr][g]);
+          st4(Y + c, make_float4(x.x * inv * (1.f + sc.x) + sh.x, x.y * inv * (1.f + sc.y) + sh.y,
+                                 x.z * inv * (1.f + sc.z) + sh.z, x.w * inv * (1.f + sc.w) + sh.w));
+        } else {
+          const float4 gm = csc[g];
+          st4(Y + c, make_float4(x.x * inv * (1.f + gm.x), x.y * inv * (1.f + gm.y), x.z * inv * (1.f + gm.z),
+                                 x.w * inv * (1.f + gm.w)));
+        }
+      }
     }
   }
 }
 
+namespace {
+int g_norm_sms = 0;
+}
+
+template <typename T>
+cudaError_t launch_ada_norm_t(const NormArgs& a, cudaStream_t st) {
+  if (!g_norm_sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&g_norm_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || g_norm_sms < 1)
+      g_norm_sms = 132;
+  }
+  const int G = (a.D + 1023) / 1024;
+  const int R = (G >= 4) ? 1 : 4 / G;
+  // rows per block: enough blocks for every SM, in whole batches of R rows
+  auto rows_per_block = [&](int rows_per_robot) {
+    const int total = a.B * rows_per_robot;
+    int rb = (total + g_norm_sms - 1) / g_norm_sms;
+    rb = (rb + R - 1) / R * R;
+    return std::max(R, std::min(rb, rows_per_robot));
+  };
+  const int rb_act = rows_per_block(a.H), nb_act = (a.H + rb_act - 1) / rb_act;
+  const int nf = a.fop ? a.F : 0;
+  const int rb_fop = nf ? rows_per_block(nf) : 1, nb_fop = nf ? (nf + rb_fop - 1) / rb_fop : 0;
+  const int blocks = a.B * (nb_act + nb_fop);
+  if (blocks <= 0) return cudaSuccess;
+  NormArgs b = a;
+  b.F = nf;
+  switch (G) {
+    case 1: return launch_kernel(ada_norm_kernel<T, 1>, dim3(blocks), dim3(256), 0, st, 1, b, rb_act, nb_act, rb_fop, nb_fop);
+    case 2: return launch_kernel(ada_norm_kernel<T, 2>, dim3(blocks), dim3(256), 0, st, 1, b, rb_act, nb_act, rb_fop, nb_fop);
+    case 3: return launch_kernel(ada_norm_kernel<T, 3>, dim3(blocks), dim3(256), 0, st, 1, b, rb_act, nb_act, rb_fop, nb_fop);
+    default: return launch_kernel(ada_norm_kernel<T, 4>, dim3(blocks), dim3(256), 0, st, 1, b, rb_act, nb_act, rb_fop, nb_fop);
+  }
+}
+
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st) {
-  const int rows = a.B * a.H + (a.fop ? a.B * a.F : 0);
-  if (rows <= 0) return cudaSuccess;
-  if (dt == DT_BF16) return launch_kernel(ada_norm_kernel<bf16>, dim3(rows), dim3(256), 0, st, 1, a);
-  return launch_kernel(ada_norm_kernel<float>, dim3(rows), dim3(256), 0, st, 1, a);
+  if (a.D <= 0 || a.D > 4096 || a.D % 4) return cudaErrorInvalidValue;
+  return dt == DT_BF16 ? launch_ada_norm_t<bf16>(a, st) : launch_ada_norm_t<float>(a, st);
 }
 
 // ============================================================================ in-proj

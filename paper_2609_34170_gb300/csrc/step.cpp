@@ -260,8 +260,9 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     }                                   \
   } while (0)
   auto gemm = [&](const void* Aop, int lda, const void* W, int M, int N, int K, Epi epi, void* out, int ldo,
-                  Dtype out_dt, const float* bias) {
+                  Dtype out_dt, const float* bias, int split_cap = 0) {
     GemmArgs g{Aop, lda, W, K, M, N, K, epi, out, ldo, out_dt, bias};
+    g.max_splits = split_cap;
     return run_gemm(p, g, st);
   };
   auto rowp = [&](const void* base, size_t row, size_t ld) { return (const void*)((const char*)base + row * ld * es); };
@@ -296,6 +297,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       gq.vt_tokens = RPR;
       gq.vt_kvp = p.kvp;
       gq.vt_hkv = c.n_kv_heads;
+      gq.max_splits = p.split_cap[0];
       RUN(KK_GEMM_QKV, run_gemm(p, gq, st));
       AttnTcArgs at{p.QKV, p.nqkv, p.Vt, p.kvp, {p.ctx_k[0], p.ctx_k[1]}, {p.ctx_v[0], p.ctx_v[1]}, L, l,
                     c.max_batch, c.max_prefix, p.pst, p.ctx_state, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim,
@@ -311,11 +313,12 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
     }
     RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x, D,
-             DT_F32, nullptr));
+             DT_F32, nullptr, p.split_cap[1]));
     NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y, H};
     RUN(KK_NORM, launch_ada_norm(n2, dt, st));
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
     GemmArgs gu{p.Y, D, wgu, D, BH, 2 * Fm, D, EPI_GEGLU, p.Hm, Fm, dt, nullptr};
+    gu.max_splits = p.split_cap[2];
     if (p.use_tc && tc_gemm_supported(gu)) {
       RUN(KK_GEMM_GATE_UP, launch_gemm_tc(gu, p.tcws, p.num_sms, st));   // GeGLU fused in the epilogue
     } else {
@@ -323,7 +326,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       RUN(KK_GEGLU, launch_geglu(p.GU, BH, Fm, p.Hm, dt, st));
     }
     RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D, DT_F32,
-             nullptr));
+             nullptr, p.split_cap[3]));
   }
   NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y, H};
   RUN(KK_NORM, launch_ada_norm(nf, dt, st));

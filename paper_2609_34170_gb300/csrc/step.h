@@ -57,6 +57,8 @@ struct StepPlan {
   size_t attn_ws_bytes = 0;
   bool use_tc_attn = false;
   bool use_pdl = true;      // Programmatic Dependent Launch between the step's kernels
+  // split-K caps of the layer GEMMs {QKV, O, gate/up, down} (0: from the shape)
+  int split_cap[4] = {0, 0, 0, 0};
   TcWorkspace tcws{};       // split-K workspace of the tensor-core GEMM
   int num_sms = 0;
   bool use_tc = false;      // bf16 projections on tcgen05

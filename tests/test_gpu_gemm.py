@@ -56,16 +56,19 @@ def test_gemm_bf16(handles, M, N, K, epi):
 
 
 @pytest.mark.parametrize("M,N,K", [(50, 256, 1024), (66, 8192, 1024), (300, 1024, 256), (3200, 2048, 1024)])
-def test_gemm_geglu_bf16(handles, M, N, K):
+@pytest.mark.parametrize("with_bias", [False, True])
+def test_gemm_geglu_bf16(handles, M, N, K, with_bias):
     from paper_2609_34170_gb300 import ravel_gemm
     X, W = _rand((M, K), 5), _rand((N, K), 6, 0.05)
-    ref_all = X.astype(np.float64) @ W.astype(np.float64).T
+    bias = np.random.default_rng(9).standard_normal(N).astype(np.float32) if with_bias else np.zeros(N, np.float32)
+    ref_all = X.astype(np.float64) @ W.astype(np.float64).T + bias   # bias of each gate / up row, before GELU
     blocks = ref_all.reshape(M, N // 128, 2, 64)
     g, u = blocks[:, :, 0].reshape(M, N // 2), blocks[:, :, 1].reshape(M, N // 2)
     ref = 0.5 * g * (1 + np.tanh(np.sqrt(2 / np.pi) * (g + 0.044715 * g ** 3))) * u
     out = torch.zeros((M, N // 2), device="cuda", dtype=torch.bfloat16)
     ravel_gemm(handles["bf16"], torch.from_numpy(X).to("cuda", torch.bfloat16),
-               torch.from_numpy(W).to("cuda", torch.bfloat16), 3, out)
+               torch.from_numpy(W).to("cuda", torch.bfloat16), 3, out,
+               torch.from_numpy(bias).cuda() if with_bias else None)
     got = out.float().cpu().numpy()
     np.testing.assert_allclose(got, ref, rtol=1e-2, atol=1e-2 * (np.abs(ref).max() + 1e-3))
 
