@@ -1,6 +1,7 @@
 """Benchmark of the rolling action-expert step on GB300.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+    python bench.py --sweep            # stress grid: one JSON line per (batch, prefix, slots) point
 
 A step is one rolling step (conditioning, L transformer layers over the H
 action slots attending to the VLM prefix K/V and the FOP tokens, velocity
@@ -248,6 +249,63 @@ def cpu_baseline(cfg, budget_s=20.0):
 # ----------------------------------------------------------------------------- our arm
 
 
+def run_sweep(args):
+    """Stress grid of the pi0.5-shaped bf16 expert: batch {1, 16, 64, 256} x
+    prefix {256, 816, 2048} x slots {16, 50} (A = 32, F = 16).  Per point: graph
+    replays with one event pair per step -> p50 / p99 latency, robot-steps/s,
+    and the fraction of the step roofline max(bytes / HBM, FLOPs / tensor peak).
+    Weights are the seeded N(0, 0.02) set; prefix K/V and FOP tokens are
+    N(0, 1) drawn on the device (a speed measurement: parity is checked by the
+    tests on the same kernels)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_34170_gb300 import RollingSession
+    torch.cuda.set_device(0)
+    peaks, peak_src = load_peaks()
+    W = synth.make_weights(synth.SWEEP[0], 0)
+    st = torch.cuda.current_stream()
+    for i, cfg in enumerate(synth.SWEEP):
+        B, P, H = cfg.batch, cfg.prefix, cfg.slots
+        sess = RollingSession(cfg, W, 0)
+        sess.reset(synth.robot_seeds(7, B))
+        g = torch.Generator(device="cuda").manual_seed(1000 + i)
+        shape = (cfg.layers, B, cfg.n_kv_heads, P, cfg.head_dim)
+        k = torch.randn(shape, generator=g, device="cuda", dtype=torch.float32).to(torch.bfloat16)
+        v = torch.randn(shape, generator=g, device="cuda", dtype=torch.float32).to(torch.bfloat16)
+        sess.set_context(k, v, P)
+        z = torch.randn((B, cfg.fop_tokens, cfg.width), generator=g, device="cuda").to(torch.bfloat16)
+        t_d = torch.from_numpy(synth.staggered_times(H)).cuda()
+        delta = torch.from_numpy(synth.make_delta(B, 2, H)).cuda()
+        from paper_2609_34170_gb300 import ravel_roll_step
+        step = lambda: ravel_roll_step(sess.handle, sess.buffer, t_d, z, delta, sess.released, None, st)  # noqa: E731
+        for _ in range(max(3, args.warmup)):
+            step()
+        torch.cuda.synchronize()
+        n = max(10, min(args.steps, 200))
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        for a, b in ev:
+            a.record(st)
+            step()
+            b.record(st)
+        torch.cuda.synchronize()
+        lat = np.array([a.elapsed_time(b) for a, b in ev]) * 1e3
+        work = step_work(cfg, B, P)
+        t_bytes = work["bytes"] / (peaks["hbm_gbs"] * 1e9)
+        t_flops = work["flops"] / (peaks["bf16_tflops"] * 1e12)
+        roof_us = max(t_bytes, t_flops) * 1e6
+        p50 = float(np.percentile(lat, 50))
+        print(json.dumps({
+            "sweep_point": i, "batch": B, "prefix": P, "slots": H, "p50_us": p50,
+            "p99_us": float(np.percentile(lat, 99)), "steps_per_s": 1e6 / float(np.mean(lat)),
+            "robot_steps_per_s": B * 1e6 / float(np.mean(lat)), "roofline_us": roof_us,
+            "bound": "hbm" if t_bytes >= t_flops else "tensor", "frac_of_roofline": roof_us / p50,
+            "bytes": work["bytes"], "flops": work["flops"], "peaks": peak_src}), flush=True)
+        sess.close()
+        del k, v, z, sess
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -258,6 +316,9 @@ def main():
     ap.add_argument("--swap-every", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-steps", type=int, default=3)
+    ap.add_argument("--sweep", action="store_true",
+                    help="latency and roofline fraction over the stress grid (batch x prefix x slots); "
+                         "one JSON line per point")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     cfg = synth.PRESETS[args.config]
@@ -267,6 +328,9 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, cfg, rank)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
 
     import torch
