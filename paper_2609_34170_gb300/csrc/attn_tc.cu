@@ -129,15 +129,20 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;
   uint8_t* p_s = kv_s + (size_t)S * stage_bytes;
   uint64_t* bars = (uint64_t*)(p_s + 2 * AT_PBUF);
+  // K and V^T of a stage have their own barriers: K is released as soon as
+  // S = Q K^T has been computed, V^T only after P V, so the next K load does
+  // not wait for the softmax and the PV of the chunk it replaces
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;
-  uint64_t* kv_empty = kv_full + S;
-  uint64_t* s_full = kv_empty + S;
+  uint64_t* k_full = bars + 1;
+  uint64_t* v_full = k_full + S;
+  uint64_t* k_empty = v_full + S;
+  uint64_t* v_empty = k_empty + S;
+  uint64_t* s_full = v_empty + S;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
   uint64_t* pv_done = p_full + 2;   // [2]: PV of chunk i completes pv_done[i & 1]
   uint32_t* tmem_slot = (uint32_t*)(pv_done + 2);
-  int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] issued, [2] consumed
+  int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] K issued, [2] K consumed, [3] V issued, [4] V consumed
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qt = blockIdx.x, bg = blockIdx.y, split = blockIdx.z;
@@ -165,8 +170,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < S; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], p.mc);   // released by the PV commit of every CTA sharing the chunk
+      mbar_init(&k_full[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&k_empty[s], p.mc);   // released by the S (K) / PV (V) commit of every CTA sharing the chunk
+      mbar_init(&v_empty[s], p.mc);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
@@ -175,7 +182,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
     mbar_init(&pv_done[0], 1);
     mbar_init(&pv_done[1], 1);
-    flags[0] = flags[1] = flags[2] = 0;
+    flags[0] = flags[1] = flags[2] = flags[3] = flags[4] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   // with multicast, every CTA's barriers must exist before a peer targets them
@@ -188,26 +195,30 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   // K and V^T of chunk c into stage s: all of it, or (multicast) this CTA's
   // share -- head-dim blocks rank, rank+mc, .. of K and V^T rows
   // [rank*hd/mc, (rank+1)*hd/mc) -- sent to every CTA of the cluster
-  auto load_chunk = [&](int c, int s, uint64_t pol) {
+  auto load_k = [&](int c, int s, uint64_t pol) {
     uint8_t* ks = kv_s + (size_t)s * stage_bytes;
-    mbar_expect_tx(&kv_full[s], k_bytes + 128u * (uint32_t)p.hd);   // the whole chunk, whoever sends it
+    mbar_expect_tx(&k_full[s], k_bytes);   // the whole chunk, whoever sends it
     const bool pre = c < p.n_pre;
     const int cc = c - p.n_pre;
     const CUtensorMap* km = pre ? pk : &maps.k;
     const int ky = pre ? c * AT_BKV : g, kz = pre ? ctx_z : b * rows_per_robot + cc * AT_BKV;
+    for (int blk = (p.mc == 1 ? 0 : mrank); blk < p.nblk; blk += p.mc) {
+      if (p.mc == 1) tma_load_3d(km, &k_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, pol);
+      else tma_load_3d_mc(km, &k_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, mmask, pol);
+    }
+  };
+  auto load_v = [&](int c, int s, uint64_t pol) {
+    uint8_t* vs = kv_s + (size_t)s * stage_bytes + k_bytes;
+    mbar_expect_tx(&v_full[s], 128u * (uint32_t)p.hd);
+    const bool pre = c < p.n_pre;
+    const int cc = c - p.n_pre;
     const int vx = (pre ? c : cc) * AT_BKV, vz = pre ? ctx_z : b * p.Hkv + g;
     if (p.mc == 1) {
-      for (int blk = 0; blk < p.nblk; ++blk)
-        if (pre) tma_load_3d(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, pol);
-        else tma_load_3d(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, kz, pol);
-      tma_load_3d(pre ? pv : &maps.vt, &kv_full[s], ks + k_bytes, vx, 0, vz, pol);
+      tma_load_3d(pre ? pv : &maps.vt, &v_full[s], vs, vx, 0, vz, pol);
     } else {
-      for (int blk = mrank; blk < p.nblk; blk += p.mc)
-        if (pre) tma_load_3d_mc(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, mmask, pol);
-        else tma_load_3d_mc(km, &kv_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, g, kz, mmask, pol);
       const int rows = p.hd / p.mc;
-      tma_load_3d_mc(pre ? pvs : &maps.vts, &kv_full[s], ks + k_bytes + (size_t)mrank * rows * 128, vx, mrank * rows,
-                     vz, mmask, pol);
+      tma_load_3d_mc(pre ? pvs : &maps.vts, &v_full[s], vs + (size_t)mrank * rows * 128, vx, mrank * rows, vz, mmask,
+                     pol);
     }
   };
   if (threadIdx.x == 0) {
@@ -215,7 +226,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_kv));
     for (; c_next < c1 && c_next < p.n_pre && npre < S; ++c_next) {
       if (c_next * AT_BKV >= P) continue;
-      load_chunk(c_next, npre, pol_kv);
+      load_k(c_next, npre, pol_kv);
+      load_v(c_next, npre, pol_kv);
       ++npre;
     }
     // and warm L2 with the prefix chunks that will refill those stages
@@ -257,25 +269,38 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       for (int blk = 0; blk < p.nblk; ++blk)
         tma_load_3d(&maps.q, q_full, q_s + (size_t)blk * AT_QBLK, blk * 64, g * p.G, b * rows_per_robot + qt * p.TQ,
                     pol_q);
-      int i = npre;
-      for (int c = c_next; c < c1; ++c) {
-        if (c < p.n_pre && c * AT_BKV >= P) continue;
-        const int s = i % S;
-        if (!mbar_wait(&kv_empty[s], ((uint32_t)(i / S) & 1u) ^ 1u)) {
-          flags[0] = 1;
-          break;
-        }
-        load_chunk(c, s, c < p.n_pre ? pol_kv : pol_q);
-        {   // keep the L2 warm S chunks ahead of the loads (prefix chunks only)
-          const int cf = chunk_at(p, P, c0, c1, i + 2 * S);
-          if (cf >= 0 && cf < p.n_pre) {
-            for (int blk = 0; blk < p.nblk; ++blk) prefetch_l2_3d(pk, blk * 64, cf * AT_BKV, ctx_z);
-            prefetch_l2_3d(pv, cf * AT_BKV, 0, ctx_z);
+      // K of chunk nk and V^T of chunk nv (nv <= nk), each as soon as its slot
+      // is free; K may run up to S chunks ahead of V
+      int nk = npre, nv = npre;
+      unsigned long long t_last = globaltimer();
+      bool ok = true;
+      while (ok && (nk < n || nv < n)) {
+        bool progress = false;
+        if (nk < n && mbar_test_wait(&k_empty[nk % S], ((uint32_t)(nk / S) & 1u) ^ 1u)) {
+          const int c = chunk_at(p, P, c0, c1, nk);
+          load_k(c, nk % S, c < p.n_pre ? pol_kv : pol_q);
+          {   // keep the L2 warm 2S chunks ahead of the loads (prefix chunks only)
+            const int cf = chunk_at(p, P, c0, c1, nk + 2 * S);
+            if (cf >= 0 && cf < p.n_pre) {
+              for (int blk = 0; blk < p.nblk; ++blk) prefetch_l2_3d(pk, blk * 64, cf * AT_BKV, ctx_z);
+              prefetch_l2_3d(pv, cf * AT_BKV, 0, ctx_z);
+            }
           }
+          ++nk;
+          progress = true;
         }
-        ++i;
+        if (nv < nk && mbar_test_wait(&v_empty[nv % S], ((uint32_t)(nv / S) & 1u) ^ 1u)) {
+          const int c = chunk_at(p, P, c0, c1, nv);
+          load_v(c, nv % S, c < p.n_pre ? pol_kv : pol_q);
+          ++nv;
+          progress = true;
+        }
+        if (progress) t_last = globaltimer();
+        else if (globaltimer() - t_last > kTcTimeoutNs) ok = false;
       }
-      flags[1] = i;
+      if (!ok) flags[0] = 1;
+      flags[1] = nk;
+      flags[3] = nv;
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -293,7 +318,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         bool progress = false;
         if (ns < n && ns <= i + 1) {
           const int s = ns % S;
-          if (mbar_test_wait(&kv_full[s], (uint32_t)(ns / S) & 1u) &&
+          if (mbar_test_wait(&k_full[s], (uint32_t)(ns / S) & 1u) &&
               (ns < 2 || mbar_test_wait(&s_free[ns & 1], (uint32_t)((ns >> 1) - 1) & 1u))) {
             tc_fence_after();
             const uint8_t* ks = kv_s + (size_t)s * stage_bytes;
@@ -306,11 +331,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
                           (blk > 0 || k > 0) ? 1u : 0u);
             }
             umma_commit(&s_full[ns & 1]);
+            if (p.mc > 1) umma_commit_mc(&k_empty[s], mmask);   // K of this stage is free once S is done
+            else umma_commit(&k_empty[s]);
             ++ns;
             progress = true;
           }
         }
-        if (i < ns && mbar_test_wait(&p_full[i & 1], (uint32_t)(i >> 1) & 1u)) {
+        if (i < ns && mbar_test_wait(&p_full[i & 1], (uint32_t)(i >> 1) & 1u) &&
+            mbar_test_wait(&v_full[i % S], (uint32_t)(i / S) & 1u)) {
           tc_fence_after();
           const int s = i % S;
           const uint64_t ad = sw128_desc(smem_u32(p_s + (size_t)(i & 1) * AT_PBUF));
@@ -318,8 +346,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
 #pragma unroll
           for (int k = 0; k < 4; ++k)
             umma_bf16(tmem + o_col, ad + 2 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
-          if (p.mc > 1) umma_commit_mc(&kv_empty[s], mmask);
-          else umma_commit(&kv_empty[s]);
+          if (p.mc > 1) umma_commit_mc(&v_empty[s], mmask);
+          else umma_commit(&v_empty[s]);
           umma_commit(&pv_done[i & 1]);
           ++i;
           progress = true;
@@ -331,7 +359,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         }
       }
       if (!ok) flags[0] = 1;
-      flags[2] = ns;   // chunks whose K/V arrival was consumed
+      flags[2] = ns;   // chunks whose K arrival was consumed
+      flags[4] = i;    // chunks whose V^T arrival was consumed
     }
     __syncwarp();
   } else {
@@ -492,7 +521,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   cta_sync();
   if (flags[0]) {
     if (threadIdx.x == 0) {
-      for (int i = flags[2]; i < flags[1]; ++i) mbar_wait(&kv_full[i % S], (uint32_t)(i / S) & 1u);
+      for (int i = flags[2]; i < flags[1]; ++i) mbar_wait(&k_full[i % S], (uint32_t)(i / S) & 1u);
+      for (int i = flags[4]; i < flags[3]; ++i) mbar_wait(&v_full[i % S], (uint32_t)(i / S) & 1u);
       raise_error(p.err, ERR_TIMEOUT);
     }
     cta_sync();
