@@ -7,7 +7,7 @@
 // (context slot, valid length read on the device), then the FOP tokens and
 // the H action slots of this step (the QKV buffer).  Per chunk:
 //   S = Q K^T        tcgen05.mma, M = 128 query rows, N = 64 keys, into TMEM
-//   P = exp(S - m)   softmax warps: TMEM -> registers -> bf16 P in shared memory
+//   P = exp(S - m)   softmax warps: TMEM -> registers -> bf16 P back into TMEM
 //   O += P V         tcgen05.mma, M = 128, N = head dim, K = 64 keys, O in TMEM
 // Every operand is K-major with 128-byte swizzling; V is kept transposed
 // (keys contiguous) for that: the context's V is transposed when a context
@@ -43,14 +43,13 @@ constexpr int AT_BKV = 64;
 constexpr int AT_SMEM_MAX = 227 * 1024;
 constexpr uint32_t AT_QBLK = AT_BM * 128;     // bytes of one 64-wide head-dim block of Q
 constexpr uint32_t AT_KBLK = AT_BKV * 128;    // bytes of one 64-wide head-dim block of a K chunk
-constexpr uint32_t AT_PBUF = AT_BM * 128;     // bytes of one P tile (128 rows x 64 keys bf16)
 
 struct AtParams {
   int B, H, F, Hq, Hkv, G, hd, hdp;   // hdp: head dim rounded up to 16 (MMA N of P V)
   int TQ, q_tiles;
   int Pmax, n_pre, n_kv, splits;
   int layer, Bmax, mask_mode;
-  int nblk, stages;
+  int nblk, k_slots, v_slots;         // head-dim blocks of 64; K and V^T ring depths
   int mc;                             // query tiles of a (b, g) pair sharing each K/V chunk by multicast (1 = none)
   uint32_t vt_bytes;                  // bytes of one transposed-V chunk (hd rows x 128 B)
   const int* ctx_state;
@@ -122,22 +121,21 @@ __device__ __forceinline__ void combine_slice(const float* src0, size_t sstride,
 __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_constant__ AtMaps maps, AtParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  const int S = p.stages;
+  const int SK = p.k_slots, SV = p.v_slots;   // K and V^T ring depths
   const uint32_t k_bytes = (uint32_t)p.nblk * AT_KBLK;
-  const uint32_t stage_bytes = k_bytes + p.vt_bytes;   // both multiples of 1024
   uint8_t* q_s = smem;
-  uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;
-  uint8_t* p_s = kv_s + (size_t)S * stage_bytes;
-  uint64_t* bars = (uint64_t*)(p_s + 2 * AT_PBUF);
+  uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;   // K ring, then V^T ring
+  uint8_t* v_ring = kv_s + (size_t)SK * k_bytes;
+  uint64_t* bars = (uint64_t*)(v_ring + (size_t)SV * p.vt_bytes);
   // K and V^T of a stage have their own barriers: K is released as soon as
   // S = Q K^T has been computed, V^T only after P V, so the next K load does
   // not wait for the softmax and the PV of the chunk it replaces
   uint64_t* q_full = bars;
   uint64_t* k_full = bars + 1;
-  uint64_t* v_full = k_full + S;
-  uint64_t* k_empty = v_full + S;
-  uint64_t* v_empty = k_empty + S;
-  uint64_t* s_full = v_empty + S;
+  uint64_t* v_full = k_full + SK;
+  uint64_t* k_empty = v_full + SV;
+  uint64_t* v_empty = k_empty + SK;
+  uint64_t* s_full = v_empty + SV;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
   uint64_t* pv_done = p_full + 2;   // [2]: PV of chunk i completes pv_done[i & 1]
@@ -169,11 +167,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < S; ++s) {
+    for (int s = 0; s < SK; ++s) {
       mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], p.mc);   // released by the S commit of every CTA sharing the chunk
+    }
+    for (int s = 0; s < SV; ++s) {
       mbar_init(&v_full[s], 1);
-      mbar_init(&k_empty[s], p.mc);   // released by the S (K) / PV (V) commit of every CTA sharing the chunk
-      mbar_init(&v_empty[s], p.mc);
+      mbar_init(&v_empty[s], p.mc);   // released by the PV commit of every CTA sharing the chunk
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   // share -- head-dim blocks rank, rank+mc, .. of K and V^T rows
   // [rank*hd/mc, (rank+1)*hd/mc) -- sent to every CTA of the cluster
   auto load_k = [&](int c, int s, uint64_t pol) {
-    uint8_t* ks = kv_s + (size_t)s * stage_bytes;
+    uint8_t* ks = kv_s + (size_t)s * k_bytes;
     mbar_expect_tx(&k_full[s], k_bytes);   // the whole chunk, whoever sends it
     const bool pre = c < p.n_pre;
     const int cc = c - p.n_pre;
@@ -208,7 +208,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
   };
   auto load_v = [&](int c, int s, uint64_t pol) {
-    uint8_t* vs = kv_s + (size_t)s * stage_bytes + k_bytes;
+    uint8_t* vs = v_ring + (size_t)s * p.vt_bytes;
     mbar_expect_tx(&v_full[s], 128u * (uint32_t)p.hd);
     const bool pre = c < p.n_pre;
     const int cc = c - p.n_pre;
@@ -224,14 +224,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   if (threadIdx.x == 0) {
     uint64_t pol_kv;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_kv));
-    for (; c_next < c1 && c_next < p.n_pre && npre < S; ++c_next) {
+    for (; c_next < c1 && c_next < p.n_pre && npre < min(SK, SV); ++c_next) {
       if (c_next * AT_BKV >= P) continue;
       load_k(c_next, npre, pol_kv);
       load_v(c_next, npre, pol_kv);
       ++npre;
     }
     // and warm L2 with the prefix chunks that will refill those stages
-    for (int k = 0; k < S; ++k) {
+    for (int k = 0; k < SK; ++k) {
       const int c = chunk_at(p, P, c0, c1, npre + k);
       if (c < 0 || c >= p.n_pre) break;
       for (int blk = 0; blk < p.nblk; ++blk) prefetch_l2_3d(pk, blk * 64, c * AT_BKV, ctx_z);
@@ -270,17 +270,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         tma_load_3d(&maps.q, q_full, q_s + (size_t)blk * AT_QBLK, blk * 64, g * p.G, b * rows_per_robot + qt * p.TQ,
                     pol_q);
       // K of chunk nk and V^T of chunk nv (nv <= nk), each as soon as its slot
-      // is free; K may run up to S chunks ahead of V
+      // is free; K may run ahead of V
       int nk = npre, nv = npre;
       unsigned long long t_last = globaltimer();
       bool ok = true;
       while (ok && (nk < n || nv < n)) {
         bool progress = false;
-        if (nk < n && mbar_test_wait(&k_empty[nk % S], ((uint32_t)(nk / S) & 1u) ^ 1u)) {
+        if (nk < n && mbar_test_wait(&k_empty[nk % SK], ((uint32_t)(nk / SK) & 1u) ^ 1u)) {
           const int c = chunk_at(p, P, c0, c1, nk);
-          load_k(c, nk % S, c < p.n_pre ? pol_kv : pol_q);
-          {   // keep the L2 warm 2S chunks ahead of the loads (prefix chunks only)
-            const int cf = chunk_at(p, P, c0, c1, nk + 2 * S);
+          load_k(c, nk % SK, c < p.n_pre ? pol_kv : pol_q);
+          {   // keep the L2 warm 2 SK chunks ahead of the loads (prefix chunks only)
+            const int cf = chunk_at(p, P, c0, c1, nk + 2 * SK);
             if (cf >= 0 && cf < p.n_pre) {
               for (int blk = 0; blk < p.nblk; ++blk) prefetch_l2_3d(pk, blk * 64, cf * AT_BKV, ctx_z);
               prefetch_l2_3d(pv, cf * AT_BKV, 0, ctx_z);
@@ -289,9 +289,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           ++nk;
           progress = true;
         }
-        if (nv < nk && mbar_test_wait(&v_empty[nv % S], ((uint32_t)(nv / S) & 1u) ^ 1u)) {
+        if (nv < nk && mbar_test_wait(&v_empty[nv % SV], ((uint32_t)(nv / SV) & 1u) ^ 1u)) {
           const int c = chunk_at(p, P, c0, c1, nv);
-          load_v(c, nv % S, c < p.n_pre ? pol_kv : pol_q);
+          load_v(c, nv % SV, c < p.n_pre ? pol_kv : pol_q);
           ++nv;
           progress = true;
         }
@@ -317,11 +317,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       while (ok && i < n) {
         bool progress = false;
         if (ns < n && ns <= i + 1) {
-          const int s = ns % S;
-          if (mbar_test_wait(&k_full[s], (uint32_t)(ns / S) & 1u) &&
+          const int s = ns % SK;
+          if (mbar_test_wait(&k_full[s], (uint32_t)(ns / SK) & 1u) &&
               (ns < 2 || mbar_test_wait(&s_free[ns & 1], (uint32_t)((ns >> 1) - 1) & 1u))) {
             tc_fence_after();
-            const uint8_t* ks = kv_s + (size_t)s * stage_bytes;
+            const uint8_t* ks = kv_s + (size_t)s * k_bytes;
             for (int blk = 0; blk < p.nblk; ++blk) {
               const uint64_t ad = sw128_desc(smem_u32(q_s + (size_t)blk * AT_QBLK));
               const uint64_t bd = sw128_desc(smem_u32(ks + (size_t)blk * AT_KBLK));
@@ -338,14 +338,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           }
         }
         if (i < ns && mbar_test_wait(&p_full[i & 1], (uint32_t)(i >> 1) & 1u) &&
-            mbar_test_wait(&v_full[i % S], (uint32_t)(i / S) & 1u)) {
+            mbar_test_wait(&v_full[i % SV], (uint32_t)(i / SV) & 1u)) {
           tc_fence_after();
-          const int s = i % S;
-          const uint64_t ad = sw128_desc(smem_u32(p_s + (size_t)(i & 1) * AT_PBUF));
-          const uint64_t bd = sw128_desc(smem_u32(kv_s + (size_t)s * stage_bytes + k_bytes));
+          const int s = i % SV;
+          // A = P from TMEM (the S tile's first 32 columns, two bf16 per column)
+          const uint32_t pa = tmem + (uint32_t)(i & 1) * AT_BKV;
+          const uint64_t bd = sw128_desc(smem_u32(v_ring + (size_t)s * p.vt_bytes));
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_bf16(tmem + o_col, ad + 2 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
+            umma_bf16_ts(tmem + o_col, pa + 8 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
           if (p.mc > 1) umma_commit_mc(&v_empty[s], mmask);
           else umma_commit(&v_empty[s]);
           umma_commit(&pv_done[i & 1]);
@@ -428,26 +429,27 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       }
       if (need) m_used = m_new;
       const float nb = (m_used == -INFINITY) ? 0.f : -m_used;
-      // the P buffer of this chunk was last read by PV of chunk i - 2
-      if (i >= 2) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[i & 1], (uint32_t)((i - 2) >> 1) & 1u)) && ok;
-        tc_fence_after();
-      }
-      uint8_t* prow = p_s + (size_t)(i & 1) * AT_PBUF + (size_t)r * 128;
+      // P (bf16) overwrites the first 32 columns of this chunk's S tile: S of
+      // chunk i + 2 reuses the tile only after PV of chunk i has been issued,
+      // and the tensor pipe runs them in order
+      const uint32_t prow = lane_base + (uint32_t)(i & 1) * AT_BKV;
       float ls[8];
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {
-        float e[8];
+      for (int h2 = 0; h2 < 2; ++h2) {
+        uint32_t w[16];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) e[q] = fast_exp2(fmaf(sc[8 * ch + q], sl2, nb));
-        ls[ch] = ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
-        uint32_t w[4];
+        for (int ch = 0; ch < 4; ++ch) {
+          float e[8];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) w[q] = pack_bf16x2(e[2 * q], e[2 * q + 1]);
-        *(uint4*)(prow + ((ch ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+          for (int q = 0; q < 8; ++q) e[q] = fast_exp2(fmaf(sc[32 * h2 + 8 * ch + q], sl2, nb));
+          ls[4 * h2 + ch] = ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
+#pragma unroll
+          for (int q = 0; q < 4; ++q) w[4 * ch + q] = pack_bf16x2(e[2 * q], e[2 * q + 1]);
+        }
+        tmem_st16u(prow + 16 * h2, w);
       }
+      tmem_wait_st();
       l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
       mbar_arrive(&p_full[i & 1]);
       ++i;
@@ -458,13 +460,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
     if (!ok && lane == 0) flags[0] = 1;
     if (p.splits == 1) {
-      // O / l as bf16, staged row by row in the K/V stages (every chunk has
-      // been consumed and every MMA has completed, so nothing writes there
-      // any more), then stored by whole rows: a warp writes one output row of
-      // hd values per instruction instead of one value per lane.  16-byte
-      // column blocks are XOR-swizzled by row so that neither side conflicts.
+      // O / l as bf16: this thread stages its row in the rings (every chunk
+      // has been consumed and every MMA has completed, so nothing writes
+      // there any more; rows padded by 16 bytes so that the warp's 16-byte
+      // stores hit distinct banks) and hands it to the bulk copy engine as one
+      // contiguous hd-wide output row
       const float inv = (l > 0.f && n > 0) ? 1.f / l : 0.f;
-      const int rbytes = (2 * p.hdp + 127) & ~127;   // whole 128-byte swizzle spans
+      const int rbytes = ((2 * p.hdp + 63) & ~63) + 16;   // whole 32-column writes, + 16 against bank conflicts
       uint8_t* srow = kv_s + (size_t)r * rbytes;
       for (int cb = 0; cb < p.hdp; cb += 32) {
         uint32_t raw[32];
@@ -478,19 +480,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           w.y = pack_bf16x2(__uint_as_float(raw[8 * q + 2]) * inv, __uint_as_float(raw[8 * q + 3]) * inv);
           w.z = pack_bf16x2(__uint_as_float(raw[8 * q + 4]) * inv, __uint_as_float(raw[8 * q + 5]) * inv);
           w.w = pack_bf16x2(__uint_as_float(raw[8 * q + 6]) * inv, __uint_as_float(raw[8 * q + 7]) * inv);
-          const int blk = cb / 8 + q;
-          *(uint4*)(srow + ((blk ^ (r & 7)) << 4)) = w;
+          *(uint4*)(srow + (cb / 8 + q) * 16) = w;
         }
       }
-      __syncwarp();
-      const int nblk16 = p.hd / 8;   // 16-byte blocks of one output row
-      for (int rr = q4 * 32; rr < q4 * 32 + 32; ++rr) {
-        const int tt = rr / p.G, jj = qt * p.TQ + tt;
-        if (rr >= q_rows || jj >= p.H) break;   // rows are in token order
-        const uint8_t* sr = kv_s + (size_t)rr * rbytes;
-        bf16* dst = p.out + (size_t)(b * p.H + jj) * p.ld_out + (size_t)(g * p.G + rr % p.G) * p.hd;
-        for (int blk = lane; blk < nblk16; blk += 32)
-          *(uint4*)(dst + 8 * blk) = *(const uint4*)(sr + ((blk ^ (rr & 7)) << 4));
+      const int t = r / p.G, jj = qt * p.TQ + t;
+      if (r < q_rows && jj < p.H) {
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        bulk_copy_s2g(p.out + (size_t)(b * p.H + jj) * p.ld_out + (size_t)(g * p.G + r % p.G) * p.hd, srow,
+                      (uint32_t)(2 * p.hd));
+        bulk_commit();
+        bulk_wait<0>();   // written out before the shared memory goes away
       }
     } else {
       // unnormalised partial O as [ti][d/4][row][4] (a warp stores one
@@ -521,8 +520,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   cta_sync();
   if (flags[0]) {
     if (threadIdx.x == 0) {
-      for (int i = flags[2]; i < flags[1]; ++i) mbar_wait(&k_full[i % S], (uint32_t)(i / S) & 1u);
-      for (int i = flags[4]; i < flags[3]; ++i) mbar_wait(&v_full[i % S], (uint32_t)(i / S) & 1u);
+      for (int i = flags[2]; i < flags[1]; ++i) mbar_wait(&k_full[i % SK], (uint32_t)(i / SK) & 1u);
+      for (int i = flags[4]; i < flags[3]; ++i) mbar_wait(&v_full[i % SV], (uint32_t)(i / SV) & 1u);
       raise_error(p.err, ERR_TIMEOUT);
     }
     cta_sync();
@@ -662,16 +661,23 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
     p.mc = p.q_tiles;
   p.ws_o = a.ws;
   p.ws_ml = a.ws + (size_t)splits * nctas * AT_BM * p.hdp;
-  const uint32_t stage = (uint32_t)p.nblk * AT_KBLK + p.vt_bytes;
-  const size_t fixed = 1024 + (size_t)p.nblk * AT_QBLK + 2 * AT_PBUF + 256;
-  int stages = (int)std::min<size_t>(4, (AT_SMEM_MAX - fixed) / stage);
-  if (stages < 1) return cudaErrorInvalidConfiguration;
-  // the epilogue stages 128 bf16 rows of O in the K/V stages and stores them
-  // with 16-byte writes
-  if ((size_t)AT_BM * (size_t)((2 * p.hdp + 127) & ~127) > (size_t)stages * stage) return cudaErrorInvalidConfiguration;
+  // K slots: as many whole K + V^T stages as fit (<= 4); V^T slots: the K
+  // count plus what the remaining bytes hold (<= 2 more): K is free again as
+  // soon as S = Q K^T is done, V^T only after P V, so V^T needs the depth
+  const size_t k_bytes = (size_t)p.nblk * AT_KBLK;
+  const size_t stage = k_bytes + p.vt_bytes;
+  const size_t fixed = 1024 + (size_t)p.nblk * AT_QBLK + 512;
+  if (fixed + stage > (size_t)AT_SMEM_MAX) return cudaErrorInvalidConfiguration;
+  const int sk = (int)std::min<size_t>(4, (AT_SMEM_MAX - fixed) / stage);
+  const int sv = sk + (int)std::min<size_t>(2, (AT_SMEM_MAX - fixed - sk * stage) / p.vt_bytes);
+  const size_t rings = (size_t)sk * k_bytes + (size_t)sv * p.vt_bytes;
+  // the epilogue stages 128 bf16 rows of O in the rings and stores them with
+  // 16-byte writes
+  if ((size_t)AT_BM * (size_t)(((2 * p.hdp + 63) & ~63) + 16) > rings) return cudaErrorInvalidConfiguration;
   if (a.ld_out % 8 != 0 || ((uintptr_t)a.out & 15u) != 0) return cudaErrorMisalignedAddress;
-  p.stages = stages;
-  const size_t smem = fixed + (size_t)stages * stage;
+  p.k_slots = sk;
+  p.v_slots = sv;
+  const size_t smem = fixed + rings;
 
   AtMaps m;
   const int hd = a.hd, rpr = a.H + a.F;
