@@ -336,14 +336,14 @@ cudaError_t launch_ada_norm_t(const NormArgs& a, cudaStream_t st) {
   const int G = (a.D + 1023) / 1024;
   const int R = (G >= 4) ? 1 : 4 / G;
   // rows per block: enough blocks for every SM, in whole batches of R rows
-  auto rows_per_block = [&](int rows_per_robot) {
-    const int total = a.B * rows_per_robot;
-    int rb = (total + g_norm_sms - 1) / g_norm_sms;
-    rb = (rb + R - 1) / R * R;
-    return std::max(R, std::min(rb, rows_per_robot));
-  };
-  const int rb_act = rows_per_block(a.H), nb_act = (a.H + rb_act - 1) / rb_act;
+  // rows per block: all rows (action + FOP) over about three resident blocks
+  // per SM, in whole batches of R rows -- few serial batches per block
   const int nf = a.fop ? a.F : 0;
+  const int total = a.B * (a.H + nf);
+  int rb_all = (total + 3 * g_norm_sms - 1) / (3 * g_norm_sms);
+  rb_all = (rb_all + R - 1) / R * R;
+  auto rows_per_block = [&](int rows_per_robot) { return std::max(R, std::min(rb_all, rows_per_robot)); };
+  const int rb_act = rows_per_block(a.H), nb_act = (a.H + rb_act - 1) / rb_act;
   const int rb_fop = nf ? rows_per_block(nf) : 1, nb_fop = nf ? (nf + rb_fop - 1) / rb_fop : 0;
   const int blocks = a.B * (nb_act + nb_fop);
   if (blocks <= 0) return cudaSuccess;
