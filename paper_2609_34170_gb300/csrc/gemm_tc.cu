@@ -76,6 +76,8 @@ struct TcParams {
   bf16* vt;
   int v_col0, vt_hd, vt_tokens, vt_kvp, vt_hkv;
   int tma_out;          // outputs leave through TMA boxes
+  int oneshot;          // split launch whose whole K range fits the ring: tmW / tmX are 3-D maps
+                        // (64, rows, K / 64) and one box each brings all of its k-tiles
   int box_m;            // tokens per epilogue chunk (= rows of a TMA output box)
   uint32_t box_bytes;   // bytes of one TMA output box (1024-aligned)
   uint32_t stg_off;     // SIMT transpose tile, or two TMA output boxes
@@ -349,14 +351,23 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     if (p.tma_out) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
-    for (int i = 0; i < npre; ++i) {
-      mbar_expect_tx(&full[i], TC_A_BYTES + b_bytes);
-      tma_load_2d(&tmW, &full[i], a_s + (size_t)i * TC_A_BYTES, (kb0_first + i) * TC_BK, tn0 * TC_BM, pol_w);
+    if (p.oneshot) {
+      // every weight k-tile of this CTA in one box; the token k-tiles follow
+      // after the wait into the same barrier
+      // (the boxes are S = the largest split's k-tile count deep; a shorter
+      // split ignores the extra tile)
+      mbar_expect_tx(&full[0], (uint32_t)S * (TC_A_BYTES + b_bytes));
+      tma_load_3d(&tmW, &full[0], a_s, 0, tn0 * TC_BM, kb0_first, pol_w);
+    } else {
+      for (int i = 0; i < npre; ++i) {
+        mbar_expect_tx(&full[i], TC_A_BYTES + b_bytes);
+        tma_load_2d(&tmW, &full[i], a_s + (size_t)i * TC_A_BYTES, (kb0_first + i) * TC_BK, tn0 * TC_BM, pol_w);
+      }
+      // a split CTA has one short K range: the rest of its weight slice goes
+      // to L2 now, so that after the wait every operand load is an L2 hit
+      if (p.splits > 1)
+        for (int kb = kb0_first + npre; kb < kb1_first; ++kb) prefetch_l2_2d(&tmW, kb * TC_BK, tn0 * TC_BM);
     }
-    // a split CTA has one short K range: the rest of its weight slice goes
-    // to L2 now, so that after the wait every operand load is an L2 hit
-    if (p.splits > 1)
-      for (int kb = kb0_first + npre; kb < kb1_first; ++kb) prefetch_l2_2d(&tmW, kb * TC_BK, tn0 * TC_BM);
   }
   // everything below may read what earlier kernels wrote; TMEM is taken only
   // now, so a CTA waiting here never holds columns its predecessor needs
@@ -373,7 +384,10 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    if (lane == 0) {
+    if (lane == 0 && p.oneshot) {
+      tma_load_3d(&tmX, &full[0], b_s, 0, tm0 * BN, kb0_first, pol_x);
+      flags[2] = 1;
+    } else if (lane == 0) {
       int it = 0;   // ring position across all work items
       bool ok = true;
       int tn, tm, sp;
@@ -404,7 +418,24 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       int it = 0;
       bool ok = true;
       int tn, tm, sp;
-      for (int i = 0; ok && work_item(p, i, tn, tm, sp); ++i) {
+      if (p.oneshot) {   // one item, every k-tile behind one barrier
+        ok = mbar_wait(&full[0], 0);
+        if (ok) {
+          tc_fence_after();
+          for (int kb = 0; kb < kb1_first - kb0_first; ++kb) {
+            const uint64_t ad = sw128_desc(smem_u32(a_s + (size_t)kb * TC_A_BYTES));
+            const uint64_t bd = sw128_desc(smem_u32(b_s + (size_t)kb * b_bytes));
+#pragma unroll
+            for (int k = 0; k < TC_BK / 16; ++k)
+              umma_bf16(tmem, ad + 2 * k, bd + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          umma_commit(&acc_full[0]);
+          it = 1;
+        } else {
+          flags[0] = 1;
+        }
+      }
+      for (int i = 0; !p.oneshot && ok && work_item(p, i, tn, tm, sp); ++i) {
         const int b = i & 1;
         // the accumulator of item i - 2 must have been drained by the epilogue
         if (i >= 2 && !mbar_wait(&acc_empty[b], (uint32_t)((i >> 1) - 1) & 1u)) {
@@ -613,6 +644,20 @@ cudaError_t encode_2d(CUtensorMap* m, const void* base, int rows, int cols, int 
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// 3D map over a row-major bf16 [rows][cols] matrix (cols a multiple of 64)
+// viewed as (64 elements, rows, cols / 64 k-tiles): a box of box_rows x nkb
+// lands as nkb consecutive K-major 128-byte-swizzled tiles of box_rows rows.
+cudaError_t encode_kt(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows, int nkb) {
+  cuuint64_t dims[3] = {(cuuint64_t)TC_BK, (cuuint64_t)rows, (cuuint64_t)(cols / TC_BK)};
+  cuuint64_t strides[2] = {(cuuint64_t)ld * 2, (cuuint64_t)TC_BK * 2};
+  cuuint32_t box[3] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows, (cuuint32_t)nkb};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 // 2D map over a row-major output [rows][cols] (row stride ld elements) for
 // TMA stores: box = box_cols x box_rows, no swizzle (the box is dense in
 // shared memory), writes past the extents clipped.
@@ -726,6 +771,11 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   // range when that fits, so that no operand load waits for a freed stage
   if (splits > 1) stages = std::min(stages, std::max(2, TC_RING_SPLIT / stage_bytes));
   stages = std::max(2, std::min(stages, std::max(2, kb_per_item * items)));
+  // one-shot: a cluster split whose whole K range fits a ring of up to 200 KB
+  // takes its weight and token k-tiles in one box each (K a multiple of 64)
+  const bool oneshot = splits > 1 && cluster && g.K % TC_BK == 0 && g.K / TC_BK <= 256 &&
+                       (size_t)kb_per_item * stage_bytes <= (size_t)TC_SMEM_BUDGET;
+  if (oneshot) stages = kb_per_item;   // the ring is exactly one box deep
   const size_t ring = ((size_t)stages * stage_bytes + 1023) / 1024 * 1024;
   // outputs through TMA boxes when the output rows are 16-byte aligned
   const bool out_bf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
@@ -742,15 +792,17 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const size_t smem = 1024 + bar_off + (size_t)(2 * stages + 4) * 8 + 4 + 16 + 64;
   CUtensorMap mw, mx, mo;
   memset(&mo, 0, sizeof(mo));
-  cudaError_t e = encode_2d(&mw, g.W, g.N, g.K, g.ldw, TC_BM);
-  if (e == cudaSuccess) e = encode_2d(&mx, g.A, g.M, g.K, g.lda, bn);
+  cudaError_t e = oneshot ? encode_kt(&mw, g.W, g.N, g.K, g.ldw, TC_BM, kb_per_item)
+                          : encode_2d(&mw, g.W, g.N, g.K, g.ldw, TC_BM);
+  if (e == cudaSuccess)
+    e = oneshot ? encode_kt(&mx, g.A, g.M, g.K, g.lda, bn, kb_per_item) : encode_2d(&mx, g.A, g.M, g.K, g.lda, bn);
   if (e == cudaSuccess && tma_out)
     e = encode_out(&mo, g.out, g.M, g.epi == EPI_GEGLU ? g.N / 2 : g.N, g.ldo, out_bf,
                    g.epi == EPI_GEGLU ? 64 : TC_BM, box_m);
   if (e != cudaSuccess) return e;
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
-             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
+             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
              bar_off};
   const dim3 grid = splits > 1 ? dim3(tiles_n, tiles_m, splits) : dim3(grid_ctas);
   const dim3 block(TC_THREADS);
