@@ -54,7 +54,7 @@ constexpr int TC_SMEM_MAX = 227 * 1024;
 constexpr int TC_RING_SPLIT = 128 * 1024;    // operand ring of a split-K launch
 constexpr int STG_LD = 132;                  // SIMT staging pitch (floats): 16 tokens x 128 tile rows
 constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
-constexpr uint32_t XCH_BYTES = STG_BYTES;        // GeGLU transpose tile (TMA epilogue)
+constexpr uint32_t XCH_BYTES = 32 * STG_LD * 4;  // GeGLU transpose tile (TMA epilogue): <= 32 tokens x 128 rows
 
 enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2 };
 
@@ -136,7 +136,8 @@ __device__ __forceinline__ void reduce_splits_l2(const float* b0, int S, size_t 
 
 // V^T side output of the QKV projection for tokens m0 .. m0+nv-1 of this
 // thread's tile row: token m -> (robot m / T, key m % T).
-__device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, int nv, int r, const float v[16]) {
+template <int NV = 16>
+__device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, int nv, int r, const float v[NV]) {
   const int n = tile_n * TC_BM + r;
   if (n < p.v_col0 || n >= p.N) return;
   const float bb = p.bias ? p.bias[n] : 0.f;
@@ -144,7 +145,7 @@ __device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, 
   int rb = m0 / p.vt_tokens, kk = m0 % p.vt_tokens;
   bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
+  for (int i = 0; i < NV; ++i) {
     if (i < nv) {
       dst[kk] = __float2bfloat16_rn(v[i] + bb);
       if (++kk == p.vt_tokens) {
@@ -153,6 +154,32 @@ __device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, 
         dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
       }
     }
+  }
+}
+
+// v[4g + e] (g < NG <= 8: up to 32 tokens) = sum over splits s = 0..S-1 (in
+// order) of this thread's row at column group g; as reduce_splits_l2, with up
+// to 24 float4 loads in flight per batch (one batch for every launch here).
+template <int NG>
+__device__ __forceinline__ void reduce_slice_l2(const float* b0, int S, size_t sstride, float v[32]) {
+  constexpr int GB = (24 / NG) > 0 ? 24 / NG : 1;
+  for (int s0 = 0; s0 < S; s0 += GB) {
+    float4 x[GB][NG];
+#pragma unroll
+    for (int u = 0; u < GB; ++u)
+#pragma unroll
+      for (int g = 0; g < NG; ++g)
+        x[u][g] = (s0 + u < S) ? __ldcg((const float4*)(b0 + (size_t)(s0 + u) * sstride + (size_t)g * 512))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < GB; ++u)
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        v[4 * g] += x[u][g].x;
+        v[4 * g + 1] += x[u][g].y;
+        v[4 * g + 2] += x[u][g].z;
+        v[4 * g + 3] += x[u][g].w;
+      }
   }
 }
 
@@ -245,10 +272,11 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
 // shared memory (token-major, as the output), and thread 64 sends the box
 // with one TMA store (EPI_ADD_F32: TMA reduce-add into the residual stream);
 // rows past M and columns past N are clipped by the tensor map.
+template <int NV = 16>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* tmO, int tile_n, int m0, int r,
-                                             const float v[16], float brow, uint8_t* boxes, float* xch, int& ebuf) {
-  const int bm = p.box_m;
-  if (p.vt) store_vt(p, tile_n, m0, min(bm, p.M - m0), r, v);
+                                             const float v[NV], float brow, uint8_t* boxes, float* xch, int& ebuf) {
+  const int bm = p.box_m;   // <= NV
+  if (p.vt) store_vt<NV>(p, tile_n, m0, min(bm, p.M - m0), r, v);
   // the box written two chunks ago must have been read by its TMA store
   if (threadIdx.x == 64) bulk_wait_read<1>();
   epi_bar();
@@ -258,24 +286,27 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
     // transpose through xch so that every thread then forms 8 outputs of one
     // token (the GELUs spread over all 128 threads)
 #pragma unroll
-    for (int i = 0; i < 16; ++i)
+    for (int i = 0; i < NV; ++i)
       if (i < bm) xch[i * STG_LD + r] = v[i] + brow;
     epi_bar();
-    const int c = r >> 3, fg = r & 7;
-    if (c < bm) {
-      const float4* g4 = (const float4*)(xch + c * STG_LD + fg * 8);
-      const float4* u4 = (const float4*)(xch + c * STG_LD + 64 + fg * 8);
-      const float4 ga = g4[0], gb = g4[1], ua = u4[0], ub = u4[1];
-      *(uint4*)((bf16*)box + c * 64 + fg * 8) =
-          make_uint4(pack_bf16x2(gelu_tanh_f(ga.x) * ua.x, gelu_tanh_f(ga.y) * ua.y),
-                     pack_bf16x2(gelu_tanh_f(ga.z) * ua.z, gelu_tanh_f(ga.w) * ua.w),
-                     pack_bf16x2(gelu_tanh_f(gb.x) * ub.x, gelu_tanh_f(gb.y) * ub.y),
-                     pack_bf16x2(gelu_tanh_f(gb.z) * ub.z, gelu_tanh_f(gb.w) * ub.w));
+#pragma unroll
+    for (int h = 0; h < NV / 16; ++h) {
+      const int c = (r >> 3) + 16 * h, fg = r & 7;
+      if (c < bm) {
+        const float4* g4 = (const float4*)(xch + c * STG_LD + fg * 8);
+        const float4* u4 = (const float4*)(xch + c * STG_LD + 64 + fg * 8);
+        const float4 ga = g4[0], gb = g4[1], ua = u4[0], ub = u4[1];
+        *(uint4*)((bf16*)box + c * 64 + fg * 8) =
+            make_uint4(pack_bf16x2(gelu_tanh_f(ga.x) * ua.x, gelu_tanh_f(ga.y) * ua.y),
+                       pack_bf16x2(gelu_tanh_f(ga.z) * ua.z, gelu_tanh_f(ga.w) * ua.w),
+                       pack_bf16x2(gelu_tanh_f(gb.x) * ub.x, gelu_tanh_f(gb.y) * ub.y),
+                       pack_bf16x2(gelu_tanh_f(gb.z) * ub.z, gelu_tanh_f(gb.w) * ub.w));
+      }
     }
   } else if (p.out_bf16) {
     bf16* o = (bf16*)box;
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < NV; ++i) {
       float x = v[i] + brow;
       if (p.epi == EPI_STORE_SILU) x = silu_f(x);
       if (i < bm) o[i * TC_BM + r] = __float2bfloat16_rn(x);
@@ -283,7 +314,7 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   } else {
     float* o = (float*)box;
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < NV; ++i) {
       float x = v[i] + brow;
       if (p.epi == EPI_STORE_SILU) x = silu_f(x);
       if (i < bm) o[i * TC_BM + r] = x;
@@ -596,7 +627,26 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       const int n = tn0 * TC_BM + r;
       const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
       int ebuf = 0;
-      for (int cc = 0; cc < cpr; cc += p.box_m) {
+      // a slice that would take three or more 4- or 8-token chunks goes out
+      // whole: one L2 round trip, one output box
+      const bool whole = p.tma_out && cpr <= 32 && cpr > 8 && cpr % 16 != 0;
+      if (whole) {
+        float v[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = 0.f;
+        switch (cpr / 4) {
+          case 1: reduce_slice_l2<1>(base, Sp, sstride, v); break;
+          case 2: reduce_slice_l2<2>(base, Sp, sstride, v); break;
+          case 3: reduce_slice_l2<3>(base, Sp, sstride, v); break;
+          case 4: reduce_slice_l2<4>(base, Sp, sstride, v); break;
+          case 5: reduce_slice_l2<5>(base, Sp, sstride, v); break;
+          case 6: reduce_slice_l2<6>(base, Sp, sstride, v); break;
+          case 7: reduce_slice_l2<7>(base, Sp, sstride, v); break;
+          default: reduce_slice_l2<8>(base, Sp, sstride, v); break;
+        }
+        epilogue_tma<32>(p, &tmO, tn0, tm0 * BN + rank * cpr, r, v, brow, stg_raw, xch, ebuf);
+      }
+      for (int cc = 0; !whole && cc < cpr; cc += p.box_m) {
         const int nc = p.box_m;
         float v[16];
 #pragma unroll
@@ -781,7 +831,9 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const bool out_bf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
   const int es = out_bf ? 2 : 4;
   const bool tma_out = reduce != RED_WORKSPACE && ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * es) % 16 == 0;
-  const int box_m = splits == 1 ? 16 : (cpr % 16 == 0 ? 16 : (cpr % 8 == 0 ? 8 : 4));
+  const int box_m = splits == 1 ? 16
+                    : (tma_out && cpr <= 32 && cpr > 8 && cpr % 16 != 0) ? cpr   // the whole slice in one box
+                    : (cpr % 16 == 0 ? 16 : (cpr % 8 == 0 ? 8 : 4));
   const uint32_t box_bytes =
       (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
   const size_t stg_bytes = tma_out ? 2 * (size_t)box_bytes : (STG_BYTES + 1023) / 1024 * 1024;
