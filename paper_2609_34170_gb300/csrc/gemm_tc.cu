@@ -21,9 +21,11 @@
 //    SMs) with two TMEM accumulators, so the epilogue of one tile overlaps the
 //    MMAs of the next;
 //  * few tiles: the K dimension is split over grid.z.  The splits of a tile
-//    form a thread-block cluster; each writes its fp32 partial to L2, the
-//    cluster barrier publishes them, and rank q sums a token slice over the
-//    splits in order (deterministic) and applies the epilogue;
+//    form a thread-block cluster and rank q sums a token slice over the splits
+//    in order (deterministic) and applies the epilogue.  The partials travel
+//    by st.async straight into rank q's shared memory, completing on an
+//    mbarrier there (slices of up to 32 tokens), else through L2 and the
+//    cluster barrier;
 //  * workspace mode (no cluster, for callers that bring their own scratch):
 //    the last split to arrive (per-tile counter) sums all partials.
 // Epilogue: a chunk of tokens is written into a shared-memory box in the
@@ -56,7 +58,7 @@ constexpr int STG_LD = 132;                  // SIMT staging pitch (floats): 16 
 constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
 constexpr uint32_t XCH_BYTES = 32 * STG_LD * 4;  // GeGLU transpose tile (TMA epilogue): <= 32 tokens x 128 rows
 
-enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2 };
+enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3 };
 
 struct TcParams {
   int M, N, K;
@@ -82,6 +84,10 @@ struct TcParams {
   uint32_t box_bytes;   // bytes of one TMA output box (1024-aligned)
   uint32_t stg_off;     // SIMT transpose tile, or two TMA output boxes
   uint32_t xch_off;     // GeGLU exchange
+  uint32_t rcv_off;     // RED_DSMEM: the partials received from the splits, [split][cpr / 4][128 rows]
+                        // float4, overlaid on the operand ring (free once every CTA of the cluster
+                        // has finished its MMAs), else on the output boxes + exchange (used only
+                        // after the sum)
   uint32_t bar_off;     // mbarriers, TMEM slot, flags
 };
 
@@ -146,13 +152,12 @@ __device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, 
   bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
-    if (i < nv) {
-      dst[kk] = __float2bfloat16_rn(v[i] + bb);
-      if (++kk == p.vt_tokens) {
-        kk = 0;
-        ++rb;
-        dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
-      }
+    if (i >= nv) break;
+    dst[kk] = __float2bfloat16_rn(v[i] + bb);
+    if (++kk == p.vt_tokens) {
+      kk = 0;
+      ++rb;
+      dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
     }
   }
 }
@@ -180,6 +185,25 @@ __device__ __forceinline__ void reduce_slice_l2(const float* b0, int S, size_t s
         v[4 * g + 2] += x[u][g].z;
         v[4 * g + 3] += x[u][g].w;
       }
+  }
+}
+
+// v[4g + e] (g < NG <= 8) = sum over splits s = 0..S-1 (in order) of the
+// received partials: b0 points at this thread's row of split 0, group 0;
+// group g of split s is (s * NG + g) * 128 float4 further.
+template <int NG>
+__device__ __forceinline__ void reduce_slice_smem(const float4* b0, int S, float v[32]) {
+  for (int s = 0; s < S; ++s) {
+    float4 x[NG];
+#pragma unroll
+    for (int g = 0; g < NG; ++g) x[g] = b0[(size_t)(s * NG + g) * TC_BM];
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      v[4 * g] += x[g].x;
+      v[4 * g + 1] += x[g].y;
+      v[4 * g + 2] += x[g].z;
+      v[4 * g + 3] += x[g].w;
+    }
   }
 }
 
@@ -286,8 +310,10 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
     // transpose through xch so that every thread then forms 8 outputs of one
     // token (the GELUs spread over all 128 threads)
 #pragma unroll
-    for (int i = 0; i < NV; ++i)
-      if (i < bm) xch[i * STG_LD + r] = v[i] + brow;
+    for (int i = 0; i < NV; ++i) {
+      if (i >= bm) break;
+      xch[i * STG_LD + r] = v[i] + brow;
+    }
     epi_bar();
 #pragma unroll
     for (int h = 0; h < NV / 16; ++h) {
@@ -304,20 +330,36 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
       }
     }
   } else if (p.out_bf16) {
+    // (each loop stops at the box width: a short slice runs, and fetches,
+    // only its own iterations)
     bf16* o = (bf16*)box;
+    if (p.epi == EPI_STORE_SILU) {
 #pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      float x = v[i] + brow;
-      if (p.epi == EPI_STORE_SILU) x = silu_f(x);
-      if (i < bm) o[i * TC_BM + r] = __float2bfloat16_rn(x);
+      for (int i = 0; i < NV; ++i) {
+        if (i >= bm) break;
+        o[i * TC_BM + r] = __float2bfloat16_rn(silu_f(v[i] + brow));
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < NV; ++i) {
+        if (i >= bm) break;
+        o[i * TC_BM + r] = __float2bfloat16_rn(v[i] + brow);
+      }
     }
   } else {
     float* o = (float*)box;
+    if (p.epi == EPI_STORE_SILU) {
 #pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      float x = v[i] + brow;
-      if (p.epi == EPI_STORE_SILU) x = silu_f(x);
-      if (i < bm) o[i * TC_BM + r] = x;
+      for (int i = 0; i < NV; ++i) {
+        if (i >= bm) break;
+        o[i * TC_BM + r] = silu_f(v[i] + brow);
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < NV; ++i) {
+        if (i >= bm) break;
+        o[i * TC_BM + r] = v[i] + brow;
+      }
     }
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -349,7 +391,8 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;      // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
-  uint32_t* tmem_slot = (uint32_t*)(acc_empty + 2);
+  uint64_t* rcv_bar = acc_empty + 2;    // RED_DSMEM: every split's slice of this rank has arrived
+  uint32_t* tmem_slot = (uint32_t*)(rcv_bar + 1);
   int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] last split, [2] issued, [3] consumed
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -372,8 +415,11 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 128);
     }
+    if constexpr (RED == RED_DSMEM) mbar_init(rcv_bar, 1);
     flags[0] = flags[1] = flags[2] = flags[3] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    // the slices of all splits (this one's included): 128 rows x cpr tokens each
+    if constexpr (RED == RED_DSMEM) mbar_expect_tx(rcv_bar, (uint32_t)(BN * TC_BM * 4));
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     // Weights never depend on earlier kernels: stream the first stages' weight
     // tiles while the previous kernel is still finishing.
@@ -443,6 +489,9 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       flags[2] = it;
     }
     __syncwarp();
+    // RED_DSMEM: one arrival per thread on the cluster barrier that opens the
+    // exchange (the epilogue warps arrive once their MMAs are complete)
+    if constexpr (RED == RED_DSMEM) cluster_arrive_release();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(TC_BM, BN);
@@ -496,6 +545,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       flags[3] = it;
     }
     __syncwarp();
+    if constexpr (RED == RED_DSMEM) cluster_arrive_release();
   } else {
     // epilogue warps 2..5: TMEM lane quarter q = warp % 4, tile row r
     const int q = warp & 3;
@@ -505,6 +555,13 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     for (int i = 0; work_item(p, i, tn, tm, sp); ++i) {
       const int b = i & 1;
       const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[b], (uint32_t)(i >> 1) & 1u));
+      if constexpr (RED == RED_DSMEM) {
+        // past this barrier every CTA of the cluster has finished its MMAs
+        // (its operand ring may be overwritten) and armed its receive barrier;
+        // every thread arrives exactly once, whatever happened before
+        cluster_arrive_release();
+        cluster_wait_acquire();
+      }
       if (!ok) {
         if (lane == 0) flags[0] = 1;
         break;
@@ -537,6 +594,35 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
           if (more) {
             tmem_wait_ld();
             tmem_reg_fence16(nxt);
+          }
+        }
+      } else if constexpr (RED == RED_DSMEM) {
+        // token slice q of this split's partial goes to rank q (= split q) of
+        // the cluster: float4 group g of the slice lands at [sp][g][r] there
+        const int ngs = cpr / 4;
+        const uint32_t rcv0 = smem_u32(smem + p.rcv_off) + (uint32_t)(sp * ngs * TC_BM + r) * 16u;
+        const uint32_t bar0 = smem_u32(rcv_bar);
+        int dst = 0, gl = 0;   // destination rank and group of the next float4
+        for (int c0 = 0; c0 < BN; c0 += 64) {   // up to four TMEM loads in flight, one wait
+          const int nq = min(4, (BN - c0) / 16);   // BN is a multiple of 16
+          uint32_t raw[64];
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq)
+            if (qq < nq) tmem_ld16_async(trow + c0 + 16 * qq, raw + 16 * qq);
+          tmem_wait_ld();
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) tmem_reg_fence16(raw + 16 * qq);
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq) {
+            if (qq >= 4 * nq) break;
+            st_async_f4(mapa_shared(rcv0 + (uint32_t)gl * (TC_BM * 16), (uint32_t)dst),
+                        make_float4(__uint_as_float(raw[4 * qq]), __uint_as_float(raw[4 * qq + 1]),
+                                    __uint_as_float(raw[4 * qq + 2]), __uint_as_float(raw[4 * qq + 3])),
+                        mapa_shared(bar0, (uint32_t)dst));
+            if (++gl == ngs) {
+              gl = 0;
+              ++dst;
+            }
           }
         }
       } else if constexpr (RED == RED_L2_CLUSTER) {
@@ -611,6 +697,41 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       raise_error(p.err, ERR_TIMEOUT);
     }
     cta_sync();
+  }
+  if constexpr (RED == RED_DSMEM) {
+    // Rank q sums its slice of tokens [q*cpr, (q+1)*cpr) over the splits in
+    // order once every split's bytes have arrived (the wait also keeps this
+    // CTA alive until no store into its shared memory is in flight), then
+    // sends the whole slice out as one box.  (When the partials overlay the
+    // output boxes, epilogue_tma passes a barrier of all 128 threads before it
+    // writes over what was just read.)
+    if (warp >= 2) {
+      const int r = (warp & 3) * 32 + lane;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait_cluster(rcv_bar, 0));
+      if (!ok) {
+        if (lane == 0) raise_error(p.err, ERR_TIMEOUT);
+      } else {
+        const int n = tn0 * TC_BM + r;
+        const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
+        const float4* b0 = (const float4*)(smem + p.rcv_off) + r;
+        float v[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = 0.f;
+        switch (cpr / 4) {
+          case 1: reduce_slice_smem<1>(b0, p.splits, v); break;
+          case 2: reduce_slice_smem<2>(b0, p.splits, v); break;
+          case 3: reduce_slice_smem<3>(b0, p.splits, v); break;
+          case 4: reduce_slice_smem<4>(b0, p.splits, v); break;
+          case 5: reduce_slice_smem<5>(b0, p.splits, v); break;
+          case 6: reduce_slice_smem<6>(b0, p.splits, v); break;
+          case 7: reduce_slice_smem<7>(b0, p.splits, v); break;
+          default: reduce_slice_smem<8>(b0, p.splits, v); break;
+        }
+        int ebuf = 0;
+        epilogue_tma<32>(p, &tmO, tn0, tm0 * BN + sp0 * cpr, r, v, brow, stg_raw, xch, ebuf);
+        if (threadIdx.x == 64) bulk_wait<0>();
+      }
+    }
   }
   if constexpr (RED == RED_L2_CLUSTER) {
     // Every split of this tile has written its partial; the cluster barrier
@@ -751,7 +872,7 @@ cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
   const void* kernels[] = {(const void*)tc_gemm_kernel<RED_NONE>, (const void*)tc_gemm_kernel<RED_L2_CLUSTER>,
-                           (const void*)tc_gemm_kernel<RED_WORKSPACE>};
+                           (const void*)tc_gemm_kernel<RED_WORKSPACE>, (const void*)tc_gemm_kernel<RED_DSMEM>};
   for (const void* k : kernels) {
     e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
     if (e != cudaSuccess) return e;
@@ -831,17 +952,34 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const bool out_bf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
   const int es = out_bf ? 2 : 4;
   const bool tma_out = reduce != RED_WORKSPACE && ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * es) % 16 == 0;
-  const int box_m = splits == 1 ? 16
-                    : (tma_out && cpr <= 32 && cpr > 8 && cpr % 16 != 0) ? cpr   // the whole slice in one box
-                    : (cpr % 16 == 0 ? 16 : (cpr % 8 == 0 ? 8 : 4));
-  const uint32_t box_bytes =
-      (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
-  const size_t stg_bytes = tma_out ? 2 * (size_t)box_bytes : (STG_BYTES + 1023) / 1024 * 1024;
-  const size_t xch_bytes = (tma_out && g.epi == EPI_GEGLU) ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
-  const uint32_t stg_off = (uint32_t)ring;
-  const uint32_t xch_off = stg_off + (uint32_t)stg_bytes;
-  const uint32_t bar_off = xch_off + (uint32_t)xch_bytes;
-  const size_t smem = 1024 + bar_off + (size_t)(2 * stages + 4) * 8 + 4 + 16 + 64;
+  int box_m = 0;
+  uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, rcv_off = 0, bar_off = 0;
+  size_t smem = 0;
+  auto layout = [&](bool dsmem) {
+    box_m = splits == 1 ? 16
+            : (tma_out && cpr <= 32 && (dsmem || (cpr > 8 && cpr % 16 != 0))) ? cpr   // the whole slice in one box
+            : (cpr % 16 == 0 ? 16 : (cpr % 8 == 0 ? 8 : 4));
+    box_bytes = (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
+    const size_t stg_bytes = tma_out ? 2 * (size_t)box_bytes : (STG_BYTES + 1023) / 1024 * 1024;
+    const size_t xch_bytes = (tma_out && g.epi == EPI_GEGLU) ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
+    // received partials (all splits' slices of this rank) overlay the operand
+    // ring, else the boxes + exchange
+    const size_t rcv_bytes = dsmem ? (size_t)TC_BM * bn * 4 : 0;
+    const bool in_ring = rcv_bytes <= ring;
+    xch_off = stg_off + (uint32_t)stg_bytes;
+    rcv_off = in_ring ? 0u : stg_off;
+    bar_off = stg_off + (uint32_t)std::max(stg_bytes + xch_bytes, in_ring ? (size_t)0 : rcv_bytes);
+    smem = 1024 + bar_off + (size_t)(2 * stages + 5) * 8 + 4 + 16 + 64;
+  };
+  // partials by st.async into the owning rank's shared memory when the token
+  // slice fits one output box (<= 32 tokens) and the receive area fits
+  bool dsmem = reduce == RED_L2_CLUSTER && tma_out && cpr <= 32;
+  layout(dsmem);
+  if (dsmem && smem > (size_t)TC_SMEM_MAX) {
+    dsmem = false;
+    layout(false);
+  }
+  if (dsmem) reduce = RED_DSMEM;
   CUtensorMap mw, mx, mo;
   memset(&mo, 0, sizeof(mo));
   cudaError_t e = oneshot ? encode_kt(&mw, g.W, g.N, g.K, g.ldw, TC_BM, kb_per_item)
@@ -855,13 +993,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
-             bar_off};
+             rcv_off, bar_off};
   const dim3 grid = splits > 1 ? dim3(tiles_n, tiles_m, splits) : dim3(grid_ctas);
   const dim3 block(TC_THREADS);
   switch (reduce) {
     case RED_NONE: return launch_kernel(tc_gemm_kernel<RED_NONE>, grid, block, smem, st, 1u, mw, mx, mo, p);
     case RED_L2_CLUSTER:
       return launch_kernel(tc_gemm_kernel<RED_L2_CLUSTER>, grid, block, smem, st, (unsigned)splits, mw, mx, mo, p);
+    case RED_DSMEM:
+      return launch_kernel(tc_gemm_kernel<RED_DSMEM>, grid, block, smem, st, (unsigned)splits, mw, mx, mo, p);
     default: return launch_kernel(tc_gemm_kernel<RED_WORKSPACE>, grid, block, smem, st, 1u, mw, mx, mo, p);
   }
 }

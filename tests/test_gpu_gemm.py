@@ -1,7 +1,8 @@
 """The projection GEMM building block (tcgen05 / TMEM / TMA for bf16, SIMT
 for fp32) against numpy fp64 matmul of the same bf16 operands, through the C
 ABI (ravel_gemm).  Shapes cover single and multiple tiles, ragged token /
-feature / K tails, split-K and every epilogue."""
+feature / K tails, split-K (partials exchanged through shared memory for token
+slices of 4..32, through L2 for wider ones) and every epilogue."""
 import numpy as np
 import pytest
 
@@ -55,7 +56,8 @@ def test_gemm_bf16(handles, M, N, K, epi):
     np.testing.assert_allclose(got, ref, rtol=1e-4, atol=1e-4 * scale)
 
 
-@pytest.mark.parametrize("M,N,K", [(50, 256, 1024), (66, 8192, 1024), (300, 1024, 256), (3200, 2048, 1024)])
+@pytest.mark.parametrize("M,N,K", [(50, 256, 1024), (50, 8192, 1024), (66, 4096, 1024), (66, 8192, 1024),
+                                   (300, 1024, 256), (3200, 2048, 1024)])
 @pytest.mark.parametrize("with_bias", [False, True])
 def test_gemm_geglu_bf16(handles, M, N, K, with_bias):
     from paper_2609_34170_gb300 import ravel_gemm
