@@ -16,10 +16,15 @@
 // grows by more than 2^8 (the kept maximum is exact for the final
 // normalisation, so this is not an approximation).
 // At batch 1 a (b, g) pair has only a few query tiles, so the key chunks are
-// split over grid.z; the splits of a query tile form a thread-block cluster,
-// publish their partial (O, m, l) through L2 and each rank merges a slice of
-// the head dimension after the cluster barrier.  The producer keeps the L2
-// warm a few prefix chunks ahead of its loads.
+// split over grid.z; the splits of a query tile form a thread-block cluster
+// and rank q merges head-dim slice q of every split's partial.  Once every
+// split's MMAs are done (one cluster barrier), each split sends its rows'
+// (m, l) and its output normalised by its own l, in bf16 (the precision of
+// every activation between kernels of the bf16 path), by st.async straight
+// into the owning rank's shared memory (overlaid on Q and the K/V rings);
+// an mbarrier there counts the bytes.  Where that does not apply, the splits
+// publish unnormalised fp32 partials through L2 and the cluster barrier.  The
+// producer keeps the L2 warm a few prefix chunks ahead of its loads.
 //
 // Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator + MMA
 // issuer, warps 2..5 softmax / epilogue (warp w owns TMEM lanes 32*(w%4)..).
@@ -51,6 +56,7 @@ struct AtParams {
   int layer, Bmax, mask_mode;
   int nblk, k_slots, v_slots;         // head-dim blocks of 64; K and V^T ring depths
   int mc;                             // query tiles of a (b, g) pair sharing each K/V chunk by multicast (1 = none)
+  int xch;                            // splits > 1: partials through shared memory (1) or L2 (0)
   uint32_t vt_bytes;                  // bytes of one transposed-V chunk (hd rows x 128 B)
   const int* ctx_state;
   bf16* out;
@@ -139,7 +145,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
   uint64_t* pv_done = p_full + 2;   // [2]: PV of chunk i completes pv_done[i & 1]
-  uint32_t* tmem_slot = (uint32_t*)(pv_done + 2);
+  uint64_t* rcv_bar = pv_done + 2;  // xch: every split's share of this rank has arrived
+  uint32_t* tmem_slot = (uint32_t*)(rcv_bar + 1);
   int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] K issued, [2] K consumed, [3] V issued, [4] V consumed
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -152,6 +159,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   const int c0 = (int)((long)split * C / p.splits), c1 = (int)((long)(split + 1) * C / p.splits);
   const uint32_t ncols = (128 + p.hdp <= 256) ? 256u : 512u;
   const int ctx_z = (p.layer * p.Bmax + b) * p.Hkv + g;
+  // query rows of this tile that hold a slot (rows 0 .. vrows-1)
+  const int vrows = p.G * max(0, min(p.TQ, p.H - qt * p.TQ));
+  // xch: per rank, [split][cps / 8][128 rows] groups of 8 bf16, then [split][128 rows] (m, l)
+  const int cps = p.hdp / p.splits;
 
   pdl_trigger();
   if (P < 1 || P > p.Pmax) {   // uniform across the CTA: nothing allocated yet
@@ -182,8 +193,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
     mbar_init(&pv_done[0], 1);
     mbar_init(&pv_done[1], 1);
+    mbar_init(rcv_bar, 1);
     flags[0] = flags[1] = flags[2] = flags[3] = flags[4] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (p.xch) mbar_expect_tx(rcv_bar, (uint32_t)(p.splits * vrows * (2 * cps + 8)));
   }
   // with multicast, every CTA's barriers must exist before a peer targets them
   if (p.mc > 1) cluster_sync();
@@ -303,6 +316,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       flags[3] = nv;
     }
     __syncwarp();
+    // xch: one arrival per thread on the cluster barrier that opens the
+    // exchange (the softmax warps arrive once their last PV is complete)
+    if (p.xch) cluster_arrive_release();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc_s = idesc_bf16(AT_BM, AT_BKV);
@@ -364,6 +380,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       flags[4] = i;    // chunks whose V^T arrival was consumed
     }
     __syncwarp();
+    if (p.xch) cluster_arrive_release();
   } else {
     // softmax / epilogue: thread owns query row r (TMEM lane r)
     const int q4 = warp & 3;
@@ -395,13 +412,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       const int kk0 = (c < p.n_pre) ? c * AT_BKV : (c - p.n_pre) * AT_BKV;
       const int kvalid = (c < p.n_pre) ? P - kk0 : rows_per_robot - kk0;
       const bool iso = (p.mask_mode == 1) && (c >= p.n_pre) && (kk0 < p.H);
-      if (kvalid < AT_BKV || iso) {
+      // (two compact loops: this code runs cold at batch 1, where each
+      // instruction fetched costs more than it does)
+      if (kvalid < AT_BKV) {
 #pragma unroll
-        for (int k = 0; k < 64; ++k) {
-          bool v = k < kvalid;
-          if (iso && kk0 + k < p.H) v = v && (kk0 + k == j);
-          if (!v) sc[k] = -INFINITY;
-        }
+        for (int k = 0; k < 64; ++k) sc[k] = k < kvalid ? sc[k] : -INFINITY;
+      }
+      if (iso) {
+#pragma unroll
+        for (int k = 0; k < 64; ++k)
+          if (kk0 + k < p.H && kk0 + k != j) sc[k] = -INFINITY;
       }
       float m8[8];
 #pragma unroll
@@ -459,6 +479,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       tc_fence_after();
     }
     if (!ok && lane == 0) flags[0] = 1;
+    if (p.xch) {
+      // past this barrier every split of the cluster has finished its MMAs
+      // (its Q and rings may be overwritten) and armed its receive barrier;
+      // every thread arrives exactly once, whatever happened before
+      cluster_arrive_release();
+      cluster_wait_acquire();
+    }
     if (p.splits == 1) {
       // O / l as bf16: this thread stages its row in the rings (every chunk
       // has been consumed and every MMA has completed, so nothing writes
@@ -490,6 +517,56 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
                       (uint32_t)(2 * p.hd));
         bulk_commit();
         bulk_wait<0>();   // written out before the shared memory goes away
+      }
+    } else if (p.xch) {
+      // rows holding a slot: (m, l) to every rank; O / l as bf16, head-dim
+      // slice q to rank q, starting with this split's own slice so that the
+      // splits send to different ranks at any moment.  The TMEM loads are
+      // warp-collective: every lane runs them, only rows that hold a slot send.
+      const bool snd = r < vrows;
+      const bool has = n > 0 && l > 0.f;
+      const float inv = has ? 1.f / l : 0.f;
+      const int ngs = cps / 8;
+      const uint32_t base = smem_u32(smem);
+      const uint32_t o0 = base + (uint32_t)(split * ngs * AT_BM + r) * 16u;
+      const uint32_t bar0 = smem_u32(rcv_bar);
+      if (snd) {
+        const uint32_t ml0 = base + (uint32_t)(p.splits * ngs * AT_BM) * 16u + (uint32_t)(split * AT_BM + r) * 8u;
+        const float m_s = has ? m_used : -INFINITY, l_s = has ? l : 0.f;
+        for (int q = 0; q < p.splits; ++q) st_async_f2(mapa_shared(ml0, (uint32_t)q), m_s, l_s, mapa_shared(bar0, (uint32_t)q));
+      }
+      const int nch = p.hdp / 16;
+      int ch = (split * cps) / 16;
+      uint32_t cur[16];
+      tmem_ld16_async(lane_base + o_col + 16 * ch, cur);
+      tmem_wait_ld();
+      tmem_reg_fence16(cur);
+      for (int jj = 0; jj < nch; ++jj) {
+        const int chn = ch + 1 == nch ? 0 : ch + 1;
+        uint32_t nxt[16];
+        if (jj + 1 < nch) tmem_ld16_async(lane_base + o_col + 16 * chn, nxt);
+        if (snd) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {   // two groups of 8 columns
+            const int gidx = 2 * ch + h;
+            const int dst = gidx / ngs, gl = gidx - dst * ngs;
+            uint4 w;
+            w.x = pack_bf16x2(__uint_as_float(cur[8 * h]) * inv, __uint_as_float(cur[8 * h + 1]) * inv);
+            w.y = pack_bf16x2(__uint_as_float(cur[8 * h + 2]) * inv, __uint_as_float(cur[8 * h + 3]) * inv);
+            w.z = pack_bf16x2(__uint_as_float(cur[8 * h + 4]) * inv, __uint_as_float(cur[8 * h + 5]) * inv);
+            w.w = pack_bf16x2(__uint_as_float(cur[8 * h + 6]) * inv, __uint_as_float(cur[8 * h + 7]) * inv);
+            if (!has) w = make_uint4(0u, 0u, 0u, 0u);   // no key: the accumulator was never written
+            st_async_u4(mapa_shared(o0 + (uint32_t)gl * (AT_BM * 16), (uint32_t)dst), w,
+                        mapa_shared(bar0, (uint32_t)dst));
+          }
+        }
+        if (jj + 1 < nch) {
+          tmem_wait_ld();
+          tmem_reg_fence16(nxt);
+#pragma unroll
+          for (int k = 0; k < 16; ++k) cur[k] = nxt[k];
+        }
+        ch = chn;
       }
     } else {
       // unnormalised partial O as [ti][d/4][row][4] (a warp stores one
@@ -526,7 +603,64 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
     cta_sync();
   }
-  if (p.splits > 1) {
+  if (p.xch) {
+    // Rank q merges head-dim columns [q*cps, (q+1)*cps) of its rows once every
+    // split's share has arrived (the wait also keeps this CTA alive until no
+    // store into its shared memory is in flight):
+    //   O = sum_s 2^(m_s - M) l_s Ohat_s / sum_s 2^(m_s - M) l_s,  Ohat_s = O_s / l_s.
+    if (warp >= 2) {
+      const int r = (warp & 3) * 32 + lane;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait_cluster(rcv_bar, 0));
+      if (!ok) {
+        if (lane == 0) raise_error(p.err, ERR_TIMEOUT);
+      } else if (r < vrows) {
+        const int Sp = p.splits, ngs = cps / 8;
+        const uint4* og = (const uint4*)smem + r;   // [s][g][row]
+        const float2* ml = (const float2*)(smem + (size_t)Sp * ngs * AT_BM * 16) + r;   // [s][row]
+        float wgt[16];
+        float M = -INFINITY;
+#pragma unroll
+        for (int s2 = 0; s2 < 16; ++s2) {
+          if (s2 >= Sp) break;
+          const float2 v = ml[s2 * AT_BM];
+          wgt[s2] = v.x;
+          M = fmaxf(M, v.x);
+        }
+        float L = 0.f;
+#pragma unroll
+        for (int s2 = 0; s2 < 16; ++s2) {
+          if (s2 >= Sp) break;
+          const float l_s = ml[s2 * AT_BM].y;
+          wgt[s2] = (wgt[s2] == -INFINITY) ? 0.f : exp2f(wgt[s2] - M) * l_s;
+          L += wgt[s2];
+        }
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const int t = r / p.G, hh = r % p.G;
+        const int j = qt * p.TQ + t;
+        bf16* orow = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
+        for (int gq = 0; gq < ngs; ++gq) {
+          const int d = split * cps + 8 * gq;
+          if (d >= p.hd) break;
+          float acc[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+#pragma unroll
+          for (int s2 = 0; s2 < 16; ++s2) {
+            if (s2 >= Sp) break;
+            const uint4 u = og[(size_t)(s2 * ngs + gq) * AT_BM];
+            const uint32_t uu[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              acc[2 * k] += wgt[s2] * __uint_as_float(uu[k] << 16);
+              acc[2 * k + 1] += wgt[s2] * __uint_as_float(uu[k] & 0xFFFF0000u);
+            }
+          }
+          *(uint4*)(orow + d) = make_uint4(pack_bf16x2(acc[0] * inv, acc[1] * inv), pack_bf16x2(acc[2] * inv, acc[3] * inv),
+                                           pack_bf16x2(acc[4] * inv, acc[5] * inv), pack_bf16x2(acc[6] * inv, acc[7] * inv));
+        }
+      }
+    }
+  } else if (p.splits > 1) {
     // The key splits of this query tile form a cluster: once every split has
     // published its (O, m, l), rank q merges head-dim columns
     // [q*hdp/S, (q+1)*hdp/S):  O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
@@ -541,12 +675,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       float M = -INFINITY, L = 0.f;
 #pragma unroll
       for (int s2 = 0; s2 < 16; ++s2) {
-        wgt[s2] = (s2 < Sp) ? __ldcg(p.ws_ml + ((t0 + s2) * 2) * AT_BM + r) : -INFINITY;
+        wgt[s2] = -INFINITY;
+        if (s2 >= Sp) continue;
+        wgt[s2] = __ldcg(p.ws_ml + ((t0 + s2) * 2) * AT_BM + r);
         M = fmaxf(M, wgt[s2]);
       }
 #pragma unroll
       for (int s2 = 0; s2 < 16; ++s2) {
-        const float l_s = (s2 < Sp) ? __ldcg(p.ws_ml + ((t0 + s2) * 2 + 1) * AT_BM + r) : 0.f;
+        if (s2 >= Sp) break;
+        const float l_s = __ldcg(p.ws_ml + ((t0 + s2) * 2 + 1) * AT_BM + r);
         wgt[s2] = (wgt[s2] == -INFINITY) ? 0.f : exp2f(wgt[s2] - M);
         L += wgt[s2] * l_s;
       }
@@ -661,6 +798,10 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
     p.mc = p.q_tiles;
   p.ws_o = a.ws;
   p.ws_ml = a.ws + (size_t)splits * nctas * AT_BM * p.hdp;
+  // partials through shared memory: whole 8-column bf16 groups per rank slice,
+  // no multicast cluster, and the receive area (O groups + (m, l) of every
+  // split) within Q + the rings (checked below)
+  p.xch = splits > 1 && p.mc == 1 && (p.hdp / splits) % 8 == 0 ? 1 : 0;
   // K slots: as many whole K + V^T stages as fit (<= 4); V^T slots: the K
   // count plus what the remaining bytes hold (<= 2 more): K is free again as
   // soon as S = Q K^T is done, V^T only after P V, so V^T needs the depth
@@ -678,6 +819,7 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   p.k_slots = sk;
   p.v_slots = sv;
   const size_t smem = fixed + rings;
+  if (p.xch && (size_t)AT_BM * p.hdp * 2 + (size_t)splits * AT_BM * 8 > (size_t)p.nblk * AT_QBLK + rings) p.xch = 0;
 
   AtMaps m;
   const int hd = a.hd, rpr = a.H + a.F;

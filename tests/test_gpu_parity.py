@@ -65,6 +65,31 @@ def test_ragged_shapes(dtype):
     s.close()
 
 
+# Key chunks split over a thread-block cluster (2, 4, 16 splits; one and two
+# query tiles; two robots), with a partial last prefix chunk, and a prefix
+# shorter than the slot capacity so that some splits get no key at all.
+SPLIT_KV = [
+    (dict(layers=2, width=256, n_q_heads=4, n_kv_heads=1, head_dim=64, mlp_dim=512, slots=20, action_dim=7,
+          prefix=300, fop_tokens=5, batch=1), None),
+    (dict(layers=2, width=256, n_q_heads=4, n_kv_heads=2, head_dim=128, mlp_dim=512, slots=12, action_dim=5,
+          prefix=700, fop_tokens=4, batch=1), None),
+    (dict(layers=1, width=256, n_q_heads=2, n_kv_heads=1, head_dim=128, mlp_dim=256, slots=12, action_dim=5,
+          prefix=2000, fop_tokens=3, batch=1), 1500),
+    (dict(layers=1, width=256, n_q_heads=8, n_kv_heads=2, head_dim=64, mlp_dim=256, slots=40, action_dim=6,
+          prefix=500, fop_tokens=8, batch=2), None),
+]
+
+
+@pytest.mark.parametrize("kw,prefix_len", SPLIT_KV)
+def test_split_kv_attention(kw, prefix_len):
+    cfg = synth.ExpertConfig(**kw, dtype="bf16")
+    case = Case(cfg, prefix_len=prefix_len)
+    s = gpu_session(case)
+    for i in range(2):
+        check_step(case, s, label=f"split-kv step {i}")
+    s.close()
+
+
 def test_slot_isolated_mask():
     cfg = _ragged("fp32", batch=2)
     case = Case(cfg)
