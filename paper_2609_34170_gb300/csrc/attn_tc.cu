@@ -124,6 +124,63 @@ __device__ __forceinline__ void combine_slice(const float* src0, size_t sstride,
   }
 }
 
+__device__ __forceinline__ uint4 lds_u4(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ float2 lds_f2(uint32_t a) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
+  return v;
+}
+
+// Merge of this thread's row over the SP splits' shares received in shared
+// memory (O groups [s][g][row] of 8 bf16 from `og`, (m, l) [s][row] from
+// `ml`, both shared-memory addresses of row 0): head-dim groups g < ngs of
+// slice q, columns q*8*ngs + 8g, stored as bf16 (columns past hd skipped).
+//   O = sum_s 2^(m_s - M) l_s Ohat_s / sum_s 2^(m_s - M) l_s
+template <int SP>
+__device__ __forceinline__ void xch_combine(uint32_t og, uint32_t ml, int r, int ngs, int d0, int hd, bf16* orow) {
+  float2 v[SP];
+#pragma unroll
+  for (int s2 = 0; s2 < SP; ++s2) v[s2] = lds_f2(ml + (uint32_t)(s2 * AT_BM + r) * 8u);
+  float M = -INFINITY;
+#pragma unroll
+  for (int s2 = 0; s2 < SP; ++s2) M = fmaxf(M, v[s2].x);
+  float w[SP];
+  float L = 0.f;
+#pragma unroll
+  for (int s2 = 0; s2 < SP; ++s2) {
+    w[s2] = (v[s2].x == -INFINITY) ? 0.f : exp2f(v[s2].x - M) * v[s2].y;
+    L += w[s2];
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+  for (int s2 = 0; s2 < SP; ++s2) w[s2] *= inv;
+  for (int gq = 0; gq < ngs; ++gq) {
+    const int d = d0 + 8 * gq;
+    if (d >= hd) break;
+    uint4 u[SP];
+#pragma unroll
+    for (int s2 = 0; s2 < SP; ++s2) u[s2] = lds_u4(og + ((uint32_t)(s2 * ngs + gq) * AT_BM + r) * 16u);
+    float acc[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+#pragma unroll
+    for (int s2 = 0; s2 < SP; ++s2) {
+      const uint32_t uu[4] = {u[s2].x, u[s2].y, u[s2].z, u[s2].w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        acc[2 * k] = fmaf(w[s2], __uint_as_float(uu[k] << 16), acc[2 * k]);
+        acc[2 * k + 1] = fmaf(w[s2], __uint_as_float(uu[k] & 0xFFFF0000u), acc[2 * k + 1]);
+      }
+    }
+    *(uint4*)(orow + d) = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]),
+                                     pack_bf16x2(acc[4], acc[5]), pack_bf16x2(acc[6], acc[7]));
+  }
+}
+
 __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_constant__ AtMaps maps, AtParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -614,49 +671,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       if (!ok) {
         if (lane == 0) raise_error(p.err, ERR_TIMEOUT);
       } else if (r < vrows) {
-        const int Sp = p.splits, ngs = cps / 8;
-        const uint4* og = (const uint4*)smem + r;   // [s][g][row]
-        const float2* ml = (const float2*)(smem + (size_t)Sp * ngs * AT_BM * 16) + r;   // [s][row]
-        float wgt[16];
-        float M = -INFINITY;
-#pragma unroll
-        for (int s2 = 0; s2 < 16; ++s2) {
-          if (s2 >= Sp) break;
-          const float2 v = ml[s2 * AT_BM];
-          wgt[s2] = v.x;
-          M = fmaxf(M, v.x);
-        }
-        float L = 0.f;
-#pragma unroll
-        for (int s2 = 0; s2 < 16; ++s2) {
-          if (s2 >= Sp) break;
-          const float l_s = ml[s2 * AT_BM].y;
-          wgt[s2] = (wgt[s2] == -INFINITY) ? 0.f : exp2f(wgt[s2] - M) * l_s;
-          L += wgt[s2];
-        }
-        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const int ngs = cps / 8;
+        const uint32_t og = smem_u32(smem);
+        const uint32_t ml = og + (uint32_t)(p.splits * ngs * AT_BM) * 16u;
         const int t = r / p.G, hh = r % p.G;
         const int j = qt * p.TQ + t;
         bf16* orow = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
-        for (int gq = 0; gq < ngs; ++gq) {
-          const int d = split * cps + 8 * gq;
-          if (d >= p.hd) break;
-          float acc[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) acc[k] = 0.f;
-#pragma unroll
-          for (int s2 = 0; s2 < 16; ++s2) {
-            if (s2 >= Sp) break;
-            const uint4 u = og[(size_t)(s2 * ngs + gq) * AT_BM];
-            const uint32_t uu[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              acc[2 * k] += wgt[s2] * __uint_as_float(uu[k] << 16);
-              acc[2 * k + 1] += wgt[s2] * __uint_as_float(uu[k] & 0xFFFF0000u);
-            }
-          }
-          *(uint4*)(orow + d) = make_uint4(pack_bf16x2(acc[0] * inv, acc[1] * inv), pack_bf16x2(acc[2] * inv, acc[3] * inv),
-                                           pack_bf16x2(acc[4] * inv, acc[5] * inv), pack_bf16x2(acc[6] * inv, acc[7] * inv));
+        switch (p.splits) {
+          case 2: xch_combine<2>(og, ml, r, ngs, split * cps, p.hd, orow); break;
+          case 4: xch_combine<4>(og, ml, r, ngs, split * cps, p.hd, orow); break;
+          case 8: xch_combine<8>(og, ml, r, ngs, split * cps, p.hd, orow); break;
+          default: xch_combine<16>(og, ml, r, ngs, split * cps, p.hd, orow); break;
         }
       }
     }

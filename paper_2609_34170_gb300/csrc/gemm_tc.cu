@@ -141,23 +141,41 @@ __device__ __forceinline__ void reduce_splits_l2(const float* b0, int S, size_t 
 }
 
 // V^T side output of the QKV projection for tokens m0 .. m0+nv-1 of this
-// thread's tile row: token m -> (robot m / T, key m % T).
+// thread's tile row: token m -> (robot m / T, key m % T).  Eight keys that
+// start on a multiple of 8 within one robot go out as one 16-byte store (rows
+// of V^T are a multiple of 8 keys apart), the rest one by one.
 template <int NV = 16>
 __device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, int nv, int r, const float v[NV]) {
   const int n = tile_n * TC_BM + r;
   if (n < p.v_col0 || n >= p.N) return;
   const float bb = p.bias ? p.bias[n] : 0.f;
   const int g = (n - p.v_col0) / p.vt_hd, d = (n - p.v_col0) % p.vt_hd;
-  int rb = m0 / p.vt_tokens, kk = m0 % p.vt_tokens;
+  const int T = p.vt_tokens;
+  int rb = m0 / T, kk = m0 % T;
   bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
 #pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    if (i >= nv) break;
-    dst[kk] = __float2bfloat16_rn(v[i] + bb);
-    if (++kk == p.vt_tokens) {
-      kk = 0;
-      ++rb;
-      dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
+  for (int i0 = 0; i0 < NV; i0 += 8) {
+    if (i0 >= nv) break;
+    if ((kk & 7) == 0 && kk + 8 <= T && i0 + 8 <= nv) {
+      *(uint4*)(dst + kk) = make_uint4(pack_bf16x2(v[i0] + bb, v[i0 + 1] + bb), pack_bf16x2(v[i0 + 2] + bb, v[i0 + 3] + bb),
+                                       pack_bf16x2(v[i0 + 4] + bb, v[i0 + 5] + bb), pack_bf16x2(v[i0 + 6] + bb, v[i0 + 7] + bb));
+      kk += 8;
+      if (kk == T) {
+        kk = 0;
+        ++rb;
+        dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
+      }
+    } else {
+#pragma unroll
+      for (int i = i0; i < i0 + 8; ++i) {
+        if (i >= nv) break;
+        dst[kk] = __float2bfloat16_rn(v[i] + bb);
+        if (++kk == T) {
+          kk = 0;
+          ++rb;
+          dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
+        }
+      }
     }
   }
 }
