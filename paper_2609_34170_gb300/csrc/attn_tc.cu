@@ -592,20 +592,29 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         const float m_s = has ? m_used : -INFINITY, l_s = has ? l : 0.f;
         for (int q = 0; q < p.splits; ++q) st_async_f2(mapa_shared(ml0, (uint32_t)q), m_s, l_s, mapa_shared(bar0, (uint32_t)q));
       }
-      const int nch = p.hdp / 16;
-      int ch = (split * cps) / 16;
-      uint32_t cur[16];
-      tmem_ld16_async(lane_base + o_col + 16 * ch, cur);
+      // 32 columns per TMEM load (16 where hdp is not a multiple of 32), the
+      // next load in flight while this one goes out
+      const int cw = (p.hdp % 32 == 0) ? 32 : 16;
+      const int nch = p.hdp / cw;
+      int ch = (split * cps) / cw;
+      uint32_t cur[32];
+      if (cw == 32) tmem_ld32_async(lane_base + o_col + 32 * ch, cur);
+      else tmem_ld16_async(lane_base + o_col + 16 * ch, cur);
       tmem_wait_ld();
       tmem_reg_fence16(cur);
+      tmem_reg_fence16(cur + 16);
       for (int jj = 0; jj < nch; ++jj) {
         const int chn = ch + 1 == nch ? 0 : ch + 1;
-        uint32_t nxt[16];
-        if (jj + 1 < nch) tmem_ld16_async(lane_base + o_col + 16 * chn, nxt);
+        uint32_t nxt[32];
+        if (jj + 1 < nch) {
+          if (cw == 32) tmem_ld32_async(lane_base + o_col + 32 * chn, nxt);
+          else tmem_ld16_async(lane_base + o_col + 16 * chn, nxt);
+        }
         if (snd) {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {   // two groups of 8 columns
-            const int gidx = 2 * ch + h;
+          for (int h = 0; h < 4; ++h) {   // groups of 8 columns
+            if (8 * h >= cw) break;
+            const int gidx = (cw / 8) * ch + h;
             const int dst = gidx / ngs, gl = gidx - dst * ngs;
             uint4 w;
             w.x = pack_bf16x2(__uint_as_float(cur[8 * h]) * inv, __uint_as_float(cur[8 * h + 1]) * inv);
@@ -620,8 +629,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         if (jj + 1 < nch) {
           tmem_wait_ld();
           tmem_reg_fence16(nxt);
+          tmem_reg_fence16(nxt + 16);
 #pragma unroll
-          for (int k = 0; k < 16; ++k) cur[k] = nxt[k];
+          for (int k = 0; k < 32; ++k) cur[k] = nxt[k];
         }
         ch = chn;
       }
@@ -803,8 +813,23 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   p.out = (bf16*)a.out; p.ld_out = a.ld_out;
   p.err = a.err;
   p.scale_log2 = 1.4426950408889634f / sqrtf((float)a.hd);
-  const int nctas = p.q_tiles * a.B * a.Hkv;
   const int C = p.n_pre + p.n_kv;
+  // when the keys will be split (the grid leaves most SMs idle), query tiles
+  // of 64 rows: the merge moves every split's rows x hd partial between the
+  // SMs of the cluster, so its time grows with the rows of a tile, while the
+  // MMAs (always 128 rows) and the key loads of a split do not; the grid
+  // (at up to 8 splits) stays within half the SMs, which are free while the
+  // previous kernel still holds the rest, so that every CTA starts early
+  {
+    const int tq_small = std::max(1, 64 / p.G);
+    const int qt_small = (a.H + tq_small - 1) / tq_small;
+    if (p.q_tiles * a.B * a.Hkv * 2 <= a.num_sms && tq_small < p.TQ && qt_small * a.B * a.Hkv * 8 <= a.num_sms / 2 &&
+        (C + 1) / 2 >= 2) {
+      p.q_tiles = qt_small;
+      p.TQ = (a.H + qt_small - 1) / qt_small;
+    }
+  }
+  const int nctas = p.q_tiles * a.B * a.Hkv;
   // split the key chunks only when the (b, g, q-tile) grid leaves most SMs
   // idle; about two chunks per split so S(i+1) overlaps the softmax of i
   // the splits of a query tile form one cluster (power of two, <= 16) whose
