@@ -84,6 +84,7 @@ struct TcParams {
   uint32_t box_bytes;   // bytes of one TMA output box (1024-aligned)
   uint32_t stg_off;     // SIMT transpose tile, or two TMA output boxes
   uint32_t xch_off;     // GeGLU exchange
+  uint32_t vts_off;     // V^T side output (TMA epilogue): the chunk as [128 tile rows][box_m + 10] bf16
   uint32_t rcv_off;     // RED_DSMEM: the partials received from the splits, [split][cpr / 4][128 rows]
                         // float4, overlaid on the operand ring (free once every CTA of the cluster
                         // has finished its MMAs), else on the output boxes + exchange (used only
@@ -308,6 +309,11 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
   epi_bar();
 }
 
+// The V^T staging tile of the TMA epilogue.
+__device__ __forceinline__ bf16* vt_stage(const TcParams& p, uint8_t* boxes) {
+  return (bf16*)(boxes - p.stg_off + p.vts_off);
+}
+
 // TMA epilogue of tokens m0 .. m0+box_m-1 of tile row block tile_n: v[i] is
 // this thread's tile row r at token m0+i, brow its bias.  All 128 epilogue
 // threads call it together.  The chunk is written into output box `ebuf` in
@@ -318,11 +324,24 @@ template <int NV = 16>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* tmO, int tile_n, int m0, int r,
                                              const float v[NV], float brow, uint8_t* boxes, float* xch, int& ebuf) {
   const int bm = p.box_m;   // <= NV
-  if (p.vt) store_vt<NV>(p, tile_n, m0, min(bm, p.M - m0), r, v);
-  // the box written two chunks ago must have been read by its TMA store
+  // the box written two chunks ago must have been read by its TMA store (and
+  // every thread is done with the V^T tile of the previous chunk)
   if (threadIdx.x == 64) bulk_wait_read<1>();
   epi_bar();
   uint8_t* box = boxes + (size_t)ebuf * p.box_bytes;
+  const int vpitch = bm + 10;   // bf16 per V^T tile row: an odd number of words, no bank conflicts
+  // V^T side output through a transposed staging tile (below); one path for
+  // every chunk: a second, register-to-global path made the kernel's code, and
+  // every launch of it, slower
+  const bool vtile = p.vt && (tile_n + 1) * TC_BM > p.v_col0;
+  if (vtile) {   // this thread's row of the chunk, feature-major, for the V^T side output below
+    uint32_t* vrow = (uint32_t*)(vt_stage(p, boxes) + (size_t)r * vpitch);
+#pragma unroll
+    for (int i = 0; i < NV; i += 2) {
+      if (i >= bm) break;
+      vrow[i / 2] = pack_bf16x2(v[i] + brow, v[i + 1] + brow);
+    }
+  }
   if (p.epi == EPI_GEGLU) {
     // tile rows 0..63 are gate features, 64..127 the matching up features:
     // transpose through xch so that every thread then forms 8 outputs of one
@@ -386,6 +405,23 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
     if (p.epi == EPI_ADD_F32) tma_reduce_add_2d(tmO, box, tile_n * TC_BM, m0);
     else tma_store_2d(tmO, box, p.epi == EPI_GEGLU ? tile_n * 64 : tile_n * TC_BM, m0);
     bulk_commit();
+  }
+  if (vtile) {
+    // V columns of the QKV projection also go out transposed, V^T[robot][g][d][key]:
+    // warp w writes tile rows 32w..32w+31 one after the other, lane i the
+    // chunk's token i, so that each store covers one contiguous run of keys
+    const bf16* vs = vt_stage(p, boxes);
+    const int w = (threadIdx.x >> 5) & 3, lane = threadIdx.x & 31;
+    const int m = m0 + lane;
+    if (lane < bm && m < p.M) {
+      const int rb = m / p.vt_tokens, kk = m - rb * p.vt_tokens;
+      bf16* vb = p.vt + (size_t)rb * p.vt_hkv * p.vt_hd * p.vt_kvp + kk;   // row (g, d) is (g*hd + d)*kvp further
+      for (int fi = 0; fi < 32; ++fi) {
+        const int f = 32 * w + fi, n = tile_n * TC_BM + f;
+        if (n < p.v_col0 || n >= p.N) continue;
+        vb[(size_t)(n - p.v_col0) * p.vt_kvp] = vs[(size_t)f * vpitch + lane];
+      }
+    }
   }
   ebuf ^= 1;
 }
@@ -971,7 +1007,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const int es = out_bf ? 2 : 4;
   const bool tma_out = reduce != RED_WORKSPACE && ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * es) % 16 == 0;
   int box_m = 0;
-  uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, rcv_off = 0, bar_off = 0;
+  uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, vts_off = 0, rcv_off = 0, bar_off = 0;
   size_t smem = 0;
   auto layout = [&](bool dsmem) {
     box_m = splits == 1 ? 16
@@ -980,13 +1016,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
     box_bytes = (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
     const size_t stg_bytes = tma_out ? 2 * (size_t)box_bytes : (STG_BYTES + 1023) / 1024 * 1024;
     const size_t xch_bytes = (tma_out && g.epi == EPI_GEGLU) ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
+    const size_t vts_bytes = (tma_out && g.vt) ? ((size_t)TC_BM * (box_m + 10) * 2 + 1023) / 1024 * 1024 : 0;
     // received partials (all splits' slices of this rank) overlay the operand
     // ring, else the boxes + exchange
     const size_t rcv_bytes = dsmem ? (size_t)TC_BM * bn * 4 : 0;
     const bool in_ring = rcv_bytes <= ring;
     xch_off = stg_off + (uint32_t)stg_bytes;
+    vts_off = xch_off + (uint32_t)xch_bytes;
     rcv_off = in_ring ? 0u : stg_off;
-    bar_off = stg_off + (uint32_t)std::max(stg_bytes + xch_bytes, in_ring ? (size_t)0 : rcv_bytes);
+    bar_off = stg_off + (uint32_t)std::max(stg_bytes + xch_bytes + vts_bytes, in_ring ? (size_t)0 : rcv_bytes);
     smem = 1024 + bar_off + (size_t)(2 * stages + 5) * 8 + 4 + 16 + 64;
   };
   // partials by st.async into the owning rank's shared memory when the token
@@ -1011,7 +1049,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
-             rcv_off, bar_off};
+             vts_off, rcv_off, bar_off};
   const dim3 grid = splits > 1 ? dim3(tiles_n, tiles_m, splits) : dim3(grid_ctas);
   const dim3 block(TC_THREADS);
   switch (reduce) {
