@@ -38,6 +38,7 @@
 
 #include <algorithm>
 #include <cstring>
+#include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -59,6 +60,16 @@ constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
 constexpr uint32_t XCH_BYTES = 32 * STG_LD * 4;  // GeGLU transpose tile (TMA epilogue): <= 32 tokens x 128 rows
 
 enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3 };
+// Epilogue kind of an instantiation: outputs through TMA boxes as fp32, bf16
+// (+ the V^T side output), a reduce-add into the fp32 residual stream or the
+// GeGLU pair -- fixed, so that a long persistent launch carries only the code
+// of its own epilogue -- or any of these chosen at run time (EK_TMA_ANY: the
+// short split-K launches of one step then all run one binary, whose code the
+// previous launch has left in the SM's instruction cache), or stored by the
+// threads (EK_GENERIC: any epilogue; unaligned outputs and the workspace
+// reduction).
+enum { EK_F32 = 0, EK_BF16 = 1, EK_ADD = 2, EK_GEGLU = 3, EK_GENERIC = 4, EK_TMA_ANY = 5 };
+
 
 struct TcParams {
   int M, N, K;
@@ -91,6 +102,11 @@ struct TcParams {
                         // after the sum)
   uint32_t bar_off;     // mbarriers, TMEM slot, flags
 };
+
+// The TMA epilogue kind of a launch (EK_F32 .. EK_GEGLU).
+__device__ __forceinline__ int tma_kind(const TcParams& p) {
+  return p.epi == EPI_GEGLU ? EK_GEGLU : p.epi == EPI_ADD_F32 ? EK_ADD : p.out_bf16 ? EK_BF16 : EK_F32;
+}
 
 // The i-th work item of this CTA: a tile (tn, tm) and split sp.  With splits
 // the grid is (tiles_n, tiles_m, splits) and every CTA has one item; without,
@@ -320,9 +336,9 @@ __device__ __forceinline__ bf16* vt_stage(const TcParams& p, uint8_t* boxes) {
 // shared memory (token-major, as the output), and thread 64 sends the box
 // with one TMA store (EPI_ADD_F32: TMA reduce-add into the residual stream);
 // rows past M and columns past N are clipped by the tensor map.
-template <int NV = 16>
+template <int EK, int NV = 16>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* tmO, int tile_n, int m0, int r,
-                                             const float v[NV], float brow, uint8_t* boxes, float* xch, int& ebuf) {
+                                             const float* v, float brow, uint8_t* boxes, float* xch, int& ebuf) {
   const int bm = p.box_m;   // <= NV
   // the box written two chunks ago must have been read by its TMA store (and
   // every thread is done with the V^T tile of the previous chunk)
@@ -333,7 +349,8 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   // V^T side output through a transposed staging tile (below); one path for
   // every chunk: a second, register-to-global path made the kernel's code, and
   // every launch of it, slower
-  const bool vtile = p.vt && (tile_n + 1) * TC_BM > p.v_col0;
+  const int kind = EK == EK_TMA_ANY ? tma_kind(p) : EK;   // a constant in the fixed-kind instantiations
+  const bool vtile = kind == EK_BF16 && p.vt && (tile_n + 1) * TC_BM > p.v_col0;
   if (vtile) {   // this thread's row of the chunk, feature-major, for the V^T side output below
     uint32_t* vrow = (uint32_t*)(vt_stage(p, boxes) + (size_t)r * vpitch);
 #pragma unroll
@@ -342,7 +359,7 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
       vrow[i / 2] = pack_bf16x2(v[i] + brow, v[i + 1] + brow);
     }
   }
-  if (p.epi == EPI_GEGLU) {
+  if (kind == EK_GEGLU) {
     // tile rows 0..63 are gate features, 64..127 the matching up features:
     // transpose through xch so that every thread then forms 8 outputs of one
     // token (the GELUs spread over all 128 threads)
@@ -366,7 +383,7 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
                        pack_bf16x2(gelu_tanh_f(gb.z) * ub.z, gelu_tanh_f(gb.w) * ub.w));
       }
     }
-  } else if (p.out_bf16) {
+  } else if (kind == EK_BF16) {
     // (each loop stops at the box width: a short slice runs, and fetches,
     // only its own iterations)
     bf16* o = (bf16*)box;
@@ -385,7 +402,7 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
     }
   } else {
     float* o = (float*)box;
-    if (p.epi == EPI_STORE_SILU) {
+    if (kind == EK_F32 && p.epi == EPI_STORE_SILU) {
 #pragma unroll
       for (int i = 0; i < NV; ++i) {
         if (i >= bm) break;
@@ -402,8 +419,8 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   epi_bar();
   if (threadIdx.x == 64) {
-    if (p.epi == EPI_ADD_F32) tma_reduce_add_2d(tmO, box, tile_n * TC_BM, m0);
-    else tma_store_2d(tmO, box, p.epi == EPI_GEGLU ? tile_n * 64 : tile_n * TC_BM, m0);
+    if (kind == EK_ADD) tma_reduce_add_2d(tmO, box, tile_n * TC_BM, m0);
+    else tma_store_2d(tmO, box, kind == EK_GEGLU ? tile_n * 64 : tile_n * TC_BM, m0);
     bulk_commit();
   }
   if (vtile) {
@@ -426,9 +443,10 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   ebuf ^= 1;
 }
 
-// RED = p.reduce, fixed per instantiation so that each reduction mode gets
-// its own register allocation.
-template <int RED>
+// RED = p.reduce and EK = the epilogue kind, fixed per instantiation so that
+// each reduction mode gets its own register allocation and each launch only
+// the code it runs.
+template <int RED, int EK>
 __global__ void __launch_bounds__(TC_THREADS, 2)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                    const __grid_constant__ CUtensorMap tmO, TcParams p) {
@@ -457,6 +475,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   const int kb1_first = (int)((long)(sp0 + 1) * p.num_kb / p.splits);
   const int npre = has_work ? min(S, kb1_first - kb0_first) : 0;
   const int cpr = BN / p.splits;   // tokens of the slice each split rank owns (a multiple of 4)
+  constexpr bool TMA_OUT = EK != EK_GENERIC;
 
   pdl_trigger();
   uint64_t pol_w = 0, pol_x = 0;
@@ -479,7 +498,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     // tiles while the previous kernel is still finishing.
     asm volatile("prefetch.tensormap [%0];" ::"l"(&tmW) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(&tmX) : "memory");
-    if (p.tma_out) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
+    if (TMA_OUT) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
     if (p.oneshot) {
@@ -643,7 +662,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
             tc_fence_before();
             mbar_arrive(&acc_empty[b]);
           }
-          if (p.tma_out) epilogue_tma(p, &tmO, tn, m_base + c0, r, v, brow, stg_raw, xch, ebuf);
+          if constexpr (TMA_OUT) epilogue_tma<EK>(p, &tmO, tn, m_base + c0, r, v, brow, stg_raw, xch, ebuf);
           else epilogue_chunk(p, tn, m_base + c0, 16, r, v, stage);
           if (more) {
             tmem_wait_ld();
@@ -740,7 +759,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       }
     }
     // every TMA output box has been written to global memory
-    if (p.tma_out && threadIdx.x == 64) bulk_wait<0>();
+    if (TMA_OUT && threadIdx.x == 64) bulk_wait<0>();
   }
   tc_fence_before();
   cta_sync();
@@ -782,7 +801,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
           default: reduce_slice_smem<8>(b0, p.splits, v); break;
         }
         int ebuf = 0;
-        epilogue_tma<32>(p, &tmO, tn0, tm0 * BN + sp0 * cpr, r, v, brow, stg_raw, xch, ebuf);
+        if constexpr (TMA_OUT) epilogue_tma<EK, 32>(p, &tmO, tn0, tm0 * BN + sp0 * cpr, r, v, brow, stg_raw, xch, ebuf);
         if (threadIdx.x == 64) bulk_wait<0>();
       }
     }
@@ -804,7 +823,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       int ebuf = 0;
       // a slice that would take three or more 4- or 8-token chunks goes out
       // whole: one L2 round trip, one output box
-      const bool whole = p.tma_out && cpr <= 32 && cpr > 8 && cpr % 16 != 0;
+      const bool whole = TMA_OUT && cpr <= 32 && cpr > 8 && cpr % 16 != 0;
       if (whole) {
         float v[32];
 #pragma unroll
@@ -819,7 +838,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
           case 7: reduce_slice_l2<7>(base, Sp, sstride, v); break;
           default: reduce_slice_l2<8>(base, Sp, sstride, v); break;
         }
-        epilogue_tma<32>(p, &tmO, tn0, tm0 * BN + rank * cpr, r, v, brow, stg_raw, xch, ebuf);
+        if constexpr (TMA_OUT) epilogue_tma<EK, 32>(p, &tmO, tn0, tm0 * BN + rank * cpr, r, v, brow, stg_raw, xch, ebuf);
       }
       for (int cc = 0; !whole && cc < cpr; cc += p.box_m) {
         const int nc = p.box_m;
@@ -831,16 +850,33 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         else if (nc == 8) reduce_splits_l2<2>(b0, Sp, sstride, v);
         else reduce_splits_l2<1>(b0, Sp, sstride, v);
         const int m0 = tm0 * BN + rank * cpr + cc;
-        if (p.tma_out) epilogue_tma(p, &tmO, tn0, m0, r, v, brow, stg_raw, xch, ebuf);
+        if constexpr (TMA_OUT) epilogue_tma<EK>(p, &tmO, tn0, m0, r, v, brow, stg_raw, xch, ebuf);
         else epilogue_chunk(p, tn0, m0, nc, r, v, stage);
       }
-      if (p.tma_out && threadIdx.x == 64) bulk_wait<0>();
+      if (TMA_OUT && threadIdx.x == 64) bulk_wait<0>();
     }
   }
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
   }
+}
+
+using TcKernel = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, TcParams);
+
+// The instantiation for a reduction mode and epilogue kind (nullptr where the
+// pair cannot occur: the workspace mode stores from the threads, the
+// shared-memory exchange needs TMA outputs).
+TcKernel tc_kernel(int red, int ek) {
+#define RAVEL_TC_K(R, E) \
+  if (red == R && ek == E) return tc_gemm_kernel<R, E>;
+  RAVEL_TC_K(RED_NONE, EK_F32) RAVEL_TC_K(RED_NONE, EK_BF16) RAVEL_TC_K(RED_NONE, EK_ADD)
+  RAVEL_TC_K(RED_NONE, EK_GEGLU) RAVEL_TC_K(RED_NONE, EK_GENERIC)
+  RAVEL_TC_K(RED_L2_CLUSTER, EK_TMA_ANY) RAVEL_TC_K(RED_L2_CLUSTER, EK_GENERIC)
+  RAVEL_TC_K(RED_DSMEM, EK_TMA_ANY)
+  RAVEL_TC_K(RED_WORKSPACE, EK_GENERIC)
+#undef RAVEL_TC_K
+  return nullptr;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -925,8 +961,10 @@ int g_max_cluster = 8;   // largest power-of-two cluster the split-K reduction m
 cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
-  const void* kernels[] = {(const void*)tc_gemm_kernel<RED_NONE>, (const void*)tc_gemm_kernel<RED_L2_CLUSTER>,
-                           (const void*)tc_gemm_kernel<RED_WORKSPACE>, (const void*)tc_gemm_kernel<RED_DSMEM>};
+  std::vector<const void*> kernels;
+  for (int red = 0; red < 4; ++red)
+    for (int ek = 0; ek <= EK_TMA_ANY; ++ek)
+      if (TcKernel k = tc_kernel(red, ek)) kernels.push_back((const void*)k);
   for (const void* k : kernels) {
     e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
     if (e != cudaSuccess) return e;
@@ -947,7 +985,8 @@ cudaError_t init_tc_gemm() {
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel<RED_L2_CLUSTER>, &cfg) == cudaSuccess && n > 0) g_max_cluster = 16;
+    if (cudaOccupancyMaxActiveClusters(&n, tc_kernel(RED_L2_CLUSTER, EK_GENERIC), &cfg) == cudaSuccess && n > 0)
+      g_max_cluster = 16;
   }
   cudaGetLastError();
   return cudaSuccess;
@@ -1052,14 +1091,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
              vts_off, rcv_off, bar_off};
   const dim3 grid = splits > 1 ? dim3(tiles_n, tiles_m, splits) : dim3(grid_ctas);
   const dim3 block(TC_THREADS);
-  switch (reduce) {
-    case RED_NONE: return launch_kernel(tc_gemm_kernel<RED_NONE>, grid, block, smem, st, 1u, mw, mx, mo, p);
-    case RED_L2_CLUSTER:
-      return launch_kernel(tc_gemm_kernel<RED_L2_CLUSTER>, grid, block, smem, st, (unsigned)splits, mw, mx, mo, p);
-    case RED_DSMEM:
-      return launch_kernel(tc_gemm_kernel<RED_DSMEM>, grid, block, smem, st, (unsigned)splits, mw, mx, mo, p);
-    default: return launch_kernel(tc_gemm_kernel<RED_WORKSPACE>, grid, block, smem, st, 1u, mw, mx, mo, p);
-  }
+  // persistent launches: one instantiation per epilogue kind; split-K
+  // launches: one for all TMA epilogues
+  const int ek = !tma_out ? EK_GENERIC
+                 : reduce != RED_NONE ? EK_TMA_ANY
+                 : g.epi == EPI_GEGLU ? EK_GEGLU : g.epi == EPI_ADD_F32 ? EK_ADD : out_bf ? EK_BF16 : EK_F32;
+  const TcKernel k = tc_kernel(reduce, ek);
+  if (!k) return cudaErrorInvalidConfiguration;
+  const bool clustered = reduce == RED_L2_CLUSTER || reduce == RED_DSMEM;
+  return launch_kernel(k, grid, block, smem, st, clustered ? (unsigned)splits : 1u, mw, mx, mo, p);
 }
 
 }  // namespace ravel
