@@ -862,7 +862,239 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Two-SM GEMM (persistent, many tiles): a pair of CTAs (a cluster of 2) runs
+// one M = 256 MMA per K step -- A = 256 weight rows, 128 in each CTA's shared
+// memory, B = BN tokens, BN / 2 in each -- and each CTA's TMEM accumulates its
+// own 128 rows for all BN tokens.  Per K step an SM then streams 128 + BN/2
+// operand rows through TMA and the MMA instead of 128 + BN, which is what
+// bounds the one-SM tile's main loop.  The even CTA's thread issues the MMAs
+// and owns the stage barriers: both CTAs load their halves into their own
+// shared memory and count the bytes on the even CTA's `full` barrier; the
+// MMA completion is multicast to both CTAs' `empty` / `acc_full` barriers;
+// both CTAs run the epilogue of their own rows, whose drained accumulators
+// the even CTA's `acc_empty` counts (256 arrivals).
+template <int EK>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                        const __grid_constant__ CUtensorMap tmO, TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int BN = p.bn, BNh = BN / 2, S = p.stages;
+  const uint32_t bh_bytes = (uint32_t)BNh * TC_BK * 2;
+  const uint32_t stage_tx = 2u * (TC_A_BYTES + bh_bytes);   // both CTAs' halves of a stage
+  uint8_t* a_s = smem;
+  uint8_t* b_s = smem + (size_t)S * TC_A_BYTES;
+  uint8_t* stg_raw = smem + p.stg_off;
+  float* xch = (float*)(smem + p.xch_off);
+  uint64_t* full = (uint64_t*)(smem + p.bar_off);   // the even CTA's count both halves
+  uint64_t* empty = full + S;
+  uint64_t* acc_full = empty + S;      // [2]
+  uint64_t* acc_empty = acc_full + 2;  // [2] the even CTA's: 256 arrivals
+  uint32_t* tmem_slot = (uint32_t*)(acc_empty + 2);
+  int* flags = (int*)(tmem_slot + 1);  // [0] abort, [2] stages issued, [3] stages consumed
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int pair = (int)(blockIdx.x >> 1), npairs = (int)(gridDim.x >> 1);
+  const uint32_t ncols = 2 * p.acc_cols;
+  // work item i of this pair: pair tile pair + i * npairs = (256-row block tn2, token tile tm)
+  auto item = [&](int i, int& tn2, int& tm) -> bool {
+    const int t = pair + i * npairs;
+    if (t >= p.num_tiles) return false;
+    tm = t % p.tiles_m;
+    tn2 = t / p.tiles_m;
+    return true;
+  };
+  int tn0 = 0, tm0 = 0;
+  const bool has_work = item(0, tn0, tm0);
+  const int npre = has_work ? min(S, p.num_kb) : 0;
+  constexpr bool TMA_OUT = EK != EK_GENERIC;
+  static_assert(TMA_OUT, "the pair kernel stores through TMA boxes");
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 256);
+    }
+    flags[0] = flags[1] = flags[2] = flags[3] = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  // both CTAs' barriers exist before either signals the other's
+  cluster_sync();
+  const uint32_t full0 = mapa_shared(smem_u32(full), 0);          // the even CTA's full[0]
+  const uint32_t acc_empty0 = mapa_shared(smem_u32(acc_empty), 0);
+  uint64_t pol_w = 0, pol_x = 0;
+  if (threadIdx.x == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&tmW) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&tmX) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
+    // the first stages' weight halves, before the wait on the previous kernel
+    for (int i = 0; i < npre; ++i) {
+      if (leader) mbar_expect_tx(&full[i], stage_tx);
+      tma_load_2d_pair(&tmW, full0 + 8u * (uint32_t)i, a_s + (size_t)i * TC_A_BYTES, i * TC_BK,
+                       (2 * tn0 + (int)rank) * TC_BM, pol_w);
+    }
+  }
+  pdl_wait();
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  cta_sync();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {   // producer (both CTAs): this CTA's A rows and B half of each stage
+      int it = 0;
+      bool ok = true;
+      int tn2, tm;
+      for (int i = 0; ok && item(i, tn2, tm); ++i) {
+        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+          const int s = it % S;
+          const uint32_t fb = full0 + 8u * (uint32_t)s;
+          if (it < npre) {   // weight half already in flight
+            tma_load_2d_pair(&tmX, fb, b_s + (size_t)s * bh_bytes, kb * TC_BK, tm * BN + (int)rank * BNh, pol_x);
+            continue;
+          }
+          if (!mbar_wait(&empty[s], ((uint32_t)(it / S) & 1u) ^ 1u)) {
+            flags[0] = 1;
+            ok = false;
+            break;
+          }
+          if (leader) mbar_expect_tx(&full[s], stage_tx);
+          tma_load_2d_pair(&tmW, fb, a_s + (size_t)s * TC_A_BYTES, kb * TC_BK, (2 * tn2 + (int)rank) * TC_BM, pol_w);
+          tma_load_2d_pair(&tmX, fb, b_s + (size_t)s * bh_bytes, kb * TC_BK, tm * BN + (int)rank * BNh, pol_x);
+        }
+      }
+      flags[2] = it;
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {   // MMA issuer: the even CTA only
+      const uint32_t idesc = idesc_bf16(2 * TC_BM, BN);
+      int it = 0;
+      bool ok = true;
+      int tn2, tm;
+      for (int i = 0; ok && item(i, tn2, tm); ++i) {
+        const int b = i & 1;
+        // both CTAs' epilogues must have drained the accumulator of item i - 2
+        if (i >= 2 && !mbar_wait(&acc_empty[b], (uint32_t)((i >> 1) - 1) & 1u)) {
+          flags[0] = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)b * p.acc_cols;
+        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait(&full[s], (uint32_t)(it / S) & 1u)) {
+            flags[0] = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = sw128_desc(smem_u32(a_s + (size_t)s * TC_A_BYTES));
+          const uint64_t bd = sw128_desc(smem_u32(b_s + (size_t)s * bh_bytes));
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k) umma_bf16_pair(d, ad + 2 * k, bd + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit_pair_mc(&empty[s], 3);   // both CTAs' halves of the stage are free
+        }
+        if (ok) umma_commit_pair_mc(&acc_full[b], 3);
+      }
+      flags[3] = it;
+    }
+    __syncwarp();
+  } else {
+    // epilogue warps 2..5 of both CTAs: TMEM lane quarter q, this CTA's tile row r
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    int ebuf = 0;
+    int tn2, tm;
+    for (int i = 0; item(i, tn2, tm); ++i) {
+      const int b = i & 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[b], (uint32_t)(i >> 1) & 1u));
+      if (!ok) {
+        if (lane == 0) flags[0] = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)b * p.acc_cols;
+      const int tile_n = 2 * tn2 + (int)rank;   // this CTA's 128-row block
+      const int m_base = tm * BN;
+      const int n = tile_n * TC_BM + r;
+      const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
+      // 32-token chunks (BN is a multiple of 32): half the barriers and box
+      // hand-offs per token of 16-token chunks
+      uint32_t nxt[32];
+      tmem_ld32_async(trow, nxt);
+      tmem_wait_ld();
+      tmem_reg_fence16(nxt);
+      tmem_reg_fence16(nxt + 16);
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        float v[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(nxt[k]);
+        const bool more = c0 + 32 < BN;
+        if (more) {
+          tmem_ld32_async(trow + c0 + 32, nxt);
+        } else {   // this CTA's accumulator drained: tell the MMA issuer
+          tc_fence_before();
+          mbar_arrive_remote(acc_empty0 + 8u * (uint32_t)b);
+        }
+        epilogue_tma<EK, 32>(p, &tmO, tile_n, m_base + c0, r, v, brow, stg_raw, xch, ebuf);
+        if (more) {
+          tmem_wait_ld();
+          tmem_reg_fence16(nxt);
+          tmem_reg_fence16(nxt + 16);
+        }
+      }
+    }
+    if (threadIdx.x == 64) bulk_wait<0>();
+  }
+  tc_fence_before();
+  cta_sync();
+  if (flags[0]) {
+    // unwind: the even CTA waits (bounded) for stages issued but never consumed
+    if (threadIdx.x == 0) {
+      if (leader)
+        for (int i = flags[3]; i < flags[2]; ++i) mbar_wait(&full[i % S], (uint32_t)(i / S) & 1u);
+      raise_error(p.err, ERR_TIMEOUT);
+    }
+    cta_sync();
+  }
+  // neither CTA leaves while the other may still signal its barriers or
+  // (through the MMA) read its shared memory
+  cluster_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
+  }
+}
+
 using TcKernel = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, TcParams);
+
+TcKernel tc_pair_kernel(int ek) {
+  switch (ek) {
+    case EK_F32: return tc_gemm_pair_kernel<EK_F32>;
+    case EK_BF16: return tc_gemm_pair_kernel<EK_BF16>;
+    case EK_ADD: return tc_gemm_pair_kernel<EK_ADD>;
+    case EK_GEGLU: return tc_gemm_pair_kernel<EK_GEGLU>;
+    default: return nullptr;
+  }
+}
 
 // The instantiation for a reduction mode and epilogue kind (nullptr where the
 // pair cannot occur: the workspace mode stores from the threads, the
@@ -955,6 +1187,66 @@ int pick_bn(int M, int tiles_n, int num_sms) {
 }
 
 int g_max_cluster = 8;   // largest power-of-two cluster the split-K reduction may use
+bool g_pair_gemm = true;  // persistent launches of many tiles on SM pairs
+int g_pair_bn_max = 256;  // widest token tile of a pair launch
+
+// Two-SM launch of a persistent GEMM (see tc_gemm_pair_kernel): token-tile
+// width BN (a multiple of 32 in [128, 256]) minimising waves x (BN + 64) --
+// the work of a pair's tiles plus a fixed cost per tile of about 64 token
+// columns (accumulator hand-off and epilogue pipeline, ~1 us) -- larger BN on
+// ties; then the usual TMA epilogue layout.
+cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st, int ek,
+                             bool out_bf, int es) {
+  const int tiles_n = (g.N + TC_BM - 1) / TC_BM;
+  const int tiles_n2 = (g.N + 2 * TC_BM - 1) / (2 * TC_BM);
+  const int slots = num_sms / 2;
+  int bn = 256;
+  long best = -1;
+  for (int c = g_pair_bn_max; c >= 128; c -= 32) {
+    const long tiles = (long)tiles_n2 * ((g.M + c - 1) / c);
+    const long cost = (tiles + slots - 1) / slots * (c + 64);
+    if (best < 0 || cost < best) {
+      best = cost;
+      bn = c;
+    }
+  }
+  const int tiles_m = (g.M + bn - 1) / bn;
+  const int num_tiles = tiles_n2 * tiles_m;
+  const int num_kb = (g.K + TC_BK - 1) / TC_BK;
+  uint32_t acc_cols = 32;
+  while ((int)acc_cols < bn) acc_cols <<= 1;
+  const int box_m = 32;
+  const uint32_t box_bytes =
+      (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
+  const size_t stg_bytes = 2 * (size_t)box_bytes;
+  const size_t xch_bytes = g.epi == EPI_GEGLU ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
+  const size_t vts_bytes = g.vt ? ((size_t)TC_BM * (box_m + 10) * 2 + 1023) / 1024 * 1024 : 0;
+  const size_t fixed = 1024 + stg_bytes + xch_bytes + vts_bytes + 256;
+  const int stage_bytes = TC_A_BYTES + (bn / 2) * TC_BK * 2;
+  const int stages = std::min(8, (int)((TC_SMEM_MAX - fixed) / stage_bytes));
+  if (stages < 2) return cudaErrorInvalidConfiguration;
+  const size_t ring = ((size_t)stages * stage_bytes + 1023) / 1024 * 1024;
+  const uint32_t stg_off = (uint32_t)ring;
+  const uint32_t xch_off = stg_off + (uint32_t)stg_bytes;
+  const uint32_t vts_off = xch_off + (uint32_t)xch_bytes;
+  const uint32_t bar_off = vts_off + (uint32_t)vts_bytes;
+  const size_t smem = 1024 + bar_off + (size_t)(2 * stages + 4) * 8 + 4 + 16 + 64;
+  if (smem > (size_t)TC_SMEM_MAX) return cudaErrorInvalidConfiguration;
+  CUtensorMap mw, mx, mo;
+  cudaError_t e = encode_2d(&mw, g.W, g.N, g.K, g.ldw, TC_BM);
+  if (e == cudaSuccess) e = encode_2d(&mx, g.A, g.M, g.K, g.lda, bn / 2);
+  if (e == cudaSuccess)
+    e = encode_out(&mo, g.out, g.M, g.epi == EPI_GEGLU ? g.N / 2 : g.N, g.ldo, out_bf,
+                   g.epi == EPI_GEGLU ? 64 : TC_BM, box_m);
+  if (e != cudaSuccess) return e;
+  TcParams p{g.M, g.N, g.K, bn, stages, 1, num_kb, RED_NONE, (uint32_t)ring, acc_cols, tiles_n, tiles_m, num_tiles,
+             (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
+             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, 1, 0, box_m, box_bytes, stg_off, xch_off,
+             vts_off, 0, bar_off};
+  const int npairs = std::min(num_tiles, slots);
+  return launch_kernel_cluster(tc_pair_kernel(ek), dim3(2 * npairs), dim3(TC_THREADS), smem, st, dim3(2, 1, 1), mw, mx,
+                               mo, p);
+}
 
 }  // namespace
 
@@ -965,6 +1257,7 @@ cudaError_t init_tc_gemm() {
   for (int red = 0; red < 4; ++red)
     for (int ek = 0; ek <= EK_TMA_ANY; ++ek)
       if (TcKernel k = tc_kernel(red, ek)) kernels.push_back((const void*)k);
+  for (int ek = 0; ek < EK_GENERIC; ++ek) kernels.push_back((const void*)tc_pair_kernel(ek));
   for (const void* k : kernels) {
     e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_MAX);
     if (e != cudaSuccess) return e;
@@ -1023,6 +1316,17 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
     while (splits > 1 && ((size_t)splits * tiles * bn * TC_BM * 4 > ws.ws_bytes || tiles > ws.n_counters)) --splits;
   }
   int reduce = splits == 1 ? RED_NONE : (cluster ? RED_L2_CLUSTER : RED_WORKSPACE);
+  {
+    // two-SM tiles for a persistent launch whose pair tiles fill every pair of SMs
+    const bool obf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
+    const int oes = obf ? 2 : 4;
+    const bool aligned = ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * oes) % 16 == 0;
+    const long pair_tiles = (long)((g.N + 2 * TC_BM - 1) / (2 * TC_BM)) * ((g.M + 255) / 256);
+    if (cluster && g_pair_gemm && splits == 1 && aligned && pair_tiles >= num_sms / 2) {
+      const int ek = g.epi == EPI_GEGLU ? EK_GEGLU : g.epi == EPI_ADD_F32 ? EK_ADD : obf ? EK_BF16 : EK_F32;
+      return launch_gemm_pair(g, ws, num_sms, st, ek, obf, oes);
+    }
+  }
   const int cpr = bn / splits;   // a multiple of 4 whenever the splits form a cluster
   uint32_t acc_cols = 32;
   while ((int)acc_cols < bn) acc_cols <<= 1;

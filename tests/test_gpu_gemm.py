@@ -2,7 +2,9 @@
 for fp32) against numpy fp64 matmul of the same bf16 operands, through the C
 ABI (ravel_gemm).  Shapes cover single and multiple tiles, ragged token /
 feature / K tails, split-K (partials exchanged through shared memory for token
-slices of 4..32, through L2 for wider ones) and every epilogue."""
+slices of 4..32, through L2 for wider ones), persistent launches on one SM
+or on SM pairs (one 256-row MMA per K step across two CTAs) and every
+epilogue."""
 import numpy as np
 import pytest
 
@@ -33,7 +35,7 @@ def _rand(shape, seed, scale=1.0):
 
 
 SHAPES = [(1, 128, 64), (7, 100, 200), (50, 2560, 1024), (66, 1024, 2048), (50, 1024, 4096), (130, 384, 192),
-          (300, 256, 512), (3200, 1024, 1024), (51, 3000, 1024)]
+          (300, 256, 512), (3200, 1024, 1024), (51, 3000, 1024), (4224, 2560, 1024)]
 
 
 @pytest.mark.parametrize("M,N,K", SHAPES)
