@@ -1195,21 +1195,26 @@ int g_pair_bn_max = 256;  // widest token tile of a pair launch
 // the work of a pair's tiles plus a fixed cost per tile of about 64 token
 // columns (accumulator hand-off and epilogue pipeline, ~1 us) -- larger BN on
 // ties; then the usual TMA epilogue layout.
-cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st, int ek,
-                             bool out_bf, int es) {
-  const int tiles_n = (g.N + TC_BM - 1) / TC_BM;
-  const int tiles_n2 = (g.N + 2 * TC_BM - 1) / (2 * TC_BM);
-  const int slots = num_sms / 2;
+int pick_bn_pair(int M, int tiles_n2, int slots) {
   int bn = 256;
   long best = -1;
   for (int c = g_pair_bn_max; c >= 128; c -= 32) {
-    const long tiles = (long)tiles_n2 * ((g.M + c - 1) / c);
+    const long tiles = (long)tiles_n2 * ((M + c - 1) / c);
     const long cost = (tiles + slots - 1) / slots * (c + 64);
     if (best < 0 || cost < best) {
       best = cost;
       bn = c;
     }
   }
+  return bn;
+}
+
+cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st, int ek,
+                             bool out_bf, int es) {
+  const int tiles_n = (g.N + TC_BM - 1) / TC_BM;
+  const int tiles_n2 = (g.N + 2 * TC_BM - 1) / (2 * TC_BM);
+  const int slots = num_sms / 2;
+  const int bn = pick_bn_pair(g.M, tiles_n2, slots);
   const int tiles_m = (g.M + bn - 1) / bn;
   const int num_tiles = tiles_n2 * tiles_m;
   const int num_kb = (g.K + TC_BK - 1) / TC_BK;
@@ -1317,12 +1322,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   }
   int reduce = splits == 1 ? RED_NONE : (cluster ? RED_L2_CLUSTER : RED_WORKSPACE);
   {
-    // two-SM tiles for a persistent launch whose pair tiles fill every pair of SMs
+    // two-SM tiles for a persistent launch whose pair tiles fill at least
+    // three quarters of the pairs of SMs
     const bool obf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
     const int oes = obf ? 2 : 4;
     const bool aligned = ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * oes) % 16 == 0;
-    const long pair_tiles = (long)((g.N + 2 * TC_BM - 1) / (2 * TC_BM)) * ((g.M + 255) / 256);
-    if (cluster && g_pair_gemm && splits == 1 && aligned && pair_tiles >= num_sms / 2) {
+    const int tn2 = (g.N + 2 * TC_BM - 1) / (2 * TC_BM), slots = num_sms / 2;
+    const int pbn = pick_bn_pair(g.M, tn2, slots);
+    const long pair_tiles = (long)tn2 * ((g.M + pbn - 1) / pbn);
+    if (cluster && g_pair_gemm && splits == 1 && aligned && 4 * pair_tiles >= 3 * slots) {
       const int ek = g.epi == EPI_GEGLU ? EK_GEGLU : g.epi == EPI_ADD_F32 ? EK_ADD : obf ? EK_BF16 : EK_F32;
       return launch_gemm_pair(g, ws, num_sms, st, ek, obf, oes);
     }
