@@ -179,7 +179,8 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
  *       2: out += X W^T + bias (float32 out)
  *       3: GeGLU (bf16 handle, N % 128 == 0): W rows in 128-row blocks of 64
  *          gate rows then the 64 matching up rows; out[m][f] =
- *          gelu_tanh(gate) * up for f < N/2 (bias ignored)
+ *          gelu_tanh(gate + bias) * (up + bias) for f < N/2, each bias
+ *          that of its W row
  *   out device [M, ldo], out_dtype RAVEL_FP32 or RAVEL_BF16; bias device [N] or NULL
  * Enqueued on `stream`; uses the handle's split-K workspace, so it must not
  * overlap another call on the same handle. */
