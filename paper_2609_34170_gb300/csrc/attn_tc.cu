@@ -56,7 +56,9 @@ struct AtParams {
   int layer, Bmax, mask_mode;
   int nblk, k_slots, v_slots;         // head-dim blocks of 64; K and V^T ring depths
   int mc;                             // query tiles of a (b, g) pair sharing each K/V chunk by multicast (1 = none)
-  int xch;                            // splits > 1: partials through shared memory (1) or L2 (0)
+  int xch;                            // splits > 1: partials through L2 (0) or shared memory, sent once every
+                                      // split's MMAs are done (1: cluster barrier) or once every split's S
+                                      // MMAs are done (2: the receive area lies in Q and the K ring)
   uint32_t vt_bytes;                  // bytes of one transposed-V chunk (hd rows x 128 B)
   const int* ctx_state;
   bf16* out;
@@ -203,7 +205,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   uint64_t* p_full = s_free + 2;
   uint64_t* pv_done = p_full + 2;   // [2]: PV of chunk i completes pv_done[i & 1]
   uint64_t* rcv_bar = pv_done + 2;  // xch: every split's share of this rank has arrived
-  uint32_t* tmem_slot = (uint32_t*)(rcv_bar + 1);
+  uint64_t* sdone = rcv_bar + 1;    // xch 2: every split's last S MMA has completed (one arrival each)
+  uint32_t* tmem_slot = (uint32_t*)(sdone + 1);
   int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] K issued, [2] K consumed, [3] V issued, [4] V consumed
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -251,12 +254,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     mbar_init(&pv_done[0], 1);
     mbar_init(&pv_done[1], 1);
     mbar_init(rcv_bar, 1);
+    mbar_init(sdone, p.splits);
     flags[0] = flags[1] = flags[2] = flags[3] = flags[4] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     if (p.xch) mbar_expect_tx(rcv_bar, (uint32_t)(p.splits * vrows * (2 * cps + 8)));
   }
-  // with multicast, every CTA's barriers must exist before a peer targets them
-  if (p.mc > 1) cluster_sync();
+  // with multicast (or xch 2), every CTA's barriers must exist before a peer targets them
+  if (p.mc > 1 || p.xch == 2) cluster_sync();
   const int mrank = (p.mc > 1) ? (int)cluster_ctarank() : 0;
   const uint16_t mmask = (uint16_t)((1u << p.mc) - 1u);
   const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
@@ -373,9 +377,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       flags[3] = nv;
     }
     __syncwarp();
-    // xch: one arrival per thread on the cluster barrier that opens the
+    // xch 1: one arrival per thread on the cluster barrier that opens the
     // exchange (the softmax warps arrive once their last PV is complete)
-    if (p.xch) cluster_arrive_release();
+    if (p.xch == 1) cluster_arrive_release();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc_s = idesc_bf16(AT_BM, AT_BKV);
@@ -386,6 +390,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       // chain every chunk's load behind the previous PV).  S runs at most one
       // chunk ahead of PV (two S buffers in TMEM).
       int ns = 0, i = 0;   // next S, next PV
+      bool sdone_sent = false;
+      // xch 2: every split learns when this split's last S has completed
+      // (its Q and K ring may then receive the partials of the merge)
+      const uint16_t smask = (uint16_t)((1u << p.splits) - 1u);
       unsigned long long t_last = globaltimer();
       while (ok && i < n) {
         bool progress = false;
@@ -407,6 +415,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
             if (p.mc > 1) umma_commit_mc(&k_empty[s], mmask);   // K of this stage is free once S is done
             else umma_commit(&k_empty[s]);
             ++ns;
+            if (p.xch == 2 && ns == n) {
+              umma_commit_mc(sdone, smask);
+              sdone_sent = true;
+            }
             progress = true;
           }
         }
@@ -432,12 +444,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           ok = false;
         }
       }
+      // (no chunk, or an abort: arrive all the same, once earlier MMAs are done)
+      if (p.xch == 2 && !sdone_sent) umma_commit_mc(sdone, smask);
       if (!ok) flags[0] = 1;
       flags[2] = ns;   // chunks whose K arrival was consumed
       flags[4] = i;    // chunks whose V^T arrival was consumed
     }
     __syncwarp();
-    if (p.xch) cluster_arrive_release();
+    if (p.xch == 1) cluster_arrive_release();
   } else {
     // softmax / epilogue: thread owns query row r (TMEM lane r)
     const int q4 = warp & 3;
@@ -536,12 +550,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       tc_fence_after();
     }
     if (!ok && lane == 0) flags[0] = 1;
-    if (p.xch) {
+    if (p.xch == 1) {
       // past this barrier every split of the cluster has finished its MMAs
       // (its Q and rings may be overwritten) and armed its receive barrier;
       // every thread arrives exactly once, whatever happened before
       cluster_arrive_release();
       cluster_wait_acquire();
+    } else if (p.xch == 2) {
+      // every split's S MMAs are done: their Q and K rings, where the
+      // partials land, are no longer read
+      const bool okd = __all_sync(0xffffffffu, mbar_wait_cluster(sdone, 0));
+      if (!okd && lane == 0) flags[0] = 1;
     }
     if (p.splits == 1) {
       // O / l as bf16: this thread stages its row in the rings (every chunk
@@ -870,6 +889,10 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   p.v_slots = sv;
   const size_t smem = fixed + rings;
   if (p.xch && (size_t)AT_BM * p.hdp * 2 + (size_t)splits * AT_BM * 8 > (size_t)p.nblk * AT_QBLK + rings) p.xch = 0;
+  // the receive area within Q and the K ring (free once S is done): send
+  // without waiting for the other splits' PV
+  if (p.xch && (size_t)AT_BM * p.hdp * 2 + (size_t)splits * AT_BM * 8 <= (size_t)p.nblk * AT_QBLK + (size_t)sk * k_bytes)
+    p.xch = 2;
 
   AtMaps m;
   const int hd = a.hd, rpr = a.H + a.F;
