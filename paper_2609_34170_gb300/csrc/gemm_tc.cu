@@ -19,7 +19,8 @@
 // Work distribution:
 //  * no split: CTAs walk the tiles (persistent when there are more tiles than
 //    SMs) with two TMEM accumulators, so the epilogue of one tile overlaps the
-//    MMAs of the next;
+//    MMAs of the next; where the tiles are many, pairs of CTAs run 256-row
+//    tiles with the two-SM MMA instead (tc_gemm_pair_kernel, below);
 //  * few tiles: the K dimension is split over grid.z.  The splits of a tile
 //    form a thread-block cluster and rank q sums a token slice over the splits
 //    in order (deterministic) and applies the epilogue.  The partials travel
