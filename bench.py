@@ -213,6 +213,24 @@ def run_reference(args, cfg, rank):
     print(json.dumps(line), flush=True)
 
 
+def max_over_ranks(x: float, world: int, device="cuda") -> float:
+    """The largest of the ranks' values of x (a job of replicas is as slow as
+    its slowest rank); x itself on a single rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, batch: int, steps: int, seconds: float) -> float:
+    """Robot-steps per second of all ranks together: each of the `world`
+    ranks advances its own `batch` robots by `steps` steps in `seconds`."""
+    return world * batch * steps / seconds
+
+
 METRIC = "rolling-step throughput (robot-steps/s); p50/p99 step latency reported alongside"
 UNIT = "robot-steps/s"
 
@@ -396,12 +414,9 @@ def main():
         dist.barrier()
     total_ms = t_all0.elapsed_time(t_all1)
     lat = np.array([a.elapsed_time(b) for a, b in ev])
-    if world > 1:
-        tt = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(total_ms, world)
     ms_per_step = total_ms / args.steps
-    value = world * B * args.steps / (total_ms / 1e3)
+    value = whole_job_rate(world, B, args.steps, total_ms / 1e3)
 
     # ---- e2e: through the C ABI with host buffers, H2D of the step inputs and D2H of the released action
     z_h = z.cpu().pin_memory()
@@ -422,7 +437,7 @@ def main():
         ravel_roll_step(sess.handle, sess.buffer, t_d, z_dev if cfg.fop_tokens else None, delta, released, None, st)
         rel_h.copy_(released, non_blocking=True)
         st.synchronize()
-    e2e_s = (time.perf_counter() - t0) / n_e2e
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / n_e2e, world)
     h2d = z_h.numel() * z_h.element_size() + B * 4
     d2h = B * cfg.action_dim * 4
 
@@ -466,7 +481,8 @@ def main():
                      "launches_per_step": nlaunch, "avg_launch_us": avg_ms * 1e3,
                      "share_of_step": tot[dom] / grand, "peak_source": f"{peak_src} (MEASURED_PEAKS.json)"},
         "kernel_shares": {k: round(v / grand, 4) for k, v in sorted(tot.items(), key=lambda x: -x[1])},
-        "e2e": {"value": world * B / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "e2e": {"value": whole_job_rate(world, B, 1, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
         "gpu_launches": kernels_per_step * args.steps + (args.steps // args.swap_every if args.swap_every else 0),
         "clocks": clk,
     }
