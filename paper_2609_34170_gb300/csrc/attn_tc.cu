@@ -17,12 +17,14 @@
 // normalisation, so this is not an approximation).
 // At batch 1 a (b, g) pair has only a few query tiles, so the key chunks are
 // split over grid.z; the splits of a query tile form a thread-block cluster
-// and rank q merges head-dim slice q of every split's partial.  Once every
-// split's MMAs are done (one cluster barrier), each split sends its rows'
-// (m, l) and its output normalised by its own l, in bf16 (the precision of
-// every activation between kernels of the bf16 path), by st.async straight
-// into the owning rank's shared memory (overlaid on Q and the K/V rings);
-// an mbarrier there counts the bytes.  Where that does not apply, the splits
+// and rank q merges head-dim slice q of every split's partial.  Each split
+// sends its rows' (m, l) and its output normalised by its own l, in bf16 (the
+// precision of every activation between kernels of the bf16 path), by
+// st.async straight into the owning rank's shared memory, overlaid on Q and
+// the K ring, as soon as its own PV is done and every split's last S MMA has
+// completed (a multicast tcgen05.commit on each split's "S done" barrier; a
+// cluster barrier after all MMAs where the area reaches the V ring); an
+// mbarrier at the owner counts the bytes.  Where that does not apply, the splits
 // publish unnormalised fp32 partials through L2 and the cluster barrier.  The
 // producer keeps the L2 warm a few prefix chunks ahead of its loads.
 //
