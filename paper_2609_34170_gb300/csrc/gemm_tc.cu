@@ -1166,13 +1166,12 @@ cudaError_t encode_out(CUtensorMap* m, void* base, int rows, int cols, int ld, b
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-// Token-tile width: the smallest of 32/64/96/128 that holds M; beyond 128
-// tokens, the multiple of 16 in [128, 256] whose tile count fills whole waves
-// of the SMs best (per-CTA work ~ waves x BN), larger BN on ties.
+// Token-tile width: up to 128 tokens, the smallest of 32, 48, .., 128 (the
+// MMA's N steps by 16) that holds M; beyond 128 tokens, the multiple of 16 in
+// [128, 256] whose tile count fills whole waves of the SMs best (per-CTA work
+// ~ waves x BN), larger BN on ties.
 int pick_bn(int M, int tiles_n, int num_sms) {
-  const int cands[] = {32, 64, 96, 128};
-  for (int c : cands)
-    if (M <= c) return c;
+  if (M <= 128) return std::max(32, (M + 15) / 16 * 16);
   int best = 256;
   long best_cost = -1;
   for (int bn = 256; bn >= 128; bn -= 16) {
