@@ -57,7 +57,6 @@ struct AtParams {
   int Pmax, n_pre, n_kv, splits;
   int layer, Bmax, mask_mode;
   int nblk, k_slots, v_slots;         // head-dim blocks of 64; K and V^T ring depths
-  int mc;                             // query tiles of a (b, g) pair sharing each K/V chunk by multicast (1 = none)
   int xch;                            // splits > 1: partials through L2 (0) or shared memory, sent once every
                                       // split's MMAs are done (1: cluster barrier) or once every split's S
                                       // MMAs are done (2: the receive area lies in Q and the K ring)
@@ -73,7 +72,6 @@ struct AtParams {
 
 struct AtMaps {
   CUtensorMap q, k, vt, pk0, pk1, pv0, pv1;
-  CUtensorMap vts, pvs0, pvs1;   // V^T boxes of hd/mc rows (multicast slices)
 };
 
 // The idx-th chunk this CTA processes (prefix chunks past the valid prefix
@@ -242,11 +240,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     mbar_init(q_full, 1);
     for (int s = 0; s < SK; ++s) {
       mbar_init(&k_full[s], 1);
-      mbar_init(&k_empty[s], p.mc);   // released by the S commit of every CTA sharing the chunk
+      mbar_init(&k_empty[s], 1);   // released by the S commit
     }
     for (int s = 0; s < SV; ++s) {
       mbar_init(&v_full[s], 1);
-      mbar_init(&v_empty[s], p.mc);   // released by the PV commit of every CTA sharing the chunk
+      mbar_init(&v_empty[s], 1);   // released by the PV commit
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
@@ -261,27 +259,20 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     if (p.xch) mbar_expect_tx(rcv_bar, (uint32_t)(p.splits * vrows * (2 * cps + 8)));
   }
-  // with multicast (or xch 2), every CTA's barriers must exist before a peer targets them
-  if (p.mc > 1 || p.xch == 2) cluster_sync();
-  const int mrank = (p.mc > 1) ? (int)cluster_ctarank() : 0;
-  const uint16_t mmask = (uint16_t)((1u << p.mc) - 1u);
+  // (xch 2) every split's barriers must exist before a peer targets them
+  if (p.xch == 2) cluster_sync();
   const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
   const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
-  const CUtensorMap* pvs = slot ? &maps.pvs1 : &maps.pvs0;
-  // K and V^T of chunk c into stage s: all of it, or (multicast) this CTA's
-  // share -- head-dim blocks rank, rank+mc, .. of K and V^T rows
-  // [rank*hd/mc, (rank+1)*hd/mc) -- sent to every CTA of the cluster
+  // K and V^T of chunk c into stage s, each CTA loading its own copy (query
+  // tiles of one (b, g) pair read the same chunk, which L2 serves to all)
   auto load_k = [&](int c, int s, uint64_t pol) {
     uint8_t* ks = kv_s + (size_t)s * k_bytes;
-    mbar_expect_tx(&k_full[s], k_bytes);   // the whole chunk, whoever sends it
+    mbar_expect_tx(&k_full[s], k_bytes);
     const bool pre = c < p.n_pre;
     const int cc = c - p.n_pre;
     const CUtensorMap* km = pre ? pk : &maps.k;
     const int ky = pre ? c * AT_BKV : g, kz = pre ? ctx_z : b * rows_per_robot + cc * AT_BKV;
-    for (int blk = (p.mc == 1 ? 0 : mrank); blk < p.nblk; blk += p.mc) {
-      if (p.mc == 1) tma_load_3d(km, &k_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, pol);
-      else tma_load_3d_mc(km, &k_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, mmask, pol);
-    }
+    for (int blk = 0; blk < p.nblk; ++blk) tma_load_3d(km, &k_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, pol);
   };
   auto load_v = [&](int c, int s, uint64_t pol) {
     uint8_t* vs = v_ring + (size_t)s * p.vt_bytes;
@@ -289,13 +280,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     const bool pre = c < p.n_pre;
     const int cc = c - p.n_pre;
     const int vx = (pre ? c : cc) * AT_BKV, vz = pre ? ctx_z : b * p.Hkv + g;
-    if (p.mc == 1) {
-      tma_load_3d(pre ? pv : &maps.vt, &v_full[s], vs, vx, 0, vz, pol);
-    } else {
-      const int rows = p.hd / p.mc;
-      tma_load_3d_mc(pre ? pvs : &maps.vts, &v_full[s], vs + (size_t)mrank * rows * 128, vx, mrank * rows, vz, mmask,
-                     pol);
-    }
+    tma_load_3d(pre ? pv : &maps.vt, &v_full[s], vs, vx, 0, vz, pol);
   };
   if (threadIdx.x == 0) {
     uint64_t pol_kv;
@@ -414,8 +399,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
                           (blk > 0 || k > 0) ? 1u : 0u);
             }
             umma_commit(&s_full[ns & 1]);
-            if (p.mc > 1) umma_commit_mc(&k_empty[s], mmask);   // K of this stage is free once S is done
-            else umma_commit(&k_empty[s]);
+            umma_commit(&k_empty[s]);   // K of this stage is free once S is done
             ++ns;
             if (p.xch == 2 && ns == n) {
               umma_commit_mc(sdone, smask);
@@ -434,8 +418,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
 #pragma unroll
           for (int k = 0; k < 4; ++k)
             umma_bf16_ts(tmem + o_col, pa + 8 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
-          if (p.mc > 1) umma_commit_mc(&v_empty[s], mmask);
-          else umma_commit(&v_empty[s]);
+          umma_commit(&v_empty[s]);
           umma_commit(&pv_done[i & 1]);
           ++i;
           progress = true;
@@ -763,8 +746,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols) : "memory");
   }
-  // no CTA leaves while a peer may still multicast into it or arrive on its barriers
-  if (p.mc > 1) cluster_sync();
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
@@ -863,16 +844,12 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
       splits *= 2;
   }
   p.splits = splits;
-  // query tiles of a (b, g) pair share K/V chunks by multicast (clusters along x)
-  p.mc = 1;
-  if (splits == 1 && (p.q_tiles == 2 || p.q_tiles == 4) && p.nblk % p.q_tiles == 0 && (a.hd / p.q_tiles) % 8 == 0)
-    p.mc = p.q_tiles;
   p.ws_o = a.ws;
   p.ws_ml = a.ws + (size_t)splits * nctas * AT_BM * p.hdp;
-  // partials through shared memory: whole 8-column bf16 groups per rank slice,
-  // no multicast cluster, and the receive area (O groups + (m, l) of every
-  // split) within Q + the rings (checked below)
-  p.xch = splits > 1 && p.mc == 1 && (p.hdp / splits) % 8 == 0 ? 1 : 0;
+  // partials through shared memory: whole 8-column bf16 groups per rank
+  // slice, and the receive area (O groups + (m, l) of every split) within
+  // Q + the rings (checked below)
+  p.xch = splits > 1 && (p.hdp / splits) % 8 == 0 ? 1 : 0;
   // K slots: as many whole K + V^T stages as fit (<= 4); V^T slots: the K
   // count plus what the remaining bytes hold (<= 2 more): K is free again as
   // soon as S = Q K^T is done, V^T only after P V, so V^T needs the depth
@@ -913,16 +890,9 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
       e = enc3(s ? &m.pv1 : &m.pv0, a.ctx_vt[s], a.Pmax, hd, zc, (uint64_t)a.pst * 2, (uint64_t)hd * a.pst * 2,
                AT_BKV, hd, 1);
   }
-  const uint32_t vrows = (uint32_t)(hd / p.mc);
-  if (e == cudaSuccess)
-    e = enc3(&m.vts, a.vt, rpr, hd, (uint64_t)a.B * a.Hkv, (uint64_t)a.kvp * 2, (uint64_t)hd * a.kvp * 2, AT_BKV,
-             vrows, 1);
-  for (int s = 0; s < 2 && e == cudaSuccess; ++s)
-    e = enc3(s ? &m.pvs1 : &m.pvs0, a.ctx_vt[s], a.Pmax, hd, zc, (uint64_t)a.pst * 2, (uint64_t)hd * a.pst * 2,
-             AT_BKV, vrows, 1);
   if (e != cudaSuccess) return e;
   dim3 grid(p.q_tiles, a.B * a.Hkv, splits);
-  e = launch_kernel_cluster(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, dim3(p.mc, 1, splits), m, p);
+  e = launch_kernel_cluster(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, dim3(1, 1, splits), m, p);
   if (a.n_launched) ++*a.n_launched;
   return e;
 }
