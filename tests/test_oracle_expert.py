@@ -313,3 +313,67 @@ def test_conditioning_with_permutation_weights_vs_torch_silu():
         want[m] = torch.nn.functional.silu(torch.tensor(moved + b1)).numpy() * s + b2
     cond = expert.conditioning(cfg, W, x["t"], x["d"])
     np.testing.assert_allclose(cond, want["d"][:, None, :] + want["t"][None, :, :], rtol=1e-12, atol=1e-13)
+
+
+# ----------------------------------------------------------------------------- the FOP branch (Eq. 4)
+# FOP tokens z enter every layer as extra keys / values: that layer's K / V
+# projection of RMSNorm(z) * (1 + gamma_l) (the FOP-as-keys reading of Eq. 4).
+# The two pins below fail on the plausible slips of that branch: a dropped
+# RMSNorm on z, gamma used in place of 1 + gamma, the action rows' modulation
+# applied to the FOP rows, the K columns used as values, or a wrong key count.
+
+
+def test_fop_tokens_enter_through_a_scale_free_norm():
+    # RMSNorm(c z) = RMSNorm(z) for c > 0 (eps negligible: |z| ~ 100), so the
+    # velocity must not change when the tokens are rescaled -- and it must
+    # change when they are replaced.
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    z = z.astype(np.float64) * 100.0
+    a = expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d)
+    for c in (0.1, 7.3):
+        b = expert.expert_velocity(cfg, W, buf, t, k, v, P, c * z, d)
+        # eps shifts RMSNorm(c z) by ~eps (1/c^2 - 1) / (2 mean(z^2)) ~ 5e-9
+        np.testing.assert_allclose(b, a, rtol=1e-6, atol=1e-10)
+    other = synth.make_fop(cfg, 999) * 100.0
+    assert np.max(np.abs(expert.expert_velocity(cfg, W, buf, t, k, v, P, other, d) - a)) > 1e-3
+
+
+def test_fop_values_closed_form_first_layer():
+    # W_q = 0 makes every score 0, so each head's first-layer attention output
+    # is the plain mean of the P prefix, F FOP and H action values of its KV
+    # head.  With W_gate = 0 the MLP adds nothing, with W_mod = 0 every row's
+    # modulation is the bias, and with in_w = 0 every action row is the bias
+    # in_b (large, so eps is negligible).  The values are written out here
+    # from the definitions: FOP  sqrt(D) z / |z| * (1 + gamma_0) @ W_v,
+    # action  (sqrt(D) x0 / |x0| * (1 + scale) + shift) @ W_v.
+    cfg = TINY.replace(layers=1)
+    D, Hq, Hkv, hd, H, F = cfg.width, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.slots, cfg.fop_tokens
+    G = Hq // Hkv
+    W, buf, t, k, v, _, z, d, _ = _inputs(cfg)
+    P = 6
+    z = z.astype(np.float64) * 100.0
+    W1 = dict(W)
+    wqkv = W["w_qkv"].astype(np.float64).copy()
+    wqkv[:, :, :(Hq + Hkv) * hd] = 0.0                 # Q and K columns
+    W1.update(w_qkv=wqkv, w_gate=np.zeros_like(W["w_gate"]), mod_w=np.zeros_like(W["mod_w"]),
+              in_w=np.zeros_like(W["in_w"]), in_b=W["in_b"].astype(np.float64) * 1000.0)
+    W1["fop_gamma"] = W["fop_gamma"].astype(np.float64) * 20.0   # far from 0, so gamma vs 1 + gamma differs
+    tr = {}
+    expert.expert_velocity(cfg, W1, buf, t, k, v, P, z, d, trace=tr)
+    wv = wqkv[0][:, (Hq + Hkv) * hd:]                  # [D, Hkv hd]
+    x0 = W1["in_b"]
+    sc, sh = W["mod_b"][:D].astype(np.float64), W["mod_b"][D:2 * D].astype(np.float64)
+    ya = np.sqrt(D) * x0 / np.linalg.norm(x0) * (1.0 + sc) + sh
+    va = ya @ wv                                        # the same for every slot
+    o = np.zeros((cfg.batch, Hq * hd))
+    for b in range(cfg.batch):
+        yf = np.sqrt(D) * z[b] / np.linalg.norm(z[b], axis=1, keepdims=True) * (1.0 + W1["fop_gamma"][0])
+        vf = yf @ wv                                    # [F, Hkv hd]
+        for h in range(Hq):
+            g = h // G
+            tot = v[0, b, g, :P].astype(np.float64).sum(0) + vf[:, g * hd:(g + 1) * hd].sum(0) \
+                + H * va[g * hd:(g + 1) * hd]
+            o[b, h * hd:(h + 1) * hd] = tot / (P + F + H)
+    want = x0[None, None, :] + (o @ W["w_o"][0].astype(np.float64))[:, None, :]
+    np.testing.assert_allclose(tr["x"][0], np.broadcast_to(want, tr["x"][0].shape), rtol=1e-9, atol=1e-9)
