@@ -120,7 +120,9 @@ void ravel_destroy(ravel_t* r);
  * App. A.1): robot b's noise seed is seeds[b] (host, [batch]); slot j of
  * buffer (device, float32 [batch, H, A], written) receives the Gaussian action
  * of index j, and the robot's next appended action gets index H.  Enqueued on
- * `stream`.  A new batch size invalidates the current context (set it again). */
+ * `stream`.  A new batch size invalidates the current context (set it again).
+ * Also clears the handle's device error word (after synchronising the
+ * device). */
 ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* buffer, void* stream);
 
 /* Install a new VLM context (Eq. 2): k and v are device arrays
@@ -183,7 +185,9 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
  *          that of its W row
  *   out device [M, ldo], out_dtype RAVEL_FP32 or RAVEL_BF16; bias device [N] or NULL
  * Enqueued on `stream`; uses the handle's split-K workspace, so it must not
- * overlap another call on the same handle. */
+ * overlap another call on the same handle.  Like ravel_roll_step it first
+ * reports a device error raised by earlier work (RAVEL_EDEVICE /
+ * RAVEL_ETIMEOUT) and mirrors the error word after its own launch. */
 ravel_status ravel_gemm(ravel_t* r, const void* X, int M, int K, int lda, const void* W, int N, int ldw, int epi,
                         void* out, int ldo, int out_dtype, const float* bias, void* stream);
 
@@ -202,14 +206,45 @@ ravel_status ravel_gemm(ravel_t* r, const void* X, int M, int K, int lda, const 
  * above RAVEL_NOALLOC_MAX_M / _N / _K return RAVEL_ESHAPE; bad pointers or
  * modes RAVEL_EINVAL.  The first call on a device resolves the array's device
  * address (and the kernel set-up) for that device; make that first call
- * before any stream capture.  Each call clears the scratch's counters on
- * `stream` before the GEMM; every call shares the array, so calls that
- * overlap on the GPU race and must be serialised by the caller. */
+ * before any stream capture (a first call on a capturing stream returns
+ * RAVEL_EINVAL and does nothing).  Each call clears the scratch's tile
+ * counters on `stream` before the GEMM; every call shares the array, so calls
+ * that overlap on the GPU race and must be serialised by the caller.  The
+ * array also holds a device error word that calls never clear: a bounded wait
+ * that runs out inside the GEMM (its output is then not valid) stays recorded
+ * until ravel_gemm_noalloc_status reads it. */
 #define RAVEL_NOALLOC_MAX_M 32768
 #define RAVEL_NOALLOC_MAX_N 262144
 #define RAVEL_NOALLOC_MAX_K 65536
 ravel_status ravel_gemm_noalloc(const void* X, int M, int K, int lda, const void* W, int N, int ldw, int epi,
                                 void* out, int ldo, int out_dtype, const float* bias, void* stream);
+
+/* Error state of ravel_gemm_noalloc on the current device (allocates
+ * nothing): waits for `stream`, then reads and clears the device error word of
+ * the allocation-free entry point.  RAVEL_OK if no call has run into an error
+ * since the last read (or none has run), RAVEL_ETIMEOUT if a bounded wait in
+ * one of its GEMMs ran out (that call's output is not valid), RAVEL_EDEVICE for
+ * any other kernel error, RAVEL_EINVAL on a capturing stream. */
+ravel_status ravel_gemm_noalloc_status(void* stream);
+
+/* Fault injection for tests of the failure-detection paths.  No GPU fault is
+ * raised and every wait involved is bounded:
+ *   RAVEL_FAULT_PREFIX_LEN: enqueue on `stream` a write of an out-of-range
+ *     prefix length into the handle's device context state (r required; count
+ *     unused).  The attention kernels of the next step refuse it, compute
+ *     nothing and raise the device error word, and a later call on the handle
+ *     returns RAVEL_EDEVICE.  The next ravel_set_context installs a valid
+ *     state again and ravel_reset clears the error word.
+ *   RAVEL_FAULT_WITHHOLD_ARRIVAL: the next `count` tensor-core GEMM launches
+ *     that run without a thread-block cluster (for example ravel_gemm or
+ *     ravel_gemm_noalloc with K <= 64) wait for an mbarrier arrival that
+ *     nobody makes; each gives up after 2 ms, drains its copies, raises
+ *     ERR_TIMEOUT and exits.  A later call on the handle returns
+ *     RAVEL_ETIMEOUT (ravel_gemm_noalloc_status for the allocation-free
+ *     entry point).  r may be NULL.
+ * The paper has no counterpart; this serves the library's own tests. */
+enum { RAVEL_FAULT_PREFIX_LEN = 1, RAVEL_FAULT_WITHHOLD_ARRIVAL = 2 };
+ravel_status ravel_debug_inject(ravel_t* r, int fault, int count, void* stream);
 
 /* Name of a kernel kind id of ravel_profile_step ("gemm_down", ...). */
 const char* ravel_kernel_kind_name(int kind);

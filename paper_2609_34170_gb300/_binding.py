@@ -15,6 +15,7 @@ from . import build as _build
 
 RAVEL_FP32, RAVEL_BF16 = 0, 1
 RAVEL_MASK_FULL, RAVEL_MASK_SLOT_ISOLATED = 0, 1
+RAVEL_FAULT_PREFIX_LEN, RAVEL_FAULT_WITHHOLD_ARRIVAL = 1, 2
 
 STATUS = ["RAVEL_OK", "RAVEL_EINVAL", "RAVEL_ESHAPE", "RAVEL_ENOMEM", "RAVEL_ECUDA", "RAVEL_ENOCONTEXT",
           "RAVEL_EBUSY", "RAVEL_EDEVICE", "RAVEL_ETIMEOUT", "RAVEL_ENOTREADY"]
@@ -71,6 +72,8 @@ def load(path: str | None = None):
         "ravel_kernel_kind_name": (C.c_char_p, [i]),
         "ravel_gemm": (i, [vp, vp, i, i, i, vp, i, i, i, vp, i, i, vp, vp]),
         "ravel_gemm_noalloc": (i, [vp, i, i, i, vp, i, i, i, vp, i, i, vp, vp]),
+        "ravel_gemm_noalloc_status": (i, [vp]),
+        "ravel_debug_inject": (i, [vp, i, i, vp]),
         "ravel_status_string": (C.c_char_p, [i]),
         "ravel_last_error": (C.c_char_p, [vp]),
     }
@@ -202,6 +205,17 @@ def ravel_gemm_noalloc(X, W, epi: int, out, bias=None, K: int | None = None, str
                                            N, ldw, epi, _dptr(out, name="out"), out.shape[1], od,
                                            _dptr(bias, torch.float32, "bias"), _stream_ptr(stream)),
            "ravel_gemm_noalloc")
+
+
+def ravel_gemm_noalloc_status(stream=None) -> int:
+    """Status of the allocation-free GEMM's device error word (read and
+    cleared); returned as the raw ravel_status value."""
+    return int(load().ravel_gemm_noalloc_status(_stream_ptr(stream)))
+
+
+def ravel_debug_inject(h, fault: int, count: int = 1, stream=None):
+    """Fault injection of the failure-path tests (see ravel.h)."""
+    _check(h, load().ravel_debug_inject(h, fault, count, _stream_ptr(stream)), "ravel_debug_inject")
 
 
 def ravel_get_state(h, batch: int) -> np.ndarray:

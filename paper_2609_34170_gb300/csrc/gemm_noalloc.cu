@@ -14,7 +14,9 @@
 // holds it until the process exits.  All calls share it, so calls that
 // overlap on the GPU (different streams, or different host threads) race on
 // it and must be serialised by the caller.  It keeps the last call's
-// contents; each call clears the part that must start at zero.
+// contents; each call clears the part that must start at zero (the tile
+// counters).  Its error word is sticky: a bounded wait that runs out inside a
+// GEMM sets it, and it stays set until ravel_gemm_noalloc_status reads it.
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -27,8 +29,8 @@ namespace {
 
 constexpr size_t kPartialBytes = (size_t)8 << 20;   // split-K partial tiles (fp32)
 constexpr int kCounters = 1024;                      // per-tile arrival counters
-constexpr size_t kZeroBytes = (kCounters + 64) * sizeof(int);   // counters + error word, cleared per call
-constexpr size_t kScratchBytes = kPartialBytes + kZeroBytes;
+constexpr size_t kCounterBytes = kCounters * sizeof(int);       // cleared by every call
+constexpr size_t kScratchBytes = kPartialBytes + kCounterBytes + 64 * sizeof(int);   // + the error word
 constexpr int kMaxDevices = 64;
 
 // The scratch: [partials | counters | error word].  In host code the name is
@@ -47,24 +49,28 @@ std::mutex g_mutex;
 
 // Once per device, with that device current: resolve the array's device
 // address, the SM count and the tensor-map encoder, and raise the kernel's
-// shared-memory limit.  Nothing here allocates.
-cudaError_t setup_device(int dev, DeviceState** out) {
+// shared-memory limit.  Nothing here allocates.  None of it may run while `st`
+// is being captured into a graph (it would invalidate the capture): a first
+// call under capture is refused.
+ravel_status setup_device(int dev, cudaStream_t st, DeviceState** out) {
   std::lock_guard<std::mutex> lock(g_mutex);
   DeviceState& s = g_state[dev];
   if (!s.ready) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return RAVEL_ECUDA;
+    if (cs != cudaStreamCaptureStatusNone) return RAVEL_EINVAL;
     unsigned char* ptr = nullptr;
-    cudaError_t e = cudaGetSymbolAddress((void**)&ptr, g_scratch);
-    if (e != cudaSuccess) return e;
-    e = cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    e = init_tc_gemm();
-    if (e != cudaSuccess) return e;
+    if (cudaGetSymbolAddress((void**)&ptr, g_scratch) != cudaSuccess) return RAVEL_ECUDA;
+    if (cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return RAVEL_ECUDA;
+    if (init_tc_gemm() != cudaSuccess) return RAVEL_ECUDA;
     s.scratch = ptr;
     s.ready = true;
   }
   *out = &s;
-  return cudaSuccess;
+  return RAVEL_OK;
 }
+
+int* error_word(const DeviceState* s) { return (int*)(s->scratch + kPartialBytes + kCounterBytes); }
 
 }  // namespace
 }  // namespace ravel
@@ -86,14 +92,36 @@ extern "C" ravel_status ravel_gemm_noalloc(const void* X, int M, int K, int lda,
   if (M == 0) return RAVEL_OK;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RAVEL_ECUDA;
-  DeviceState* s = nullptr;
-  if (setup_device(dev, &s) != cudaSuccess) return RAVEL_ECUDA;
   cudaStream_t st = (cudaStream_t)stream;
-  unsigned char* zero = s->scratch + kPartialBytes;
-  if (cudaMemsetAsync(zero, 0, kZeroBytes, st) != cudaSuccess) return RAVEL_ECUDA;
+  DeviceState* s = nullptr;
+  const ravel_status rs = setup_device(dev, st, &s);
+  if (rs != RAVEL_OK) return rs;
+  int* counters = (int*)(s->scratch + kPartialBytes);
+  if (cudaMemsetAsync(counters, 0, kCounterBytes, st) != cudaSuccess) return RAVEL_ECUDA;
   // The split plan is chosen so that the partials fit the array (fewer
   // splits, or none, when they would not).
-  TcWorkspace ws{(float*)s->scratch, kPartialBytes, (int*)zero, kCounters, (int*)zero + kCounters};
+  TcWorkspace ws{(float*)s->scratch, kPartialBytes, counters, kCounters, error_word(s)};
   if (launch_gemm_tc(g, ws, s->num_sms, st, /*cluster=*/false) != cudaSuccess) return RAVEL_ECUDA;
   return RAVEL_OK;
+}
+
+extern "C" ravel_status ravel_gemm_noalloc_status(void* stream) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RAVEL_ECUDA;
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return RAVEL_ECUDA;
+  if (cs != cudaStreamCaptureStatusNone) return RAVEL_EINVAL;
+  const DeviceState* s = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_mutex);
+    if (!g_state[dev].ready) return RAVEL_OK;   // no call has run on this device
+    s = &g_state[dev];
+  }
+  if (cudaStreamSynchronize(st) != cudaSuccess) return RAVEL_ECUDA;
+  int bits = 0;   // a synchronous copy into host memory: no staging buffer of ours
+  if (cudaMemcpy(&bits, error_word(s), sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return RAVEL_ECUDA;
+  if (!bits) return RAVEL_OK;
+  if (cudaMemset(error_word(s), 0, sizeof(int)) != cudaSuccess) return RAVEL_ECUDA;
+  return (bits & ERR_TIMEOUT) ? RAVEL_ETIMEOUT : RAVEL_EDEVICE;
 }

@@ -38,6 +38,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstring>
 #include <vector>
 
@@ -102,6 +103,9 @@ struct TcParams {
                         // has finished its MMAs), else on the output boxes + exchange (used only
                         // after the sum)
   uint32_t bar_off;     // mbarriers, TMEM slot, flags
+  unsigned long long wait_ns;   // limit of every bounded wait (ERR_TIMEOUT after it)
+  int withhold;         // fault injection (tests): the MMA thread first waits for an arrival that
+                        // nobody makes, so the launch gives up after wait_ns and unwinds
 };
 
 // The TMA epilogue kind of a launch (EK_F32 .. EK_GEGLU).
@@ -489,7 +493,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 128);
     }
-    if constexpr (RED == RED_DSMEM) mbar_init(rcv_bar, 1);
+    mbar_init(rcv_bar, 1);   // RED_DSMEM: the partials' arrival; otherwise armed by nobody
     flags[0] = flags[1] = flags[2] = flags[3] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // the slices of all splits (this one's included): 128 rows x cpr tokens each
@@ -550,7 +554,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
             tma_load_2d(&tmX, &full[s], b_s + (size_t)s * b_bytes, kb * TC_BK, tm * BN, pol_x);
             continue;
           }
-          if (!mbar_wait(&empty[s], ((uint32_t)(it / S) & 1u) ^ 1u)) {
+          if (!mbar_wait(&empty[s], ((uint32_t)(it / S) & 1u) ^ 1u, p.wait_ns)) {
             flags[0] = 1;
             ok = false;
             break;
@@ -572,8 +576,14 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       int it = 0;
       bool ok = true;
       int tn, tm, sp;
-      if (p.oneshot) {   // one item, every k-tile behind one barrier
-        ok = mbar_wait(&full[0], 0);
+      // fault injection: an arrival that never comes (rcv_bar is armed by
+      // nobody outside RED_DSMEM, which the host never combines with this)
+      if (p.withhold && !mbar_wait(rcv_bar, 0, p.wait_ns)) {
+        flags[0] = 1;
+        ok = false;
+      }
+      if (ok && p.oneshot) {   // one item, every k-tile behind one barrier
+        ok = mbar_wait(&full[0], 0, p.wait_ns);
         if (ok) {
           tc_fence_after();
           for (int kb = 0; kb < kb1_first - kb0_first; ++kb) {
@@ -592,7 +602,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       for (int i = 0; !p.oneshot && ok && work_item(p, i, tn, tm, sp); ++i) {
         const int b = i & 1;
         // the accumulator of item i - 2 must have been drained by the epilogue
-        if (i >= 2 && !mbar_wait(&acc_empty[b], (uint32_t)((i >> 1) - 1) & 1u)) {
+        if (i >= 2 && !mbar_wait(&acc_empty[b], (uint32_t)((i >> 1) - 1) & 1u, p.wait_ns)) {
           flags[0] = 1;
           break;
         }
@@ -601,7 +611,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         const int kb0 = (int)((long)sp * p.num_kb / p.splits), kb1 = (int)((long)(sp + 1) * p.num_kb / p.splits);
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % S;
-          if (!mbar_wait(&full[s], (uint32_t)(it / S) & 1u)) {
+          if (!mbar_wait(&full[s], (uint32_t)(it / S) & 1u, p.wait_ns)) {
             flags[0] = 1;
             ok = false;
             break;
@@ -628,7 +638,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     int tn, tm, sp;
     for (int i = 0; work_item(p, i, tn, tm, sp); ++i) {
       const int b = i & 1;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[b], (uint32_t)(i >> 1) & 1u));
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[b], (uint32_t)(i >> 1) & 1u, p.wait_ns));
       if constexpr (RED == RED_DSMEM) {
         // past this barrier every CTA of the cluster has finished its MMAs
         // (its operand ring may be overwritten) and armed its receive barrier;
@@ -781,7 +791,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     // writes over what was just read.)
     if (warp >= 2) {
       const int r = (warp & 3) * 32 + lane;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait_cluster(rcv_bar, 0));
+      const bool ok = __all_sync(0xffffffffu, mbar_wait_cluster(rcv_bar, 0, p.wait_ns));
       if (!ok) {
         if (lane == 0) raise_error(p.err, ERR_TIMEOUT);
       } else {
@@ -1187,6 +1197,8 @@ int pick_bn(int M, int tiles_n, int num_sms) {
 }
 
 int g_max_cluster = 8;   // largest power-of-two cluster the split-K reduction may use
+std::atomic<int> g_withhold{0};   // launches left to run with a withheld arrival (fault injection)
+constexpr unsigned long long kWithholdWaitNs = 2000000ull;   // their wait limit: 2 ms
 bool g_pair_gemm = true;  // persistent launches of many tiles on SM pairs
 int g_pair_bn_max = 256;  // widest token tile of a pair launch
 
@@ -1247,13 +1259,15 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
   TcParams p{g.M, g.N, g.K, bn, stages, 1, num_kb, RED_NONE, (uint32_t)ring, acc_cols, tiles_n, tiles_m, num_tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, 1, 0, box_m, box_bytes, stg_off, xch_off,
-             vts_off, 0, bar_off};
+             vts_off, 0, bar_off, kTcTimeoutNs, 0};
   const int npairs = std::min(num_tiles, slots);
   return launch_kernel_cluster(tc_pair_kernel(ek), dim3(2 * npairs), dim3(TC_THREADS), smem, st, dim3(2, 1, 1), mw, mx,
                                mo, p);
 }
 
 }  // namespace
+
+void debug_withhold_gemm(int launches) { g_withhold.store(launches > 0 ? launches : 0); }
 
 cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
@@ -1400,7 +1414,13 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
-             vts_off, rcv_off, bar_off};
+             vts_off, rcv_off, bar_off, kTcTimeoutNs, 0};
+  // fault injection (tests): a launch without a cluster may be told to wait
+  // for an arrival that never comes, with a short limit
+  if ((reduce == RED_NONE || reduce == RED_WORKSPACE) && g_withhold.load() > 0 && g_withhold.fetch_sub(1) > 0) {
+    p.withhold = 1;
+    p.wait_ns = kWithholdWaitNs;
+  }
   const dim3 grid = splits > 1 ? dim3(tiles_n, tiles_m, splits) : dim3(grid_ctas);
   const dim3 block(TC_THREADS);
   // persistent launches: one instantiation per epilogue kind; split-K

@@ -68,6 +68,11 @@ bool tc_gemm_supported(const GemmArgs& g);
 // workspace `ws` with a last-arriving-CTA fix-up.
 cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms, cudaStream_t st,
                            bool cluster = true);
+// Fault injection for tests: the next `launches` tensor-core GEMM launches
+// that run without a thread-block cluster make their MMA thread wait for an
+// mbarrier arrival that nobody makes, with a 2 ms limit; each gives up,
+// drains its copies, raises ERR_TIMEOUT and exits (no fault, no hang).
+void debug_withhold_gemm(int launches);
 
 // ---- adaRMSNorm rows ---------------------------------------------------------
 // Action rows r < B*H (b = r / H, j = r % H):

@@ -131,8 +131,12 @@ ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* bu
   if (batch < 1 || batch > r->plan.cfg.max_batch) return fail(r, RAVEL_ESHAPE, "reset: batch outside [1, max_batch]");
   RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
   cudaStream_t st = (cudaStream_t)stream;
-  // seeds go through a synchronous copy: the host array may be freed on return
-  RV_CUDA(r, cudaStreamSynchronize(st), "reset: sync");
+  // seeds go through a synchronous copy: the host array may be freed on
+  // return; every earlier step has finished, so the error word and its mirror
+  // can be cleared
+  RV_CUDA(r, cudaDeviceSynchronize(), "reset: sync");
+  RV_CUDA(r, cudaMemset(r->plan.err, 0, sizeof(int)), "reset: clear error word");
+  *r->err_host = 0;
   RV_CUDA(r, cudaMemcpy(r->plan.seeds, seeds, sizeof(uint64_t) * batch, cudaMemcpyHostToDevice), "reset: seeds");
   RV_CUDA(r, launch_reset(buffer, r->plan.seeds, r->plan.counters, batch, r->plan.cfg.slots,
                           r->plan.cfg.action_dim, st),
@@ -260,9 +264,28 @@ ravel_status ravel_gemm(ravel_t* r, const void* X, int M, int K, int lda, const 
   if (epi != EPI_GEGLU && ldo < N) return fail(r, RAVEL_EINVAL, "gemm: ldo < N");
   if (epi == EPI_ADD_F32 && out_dtype != 0) return fail(r, RAVEL_EINVAL, "gemm: accumulate needs a float32 output");
   if (M == 0) return RAVEL_OK;
+  ravel_status s = check_device_errors(r);
+  if (s != RAVEL_OK) return s;
   RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
   GemmArgs g{X, lda, W, ldw, M, N, K, (Epi)epi, out, ldo, out_dtype ? DT_BF16 : DT_F32, bias};
-  RV_CUDA(r, run_gemm(r->plan, g, (cudaStream_t)stream), "gemm");
+  cudaStream_t st = (cudaStream_t)stream;
+  RV_CUDA(r, run_gemm(r->plan, g, st), "gemm");
+  RV_CUDA(r, cudaMemcpyAsync(r->err_host, r->plan.err, sizeof(int), cudaMemcpyDeviceToHost, st), "error mirror");
+  return RAVEL_OK;
+}
+
+ravel_status ravel_debug_inject(ravel_t* r, int fault, int count, void* stream) {
+  if (fault == RAVEL_FAULT_WITHHOLD_ARRIVAL) {
+    debug_withhold_gemm(count);
+    return RAVEL_OK;
+  }
+  if (fault != RAVEL_FAULT_PREFIX_LEN) return fail(r, RAVEL_EINVAL, "debug_inject: unknown fault");
+  if (!r) return RAVEL_EINVAL;
+  if (!r->have_ctx) return fail(r, RAVEL_ENOCONTEXT, "debug_inject: no context set");
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  // the device state {active slot, prefix length}: a length past max_prefix
+  RV_CUDA(r, launch_flip(r->plan.ctx_state, r->active_host, r->plan.cfg.max_prefix + 1000, (cudaStream_t)stream),
+          "debug_inject: state write");
   return RAVEL_OK;
 }
 

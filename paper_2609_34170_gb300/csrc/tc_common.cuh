@@ -67,21 +67,22 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t pa
   return ok != 0;
 }
 
-__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity,
+                                                  unsigned long long limit_ns = kTcTimeoutNs) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
   while (!mbar_try_wait_cluster(bar, parity)) {
-    if (globaltimer() - t0 > kTcTimeoutNs) return false;
+    if (globaltimer() - t0 > limit_ns) return false;
   }
   return true;
 }
 
-// Wait for the phase of `parity` to complete; false after kTcTimeoutNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Wait for the phase of `parity` to complete; false after limit_ns.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned long long limit_ns = kTcTimeoutNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
   while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer() - t0 > kTcTimeoutNs) return false;
+    if (globaltimer() - t0 > limit_ns) return false;
   }
   return true;
 }
