@@ -208,6 +208,38 @@ def roll_step(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, 
     return released, new, counters, v
 
 
+def denoise_chunk(cfg, W, seeds, counters, n_steps: int, ctx_k, ctx_v, prefix_len, fop, delta,
+                  field=None, mask: str = "full"):
+    """The full-horizon (synchronous) denoising baseline the paper compares
+    rolling inference with (Experiments, synchronous simulation: ten
+    full-horizon denoising steps per policy query, Table 1): a fresh chunk of H
+    Gaussian actions -- robot b's actions of indices counters_b ..
+    counters_b + H - 1 -- starts at flow time t = 1 and all H slots take
+    ``n_steps`` Euler steps together, step n at t_n = 1 - n / n_steps (as
+    float32, the precision of the flow times the step takes) with
+    dt_n = t_n - t_{n+1}, t_{n_steps} = 0 (Eq. 3 with every slot at the same
+    time; the step is read off the time grid as in the rolling update), each
+    one expert pass at that single flow time.  The chunk ends at t = 0, where
+    every action is executable.
+
+    ``field(n, a, times) -> [B, H, A]`` replaces the expert (for closed-form
+    checks).  Returns (chunk [B, H, A] float64, counters + H)."""
+    H, A = cfg.slots, cfg.action_dim
+    counters = np.asarray(counters, dtype=np.uint64)
+    B = len(seeds)
+    a = np.stack([action_noise(int(seeds[b]), counters[b] + np.arange(H, dtype=np.uint64), A)
+                  for b in range(B)]).astype(np.float64) if B else np.zeros((0, H, A))
+    grid = np.array([1.0 - n / n_steps for n in range(n_steps)] + [0.0], dtype=np.float32).astype(np.float64)
+    for n in range(n_steps):
+        times = np.full(H, grid[n], dtype=np.float32)
+        if field is not None:
+            v = field(n, a, times)
+        else:
+            v = expert_velocity(cfg, W, a, times, ctx_k, ctx_v, prefix_len, fop, delta, mask)
+        a = a + (grid[n] - grid[n + 1]) * _f64(v)
+    return a, counters + np.uint64(H)
+
+
 def reset(cfg, seeds, H: int | None = None):
     """Warm start with no extra initialization (App. A.1): every slot j holds
     the Gaussian action of index j; the next appended action has index H.

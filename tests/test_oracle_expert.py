@@ -377,3 +377,57 @@ def test_fop_values_closed_form_first_layer():
             o[b, h * hd:(h + 1) * hd] = tot / (P + F + H)
     want = x0[None, None, :] + (o @ W["w_o"][0].astype(np.float64))[:, None, :]
     np.testing.assert_allclose(tr["x"][0], np.broadcast_to(want, tr["x"][0].shape), rtol=1e-9, atol=1e-9)
+
+
+# ----------------------------------------------------------------------------- full-chunk denoising baseline
+
+
+def test_denoise_chunk_constant_field_and_noise_indices():
+    # c = 0 leaves the chunk at its fresh noise: actions counters .. counters + H - 1;
+    # a constant field c moves every action by c * sum(dt) = c
+    cfg = TINY.replace(batch=2, slots=5, action_dim=3)
+    seeds = synth.robot_seeds(13, 2)
+    cnt = np.array([5, 40], np.uint64)
+    for c in (0.0, 1.75):
+        for n_steps in (1, 4, 10):
+            chunk, cnt2 = expert.denoise_chunk(cfg, None, seeds, cnt, n_steps, None, None, 0, None, None,
+                                               field=lambda n, a, tt: np.full_like(a, c))
+            assert list(cnt2) == [10, 45]
+            for b in range(2):
+                for j in range(5):
+                    a0 = noise.action_noise(int(seeds[b]), int(cnt[b]) + j, 3).astype(np.float64)
+                    np.testing.assert_allclose(chunk[b, j], a0 + c, rtol=0, atol=1e-12)
+
+
+def test_denoise_chunk_is_exact_on_the_single_target_field():
+    # v*(a, t) = (target - a) / t is the flow-matching field of one data point
+    # (Eq. 5); Euler is exact on its straight path, so ten (or any number of)
+    # synchronous steps from t = 1 land every slot on its own target
+    cfg = TINY.replace(batch=2, slots=6, action_dim=4)
+    seeds = synth.robot_seeds(17, 2)
+    targets = np.random.default_rng(4).standard_normal((2, 6, 4))
+    seen = []
+
+    def field(n, a, times):
+        seen.append(float(times[0]))
+        assert np.all(times == times[0])               # one flow time for the whole chunk
+        return (targets - a) / float(times[0])
+
+    for n_steps in (1, 3, 10):
+        seen.clear()
+        chunk, _ = expert.denoise_chunk(cfg, None, seeds, np.zeros(2, np.uint64), n_steps, None, None, 0, None,
+                                        None, field=field)
+        np.testing.assert_allclose(chunk, targets, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(seen, 1.0 - np.arange(n_steps) / n_steps, rtol=1e-7)
+
+
+def test_denoise_chunk_one_step_is_one_expert_pass_at_t1():
+    cfg = TINY
+    W, _, _, k, v, P, z, d, _ = _inputs(cfg)
+    seeds = synth.robot_seeds(7, cfg.batch)
+    cnt = np.full(cfg.batch, 9, np.uint64)
+    chunk, _ = expert.denoise_chunk(cfg, W, seeds, cnt, 1, k, v, P, z, d)
+    a0 = np.stack([noise.action_noise(int(seeds[b]), 9 + np.arange(cfg.slots, dtype=np.uint64), cfg.action_dim)
+                   for b in range(cfg.batch)]).astype(np.float64)
+    vel = expert.expert_velocity(cfg, W, a0, np.ones(cfg.slots, np.float32), k, v, P, z, d)
+    np.testing.assert_allclose(chunk, a0 + vel, rtol=1e-12, atol=1e-14)
