@@ -324,6 +324,138 @@ def run_sweep(args):
         torch.cuda.empty_cache()
 
 
+def measure_workload(cfg, args, world, rank, local, e2e=True, denoise_steps=0, swap_every=None):
+    """Time K graph-replayed steps of `cfg` (after W warm-up steps) with one
+    event pair per step on the launching stream, sampling the SM clocks
+    meanwhile; then (optionally) the end-to-end rate through the C ABI with
+    host buffers, a full-horizon denoising chunk of `denoise_steps` passes,
+    and the per-kernel durations of an eager step.  Returns a dict."""
+    import torch
+    import torch.distributed as dist
+    from paper_2609_34170_gb300 import RollingSession, ravel_denoise_chunk, ravel_profile_step, ravel_roll_step
+
+    swap_every = args.swap_every if swap_every is None else swap_every
+    B, P = cfg.batch, cfg.prefix
+    W = synth.make_weights(cfg, 0)
+    sess = RollingSession(cfg, W, local)
+    del W
+    seeds = synth.robot_seeds(7 + 1000 * rank, B)
+    sess.reset(seeds)
+    dtype = sess.dtype
+    ctxs = []
+    for cs in (1000 + rank * 100, 5000 + rank * 100)[:2 if swap_every else 1]:
+        k, v = synth.make_context(cfg, cs, B)
+        ctxs.append((torch.from_numpy(k).to("cuda", dtype), torch.from_numpy(v).to("cuda", dtype)))
+        del k, v
+    sess.set_context(*ctxs[0], P)
+    side = torch.cuda.Stream()
+    z = torch.from_numpy(synth.make_fop(cfg, 2000 + rank, B)).to("cuda", dtype)
+    t_d = torch.from_numpy(synth.staggered_times(cfg.slots)).cuda()
+    deltas = [torch.from_numpy(synth.make_delta(B, 2 + (s % 10), cfg.slots)).cuda() for s in range(10)]
+    delta = torch.empty_like(deltas[0])
+    released = sess.released
+    st = torch.cuda.current_stream()
+    zz = z if cfg.fop_tokens else None
+
+    def one_step(s):
+        if swap_every and s % swap_every == 0 and s > 0:
+            sess.set_context(*ctxs[(s // swap_every) % 2], P, side_stream=side)
+        delta.copy_(deltas[s % 10], non_blocking=True)
+        ravel_roll_step(sess.handle, sess.buffer, t_d, zz, delta, released, None, st)
+
+    for s in range(args.warmup):
+        one_step(s)
+    torch.cuda.synchronize()
+    out = {"kernels_per_step": sess.kernel_count()}
+
+    # ---- timed region: K steps, one event pair per step
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_all0, t_all1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    t_all0.record(st)
+    for s in range(args.steps):
+        ev[s][0].record(st)
+        one_step(args.warmup + s)
+        ev[s][1].record(st)
+    t_all1.record(st)
+    torch.cuda.synchronize()
+    out["clocks"] = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    lat = np.array([a.elapsed_time(b) for a, b in ev])
+    out["total_ms"] = max_over_ranks(t_all0.elapsed_time(t_all1), world)
+    out["p50_us"] = float(np.percentile(lat, 50) * 1e3)
+    out["p99_us"] = float(np.percentile(lat, 99) * 1e3)
+
+    if e2e:
+        # through the C ABI with host buffers: H2D of the step inputs, D2H of the released action
+        z_h = z.cpu().pin_memory()
+        d_h = [d.cpu().pin_memory() for d in deltas]
+        rel_h = torch.empty((B, cfg.action_dim), dtype=torch.float32).pin_memory()
+        z_dev = torch.empty_like(z)
+
+        def e2e_step(s):
+            z_dev.copy_(z_h, non_blocking=True)
+            delta.copy_(d_h[s % 10], non_blocking=True)
+            ravel_roll_step(sess.handle, sess.buffer, t_d, z_dev if cfg.fop_tokens else None, delta, released, None, st)
+            rel_h.copy_(released, non_blocking=True)
+            st.synchronize()
+
+        for s in range(3):
+            e2e_step(s)
+        n_e2e = max(20, args.steps // 2)
+        t0 = time.perf_counter()
+        for s in range(n_e2e):
+            e2e_step(s)
+        out["e2e_s"] = max_over_ranks((time.perf_counter() - t0) / n_e2e, world)
+        out["h2d"] = z_h.numel() * z_h.element_size() + B * 4
+        out["d2h"] = B * cfg.action_dim * 4
+
+    if denoise_steps:
+        # the paper's baseline: a fresh chunk denoised by `denoise_steps` full-horizon passes
+        chunk = torch.empty_like(sess.buffer)
+        for _ in range(3):
+            ravel_denoise_chunk(sess.handle, chunk, denoise_steps, zz, delta, None, st)
+        torch.cuda.synchronize()
+        n_dn = max(5, min(args.steps, 30))
+        evd = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_dn)]
+        for a, b in evd:
+            a.record(st)
+            ravel_denoise_chunk(sess.handle, chunk, denoise_steps, zz, delta, None, st)
+            b.record(st)
+        torch.cuda.synchronize()
+        out["denoise_p50_us"] = float(np.percentile([a.elapsed_time(b) for a, b in evd], 50) * 1e3)
+
+    # ---- per-kernel durations (eager step, events after every launch)
+    per_kind = {}
+    for _ in range(args.profile_steps):
+        for kind, ms in ravel_profile_step(sess.handle, sess.buffer, t_d, zz, delta, released, None, st):
+            per_kind.setdefault(kind, []).append(ms)
+    out["per_kind"] = per_kind
+    sess.close()
+    del ctxs
+    return out
+
+
+def projection_rates(cfg, per_kind, profile_steps, peaks):
+    """TFLOP/s of each projection GEMM kind from its average eager launch time."""
+    rates = {}
+    for kind in ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down"):
+        if kind not in per_kind:
+            continue
+        _, fl = kind_work(kind, cfg, cfg.batch, cfg.prefix)
+        avg_s = float(np.mean(per_kind[kind])) * 1e-3
+        tf = fl / avg_s / 1e12
+        rates[kind] = {"tflops": tf, "frac_of_sustained": tf / peaks["bf16_tflops_sustained"],
+                       "avg_launch_us": avg_s * 1e6}
+    return rates
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -333,6 +465,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--swap-every", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-b64", action="store_true", help="skip the batch-64 object of the default line")
     ap.add_argument("--profile-steps", type=int, default=3)
     ap.add_argument("--sweep", action="store_true",
                     help="latency and roofline fraction over the stress grid (batch x prefix x slots); "
@@ -359,94 +492,12 @@ def main():
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2609_34170_gb300 import RollingSession, ravel_profile_step, ravel_roll_step
 
     B, P = cfg.batch, cfg.prefix
-    W = synth.make_weights(cfg, 0)
-    sess = RollingSession(cfg, W, local)
-    del W
-    seeds = synth.robot_seeds(7 + 1000 * rank, B)
-    sess.reset(seeds)
-    dtype = sess.dtype
-    ctxs = []
-    for cs in (1000 + rank * 100, 5000 + rank * 100):
-        k, v = synth.make_context(cfg, cs, B)
-        ctxs.append((torch.from_numpy(k).to("cuda", dtype), torch.from_numpy(v).to("cuda", dtype)))
-        del k, v
-    sess.set_context(*ctxs[0], P)
-    side = torch.cuda.Stream()
-    z = torch.from_numpy(synth.make_fop(cfg, 2000 + rank, B)).to("cuda", dtype)
-    t_d = torch.from_numpy(synth.staggered_times(cfg.slots)).cuda()
-    deltas = [torch.from_numpy(synth.make_delta(B, 2 + (s % 10), cfg.slots)).cuda() for s in range(10)]
-    delta = torch.empty_like(deltas[0])
-    released, velocity = sess.released, None
-    st = torch.cuda.current_stream()
-
-    def one_step(s):
-        if args.swap_every and s % args.swap_every == 0 and s > 0:
-            sess.set_context(*ctxs[(s // args.swap_every) % 2], P, side_stream=side)
-        delta.copy_(deltas[s % 10], non_blocking=True)
-        ravel_roll_step(sess.handle, sess.buffer, t_d, z if cfg.fop_tokens else None, delta, released, velocity, st)
-
-    for s in range(args.warmup):
-        one_step(s)
-    torch.cuda.synchronize()
-    kernels_per_step = sess.kernel_count()
-
-    # ---- timed region: K steps, one event pair per step
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    t_all0, t_all1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clocks = ClockSampler(local)
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)
-    t_all0.record(st)
-    for s in range(args.steps):
-        ev[s][0].record(st)
-        one_step(args.warmup + s)
-        ev[s][1].record(st)
-    t_all1.record(st)
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    if world > 1:
-        dist.barrier()
-    total_ms = t_all0.elapsed_time(t_all1)
-    lat = np.array([a.elapsed_time(b) for a, b in ev])
-    total_ms = max_over_ranks(total_ms, world)
-    ms_per_step = total_ms / args.steps
-    value = whole_job_rate(world, B, args.steps, total_ms / 1e3)
-
-    # ---- e2e: through the C ABI with host buffers, H2D of the step inputs and D2H of the released action
-    z_h = z.cpu().pin_memory()
-    d_h = [d.cpu().pin_memory() for d in deltas]
-    rel_h = torch.empty((B, cfg.action_dim), dtype=torch.float32).pin_memory()
-    z_dev = torch.empty_like(z)
-    for s in range(3):
-        z_dev.copy_(z_h, non_blocking=True)
-        delta.copy_(d_h[s % 10], non_blocking=True)
-        ravel_roll_step(sess.handle, sess.buffer, t_d, z_dev if cfg.fop_tokens else None, delta, released, None, st)
-        rel_h.copy_(released, non_blocking=True)
-        st.synchronize()
-    n_e2e = max(20, args.steps // 2)
-    t0 = time.perf_counter()
-    for s in range(n_e2e):
-        z_dev.copy_(z_h, non_blocking=True)
-        delta.copy_(d_h[s % 10], non_blocking=True)
-        ravel_roll_step(sess.handle, sess.buffer, t_d, z_dev if cfg.fop_tokens else None, delta, released, None, st)
-        rel_h.copy_(released, non_blocking=True)
-        st.synchronize()
-    e2e_s = max_over_ranks((time.perf_counter() - t0) / n_e2e, world)
-    h2d = z_h.numel() * z_h.element_size() + B * 4
-    d2h = B * cfg.action_dim * 4
-
-    # ---- per-kernel durations (eager step, events after every launch)
-    per_kind = {}
-    for _ in range(args.profile_steps):
-        for kind, ms in ravel_profile_step(sess.handle, sess.buffer, t_d, z if cfg.fop_tokens else None, delta,
-                                           released, None, st):
-            per_kind.setdefault(kind, []).append(ms)
+    m = measure_workload(cfg, args, world, rank, local, e2e=True, denoise_steps=10 if B * cfg.slots <= 512 else 0)
+    per_kind = m["per_kind"]
+    ms_per_step = m["total_ms"] / args.steps
+    value = whole_job_rate(world, B, args.steps, m["total_ms"] / 1e3)
     tot = {k: sum(v) / args.profile_steps for k, v in per_kind.items()}
     grand = sum(tot.values())
     dom = max(tot, key=tot.get)
@@ -470,28 +521,49 @@ def main():
         "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic (seeded N(0,0.02) weights, N(0,1) prefix/FOP)",
         "config": dict(workload_config(cfg), parallelism=f"replicas x{world}",
                        context_swap_every=args.swap_every),
-        "p50_us": float(np.percentile(lat, 50) * 1e3), "p99_us": float(np.percentile(lat, 99) * 1e3),
-        "steps_per_s": args.steps / (total_ms / 1e3),
+        "p50_us": m["p50_us"], "p99_us": m["p99_us"],
+        "steps_per_s": args.steps / (m["total_ms"] / 1e3),
         "step_roofline": {"bytes": work["bytes"], "flops": work["flops"], "time_us": step_roof_s * 1e6,
-                          "frac_of_p50": step_roof_s * 1e6 / float(np.percentile(lat, 50) * 1e3),
-                          "peaks": peak_src},
+                          "frac_of_p50": step_roof_s * 1e6 / m["p50_us"], "peaks": peak_src},
         "roofline": {"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
                      "frac": (achieved / peak) if achieved else None,
                      "traffic": measured_traffic(args.config, dom), "algorithmic_bytes": kb,
                      "launches_per_step": nlaunch, "avg_launch_us": avg_ms * 1e3,
                      "share_of_step": tot[dom] / grand, "peak_source": f"{peak_src} (MEASURED_PEAKS.json)"},
         "kernel_shares": {k: round(v / grand, 4) for k, v in sorted(tot.items(), key=lambda x: -x[1])},
-        "e2e": {"value": whole_job_rate(world, B, 1, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
-        "gpu_launches": kernels_per_step * args.steps + (args.steps // args.swap_every if args.swap_every else 0),
-        "clocks": clk,
+        "e2e": {"value": whole_job_rate(world, B, 1, m["e2e_s"]), "unit": UNIT, "h2d_bytes_per_step": m["h2d"],
+                "d2h_bytes_per_step": m["d2h"]},
+        "gpu_launches": m["kernels_per_step"] * args.steps + (args.steps // args.swap_every if args.swap_every else 0),
+        "clocks": m["clocks"],
     }
+    if "denoise_p50_us" in m:
+        # the structure of the paper's Table 1 (full denoising vs rolling first-action latency) on this GPU:
+        # ten full-horizon expert passes for a fresh chunk against one rolling step
+        out["paper_comparison"] = {"full_denoise_10_passes_p50_us": m["denoise_p50_us"],
+                                   "rolling_step_p50_us": m["p50_us"],
+                                   "ratio": m["denoise_p50_us"] / m["p50_us"]}
+    del m
+    if rank == 0 and world == 1 and not args.no_b64 and args.config == "pi05_bf16_b1":
+        # the throughput workload (same expert, 64 robots): latency, rate, step roofline, projection TFLOP/s
+        cfg64 = synth.PRESETS["pi05_bf16_b64"]
+        m64 = measure_workload(cfg64, args, 1, 0, local, e2e=False, swap_every=0)
+        w64 = step_work(cfg64, cfg64.batch, cfg64.prefix)
+        roof64 = max(w64["bytes"] / (peaks["hbm_gbs"] * 1e9), w64["flops"] / (peaks["bf16_tflops"] * 1e12))
+        out["b64"] = {"workload": workload_config(cfg64)["workload"], "steps": args.steps, "warmup": args.warmup,
+                      "p50_us": m64["p50_us"], "p99_us": m64["p99_us"],
+                      "robot_steps_per_s": cfg64.batch * args.steps / (m64["total_ms"] / 1e3),
+                      "step_roofline_us": roof64 * 1e6, "frac_of_p50": roof64 * 1e6 / m64["p50_us"],
+                      "projection_gemms": projection_rates(cfg64, m64["per_kind"], args.profile_steps, peaks),
+                      "peak_note": "TFLOP/s from eager per-launch CUDA events; fraction of the measured sustained "
+                                   "bf16 peak (MEASURED_PEAKS.json)",
+                      "clocks": m64["clocks"]}
+        out["gpu_launches"] += m64["kernels_per_step"] * args.steps
+        del m64
+        torch.cuda.empty_cache()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        del ctxs
         out["cpu_baseline"] = cpu_baseline(cfg)
     if rank == 0:
         print(json.dumps(out), flush=True)
-    sess.close()
     if world > 1:
         dist.destroy_process_group()
 

@@ -150,6 +150,25 @@ ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int pre
 ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
                              const float* delta, float* released, float* velocity, void* stream);
 
+/* The full-horizon (synchronous) denoising that the paper compares rolling
+ * inference with (Experiments, synchronous simulation: ten full-horizon
+ * denoising steps per policy query; Table 1): every robot draws a fresh chunk
+ * of H Gaussian actions -- its next H action indices; its counter advances by
+ * H -- and all H slots then take n_steps Euler steps together, each one pass
+ * of the same action expert with every slot at one flow time t_n = 1 - n /
+ * n_steps (float32), followed by a += (t_n - t_{n+1}) v with t_{n_steps} = 0.
+ * Nothing is released, shifted or appended: the returned chunk (t = 0) is
+ * executed as a whole.
+ *   chunk        device float32 [B, H, A], written: the denoised chunk
+ *   n_steps      1 .. 64 (the paper's baseline uses 10)
+ *   obs_tokens, delta: as for ravel_roll_step
+ *   velocity     device float32 [B, H, A] or NULL: the last pass's velocity
+ * Enqueued on `stream` as one CUDA-graph launch (captured on first use, and
+ * again when n_steps or a pointer changes); a pending context swap is applied
+ * first, as for ravel_roll_step. */
+ravel_status ravel_denoise_chunk(ravel_t* r, float* chunk, int n_steps, const void* obs_tokens, const float* delta,
+                                 float* velocity, void* stream);
+
 /* Per-robot action counters (the index of the next appended action), host
  * uint64 [B].  get synchronises the handle's device; set is synchronous and
  * lets a rollout resume bit-exactly. */

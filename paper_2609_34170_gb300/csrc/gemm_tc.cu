@@ -106,6 +106,8 @@ struct TcParams {
   unsigned long long wait_ns;   // limit of every bounded wait (ERR_TIMEOUT after it)
   int withhold;         // fault injection (tests): the MMA thread first waits for an arrival that
                         // nobody makes, so the launch gives up after wait_ns and unwinds
+  const int* skip;      // optional device flag read after the dependency wait: nonzero -> the launch
+                        // completes the copies it started and exits without computing
 };
 
 // The TMA epilogue kind of a launch (EK_F32 .. EK_GEGLU).
@@ -527,6 +529,24 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   // everything below may read what earlier kernels wrote; TMEM is taken only
   // now, so a CTA waiting here never holds columns its predecessor needs
   pdl_wait();
+  if (p.skip && *p.skip) {
+    // nothing to compute (the flag is the same for every CTA): the token
+    // tiles of the stages loaded before the wait are fetched as well, so that
+    // each barrier completes as armed, and the CTA leaves once they landed
+    if (threadIdx.x == 0 && has_work) {
+      if (p.oneshot) {
+        tma_load_3d(&tmX, &full[0], b_s, 0, tm0 * BN, kb0_first, pol_x);
+        if (!mbar_wait(&full[0], 0)) raise_error(p.err, ERR_TIMEOUT);
+      } else {
+        for (int i = 0; i < npre; ++i)
+          tma_load_2d(&tmX, &full[i], b_s + (size_t)i * b_bytes, (kb0_first + i) * TC_BK, tm0 * BN, pol_x);
+        for (int i = 0; i < npre; ++i)
+          if (!mbar_wait(&full[i], 0)) raise_error(p.err, ERR_TIMEOUT);
+      }
+    }
+    cta_sync();
+    return;
+  }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"(ncols)
@@ -957,6 +977,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
   }
   pdl_wait();
+  if (p.skip && *p.skip) {
+    // nothing to compute: both CTAs fetch the token halves of the stages
+    // loaded before the wait (completing on the even CTA's barriers), the even
+    // CTA waits for them, and neither leaves before the other
+    if (threadIdx.x == 0) {
+      for (int i = 0; i < npre; ++i)
+        tma_load_2d_pair(&tmX, full0 + 8u * (uint32_t)i, b_s + (size_t)i * bh_bytes, i * TC_BK,
+                         tm0 * BN + (int)rank * BNh, pol_x);
+      if (leader)
+        for (int i = 0; i < npre; ++i)
+          if (!mbar_wait(&full[i], 0)) raise_error(p.err, ERR_TIMEOUT);
+    }
+    cluster_sync();
+    return;
+  }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"(ncols)
@@ -1259,7 +1294,7 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
   TcParams p{g.M, g.N, g.K, bn, stages, 1, num_kb, RED_NONE, (uint32_t)ring, acc_cols, tiles_n, tiles_m, num_tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, 1, 0, box_m, box_bytes, stg_off, xch_off,
-             vts_off, 0, bar_off, kTcTimeoutNs, 0};
+             vts_off, 0, bar_off, kTcTimeoutNs, 0, g.skip};
   const int npairs = std::min(num_tiles, slots);
   return launch_kernel_cluster(tc_pair_kernel(ek), dim3(2 * npairs), dim3(TC_THREADS), smem, st, dim3(2, 1, 1), mw, mx,
                                mo, p);
@@ -1414,7 +1449,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
-             vts_off, rcv_off, bar_off, kTcTimeoutNs, 0};
+             vts_off, rcv_off, bar_off, kTcTimeoutNs, 0, g.skip};
   // fault injection (tests): a launch without a cluster may be told to wait
   // for an arrival that never comes, with a short limit
   if ((reduce == RED_NONE || reduce == RED_WORKSPACE) && g_withhold.load() > 0 && g_withhold.fetch_sub(1) > 0) {

@@ -28,11 +28,39 @@ cudaError_t launch_pack_transpose(const float* src, int K, int N, void* dst, Dty
 cudaError_t launch_convert(const float* src, size_t n, void* dst, Dtype dt, cudaStream_t st);
 
 // ---- conditioning -------------------------------------------------------------
+// Steady-state cache of the conditioning (the modulation rows of the H slot
+// times, and of up to kCondCache distinct context offsets).  cond_check
+// compares this step's slot times and offsets with the cached keys, maps each
+// robot to the modv row of its offset part (drow), lists the rows to copy
+// into the cache after the modulation GEMM, and sets `skip` when every row is
+// cached (the conditioning launches then compute nothing); cond_commit copies
+// the listed rows.  modv rows: [0, H) slot times, [H, H + Bmax) this step's
+// offsets, [H + Bmax, H + Bmax + kCondCache) cached offsets.
+constexpr int kCondCache = 16;
+struct CondCache {
+  int skip;                     // this step: every row cached
+  int t_valid;                  // t_key holds the slot times of modv rows [0, H)
+  int n_commit;
+  int next;                     // round-robin victim
+  int used[kCondCache];
+  float delta[kCondCache];
+};
+struct CondArgs {
+  CondCache* cc; float* t_key;  // [H]
+  int* drow;                    // [Bmax] out: modv row of robot b's offset part
+  int* commit;                  // [Bmax] pairs (src row, dst row) as 2 ints each -> [2 Bmax]
+  const float* slot_times; const float* delta;
+  int H, B, Bmax;
+  float* modv; int mod_ld;
+  int enabled;                  // 0: always compute, drow = H + b
+};
+cudaError_t launch_cond_check(const CondArgs& a, cudaStream_t st);
+cudaError_t launch_cond_commit(const CondArgs& a, cudaStream_t st);
 // E[r][:] = sinusoidal(x_r) for r < H (x = slot_times[r]) and H <= r < H+B
 // (x = delta[r-H]); periods geometric from 4e-3 to 4; fp64 angles reduced mod 2 pi.
 // omega: device fp64 [D/2] angular frequencies 2 pi / p_i.
 cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, const double* omega,
-                         void* E, Dtype dt, cudaStream_t st);
+                         void* E, Dtype dt, cudaStream_t st, const int* skip = nullptr);
 
 // ---- generic projection GEMM: out[m][n] = sum_k A[m][k] W[n][k] (W K-major) ----
 enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2, EPI_GEGLU = 3 };
@@ -50,6 +78,7 @@ struct GemmArgs {
   void* vt = nullptr;
   int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
   int max_splits = 0;           // tcgen05 path: cap on the split-K factor (0: chosen from the shape)
+  const int* skip = nullptr;    // optional device flag: nonzero at run time -> the launch computes nothing
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
 
@@ -85,6 +114,7 @@ struct NormArgs {
   const float* modv; int mod_ld; const float* mod_b; int off;
   const void* fop; int F; const float* gamma;
   void* Y; int row_pitch;
+  const int* drow = nullptr;    // optional: row of modv holding robot b's offset part (default H + b)
 };
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 
@@ -142,6 +172,15 @@ struct TailArgs {
   int B, H, A;
 };
 cudaError_t launch_tail(const TailArgs& a, cudaStream_t st);
+
+// Synchronous (full-horizon) denoising: buffer += (t_now - t_next) * vel for
+// every slot (vel_out optional copy); times[0..H-1] = t; a fresh chunk
+// buffer[b][j] = noise(seeds[b], counters[b] + j), counters[b] += H.
+cudaError_t launch_denoise_tail(float* buffer, const float* vel, float* vel_out, int B, int H, int A, float t_now,
+                                float t_next, cudaStream_t st);
+cudaError_t launch_fill_times(float* times, int H, float t, cudaStream_t st);
+cudaError_t launch_chunk_noise(float* buffer, const uint64_t* seeds, uint64_t* counters, int B, int H, int A,
+                               cudaStream_t st);
 
 // buffer[b][j] = noise(seeds[b], j) for j < H; counters[b] = H.
 cudaError_t launch_reset(float* buffer, const uint64_t* seeds, uint64_t* counters, int B, int H, int A,

@@ -68,9 +68,10 @@ cudaError_t launch_convert(const float* src, size_t n, void* dst, Dtype dt, cuda
 // reduced angle (|a| <= pi) in fp32.
 template <typename T>
 __global__ void embed_kernel(const float* __restrict__ slot_times, int H, const float* __restrict__ delta, int D,
-                             const double* __restrict__ omega, T* __restrict__ E) {
+                             const double* __restrict__ omega, T* __restrict__ E, const int* __restrict__ skip) {
   pdl_trigger();
   pdl_wait();
+  if (skip && *skip) return;
   const int r = blockIdx.y;
   const double x = (r < H) ? (double)slot_times[r] : (double)delta[r - H];
   const int half = D / 2;
@@ -85,11 +86,113 @@ __global__ void embed_kernel(const float* __restrict__ slot_times, int H, const 
 }
 
 cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int B, int D, const double* omega,
-                         void* E, Dtype dt, cudaStream_t st) {
+                         void* E, Dtype dt, cudaStream_t st, const int* skip) {
   dim3 grid((D / 2 + 127) / 128, H + B);
   if (dt == DT_BF16)
-    return launch_kernel(embed_kernel<bf16>, grid, dim3(128), 0, st, 1, slot_times, H, delta, D, omega, (bf16*)E);
-  return launch_kernel(embed_kernel<float>, grid, dim3(128), 0, st, 1, slot_times, H, delta, D, omega, (float*)E);
+    return launch_kernel(embed_kernel<bf16>, grid, dim3(128), 0, st, 1, slot_times, H, delta, D, omega, (bf16*)E,
+                         skip);
+  return launch_kernel(embed_kernel<float>, grid, dim3(128), 0, st, 1, slot_times, H, delta, D, omega, (float*)E,
+                       skip);
+}
+
+// ============================================================================ conditioning cache
+
+// One block: which rows of this step's conditioning are cached already (see
+// CondCache).  The slot times hit when every one equals the cached key; a
+// robot's offset hits when its value is one of the cached offsets.  Misses
+// get a cache slot (a slot already referenced in this step is never taken;
+// with no slot left the robot keeps this step's fresh row), and their keys
+// are written now: the rows themselves arrive through cond_commit before
+// any reader of this step, and a later step reads them only after that.
+__global__ void cond_check_kernel(CondArgs a) {
+  __shared__ int s_tmiss;
+  __shared__ unsigned s_ref;   // cache slots referenced by this step
+  pdl_trigger();
+  pdl_wait();
+  CondCache* cc = a.cc;
+  if (threadIdx.x == 0) {
+    s_tmiss = a.enabled ? !cc->t_valid : 1;
+    s_ref = 0u;
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j < a.H; j += blockDim.x)
+    if (a.slot_times[j] != a.t_key[j]) s_tmiss = 1;   // benign race: every writer stores 1
+  // offsets: look up in parallel; -1 = miss
+  for (int b = threadIdx.x; b < a.B; b += blockDim.x) {
+    int row = -1;
+    if (a.enabled) {
+      const float d = a.delta[b];
+      for (int c = 0; c < kCondCache; ++c)
+        if (cc->used[c] && cc->delta[c] == d) {
+          row = a.H + a.Bmax + c;
+          atomicOr(&s_ref, 1u << c);
+          break;
+        }
+    }
+    a.drow[b] = row;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int any_miss = s_tmiss, nc = 0;
+    unsigned ref = s_ref;
+    for (int b = 0; b < a.B; ++b) {
+      if (a.drow[b] >= 0) continue;
+      any_miss = 1;
+      const float d = a.delta[b];
+      int row = a.H + b;   // this step's fresh row unless a cache slot is found
+      if (a.enabled) {
+        int c = -1;
+        for (int k = 0; k < kCondCache; ++k)   // assigned to an earlier robot of this step?
+          if ((ref >> k & 1u) && cc->used[k] && cc->delta[k] == d) c = k;
+        if (c < 0) {
+          for (int k = 0; k < kCondCache && c < 0; ++k) {
+            const int v = (cc->next + k) % kCondCache;
+            if (!(ref >> v & 1u)) c = v;
+          }
+          if (c >= 0) {
+            cc->next = (c + 1) % kCondCache;
+            cc->delta[c] = d;
+            cc->used[c] = 1;
+            a.commit[2 * nc] = a.H + b;
+            a.commit[2 * nc + 1] = a.H + a.Bmax + c;
+            ++nc;
+          }
+        }
+        if (c >= 0) {
+          ref |= 1u << c;
+          row = a.H + a.Bmax + c;
+        }
+      }
+      a.drow[b] = row;
+    }
+    cc->n_commit = nc;
+    cc->skip = any_miss ? 0 : 1;
+    if (a.enabled) cc->t_valid = 1;
+  }
+  // the slot times become the key (a miss recomputes rows [0, H) this step)
+  if (a.enabled)
+    for (int j = threadIdx.x; j < a.H; j += blockDim.x) a.t_key[j] = a.slot_times[j];
+}
+
+cudaError_t launch_cond_check(const CondArgs& a, cudaStream_t st) {
+  return launch_kernel(cond_check_kernel, dim3(1), dim3(256), 0, st, 1, a);
+}
+
+// Copies the rows that cond_check listed (this step's fresh offset rows) into
+// their cache slots.
+__global__ void cond_commit_kernel(CondArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  const int n = a.cc->n_commit;
+  for (int i = 0; i < n; ++i) {
+    const float4* src = (const float4*)(a.modv + (size_t)a.commit[2 * i] * a.mod_ld);
+    float4* dst = (float4*)(a.modv + (size_t)a.commit[2 * i + 1] * a.mod_ld);
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < a.mod_ld / 4; c += gridDim.x * blockDim.x) dst[c] = src[c];
+  }
+}
+
+cudaError_t launch_cond_commit(const CondArgs& a, cudaStream_t st) {
+  return launch_kernel(cond_commit_kernel, dim3(64), dim3(256), 0, st, 1, a);
 }
 
 // ============================================================================ GEMM (SIMT)
@@ -99,9 +202,10 @@ cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int
 template <typename T, int EPI, typename TO>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, int lda, const T* __restrict__ W,
                                                         int ldw, int M, int N, int K, TO* __restrict__ out, int ldo,
-                                                        const float* __restrict__ bias) {
+                                                        const float* __restrict__ bias, const int* __restrict__ skip) {
   pdl_trigger();
   pdl_wait();
+  if (skip && *skip) return;
   __shared__ float As[32][64 + 4];
   __shared__ float Ws[32][64 + 4];
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
@@ -156,21 +260,21 @@ static cudaError_t gemm_simt_dispatch(const GemmArgs& g, cudaStream_t st) {
   const T* W = (const T*)g.W;
   if (g.epi == EPI_ADD_F32) {
     launch_kernel(gemm_simt_kernel<T, EPI_ADD_F32, float>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
-                                                                 g.ldo, g.bias);
+                                                                 g.ldo, g.bias, g.skip);
   } else if (g.out_dt == DT_BF16) {
     if (g.epi == EPI_STORE_SILU)
       launch_kernel(gemm_simt_kernel<T, EPI_STORE_SILU, bf16>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K,
-                                                                     (bf16*)g.out, g.ldo, g.bias);
+                                                                     (bf16*)g.out, g.ldo, g.bias, g.skip);
     else
       launch_kernel(gemm_simt_kernel<T, EPI_STORE, bf16>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K, (bf16*)g.out,
-                                                                g.ldo, g.bias);
+                                                                g.ldo, g.bias, g.skip);
   } else {
     if (g.epi == EPI_STORE_SILU)
       launch_kernel(gemm_simt_kernel<T, EPI_STORE_SILU, float>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K,
-                                                                      (float*)g.out, g.ldo, g.bias);
+                                                                      (float*)g.out, g.ldo, g.bias, g.skip);
     else
       launch_kernel(gemm_simt_kernel<T, EPI_STORE, float>, grid, dim3(256), 0, st, 1, A, g.lda, W, g.ldw, g.M, g.N, g.K, (float*)g.out,
-                                                                 g.ldo, g.bias);
+                                                                 g.ldo, g.bias, g.skip);
   }
   return cudaGetLastError();
 }
@@ -247,7 +351,7 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, i
     }
   }
   pdl_wait();
-  const float* md = a.modv + (size_t)(a.H + b) * a.mod_ld + a.off;
+  const float* md = a.modv + (size_t)(a.drow ? a.drow[b] : a.H + b) * a.mod_ld + a.off;
   int buf = 0;
   for (int j = j0; j < j1; j += R, buf ^= 1) {
     float4 xv[R][G], ts[R][G], th[R][G];
@@ -591,6 +695,67 @@ cudaError_t launch_tail(const TailArgs& a, cudaStream_t st) {
   if (a.B <= 0) return cudaSuccess;
   const size_t smem = (size_t)a.H * a.A * sizeof(float);
   return launch_kernel(tail_kernel, dim3(a.B), dim3(256), smem, st, 1, a);
+}
+
+// Full-horizon denoising (the synchronous baseline): every slot takes the
+// same Euler step a += dt v with dt = t_now - t_next (float32, read off the
+// time grid like the rolling step's dt_j); nothing is released or shifted.
+__global__ void denoise_tail_kernel(float* __restrict__ buffer, const float* __restrict__ vel, float* __restrict__ vel_out,
+                                    int n, float t_now, float t_next) {
+  pdl_trigger();
+  pdl_wait();
+  const float dt = __fsub_rn(t_now, t_next);
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+    const float v = vel[i];
+    buffer[i] = fmaf(dt, v, buffer[i]);
+    if (vel_out) vel_out[i] = v;
+  }
+}
+
+cudaError_t launch_denoise_tail(float* buffer, const float* vel, float* vel_out, int B, int H, int A, float t_now,
+                                float t_next, cudaStream_t st) {
+  const int n = B * H * A;
+  if (n <= 0) return cudaSuccess;
+  const int blocks = std::min((n + 255) / 256, 1024);
+  return launch_kernel(denoise_tail_kernel, dim3(blocks), dim3(256), 0, st, 1, buffer, vel, vel_out, n, t_now, t_next);
+}
+
+// times[0..H-1] = t (the single flow time of a synchronous denoising pass).
+__global__ void fill_times_kernel(float* __restrict__ times, int H, float t) {
+  pdl_trigger();
+  pdl_wait();
+  for (int j = threadIdx.x; j < H; j += blockDim.x) times[j] = t;
+}
+
+cudaError_t launch_fill_times(float* times, int H, float t, cudaStream_t st) {
+  return launch_kernel(fill_times_kernel, dim3(1), dim3(128), 0, st, 1, times, H, t);
+}
+
+// A fresh chunk: slot j of robot b receives the Gaussian action of index
+// counters[b] + j, and the counter advances by H.
+__global__ void chunk_noise_kernel(float* __restrict__ buffer, const uint64_t* __restrict__ seeds,
+                                   uint64_t* __restrict__ counters, int H, int A) {
+  pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int groups = (A + 3) / 4;
+  const uint64_t n0 = counters[b];
+  for (int i = threadIdx.x; i < H * groups; i += blockDim.x) {
+    const int j = i / groups, g = i % groups;
+    float z[4];
+    action_noise4(seeds[b], n0 + (uint64_t)j, (uint32_t)g, z);
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+      if (4 * g + t < A) buffer[((size_t)b * H + j) * A + 4 * g + t] = z[t];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) counters[b] = n0 + (uint64_t)H;
+}
+
+cudaError_t launch_chunk_noise(float* buffer, const uint64_t* seeds, uint64_t* counters, int B, int H, int A,
+                               cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  return launch_kernel(chunk_noise_kernel, dim3(B), dim3(128), 0, st, 1, buffer, seeds, counters, H, A);
 }
 
 cudaError_t init_simt_kernels() {

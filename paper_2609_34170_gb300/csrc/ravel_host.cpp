@@ -42,6 +42,10 @@ struct ravel_ctx {
   StepIO graph_io{};
   int graph_batch = -1;
   int graph_kernels = 0;
+  // graph of a full-horizon denoising chunk (ravel_denoise_chunk)
+  cudaGraphExec_t dn_gexec = nullptr;
+  StepIO dn_io{};
+  int dn_batch = -1, dn_steps = 0;
   // asynchronously mirrored device error word
   int* err_host = nullptr;     // pinned
   std::string last_error;
@@ -118,6 +122,7 @@ void ravel_destroy(ravel_t* r) {
   cudaSetDevice(r->device);
   cudaDeviceSynchronize();
   if (r->gexec) cudaGraphExecDestroy(r->gexec);
+  if (r->dn_gexec) cudaGraphExecDestroy(r->dn_gexec);
   if (r->cap_stream) cudaStreamDestroy(r->cap_stream);
   if (r->ev_step_done) cudaEventDestroy(r->ev_step_done);
   if (r->ev_ctx_ready) cudaEventDestroy(r->ev_ctx_ready);
@@ -136,6 +141,9 @@ ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* bu
   // can be cleared
   RV_CUDA(r, cudaDeviceSynchronize(), "reset: sync");
   RV_CUDA(r, cudaMemset(r->plan.err, 0, sizeof(int)), "reset: clear error word");
+  // a new rollout starts with an empty conditioning cache (its rows are then
+  // computed at this batch size only)
+  RV_CUDA(r, cudaMemset(r->plan.cond, 0, sizeof(CondCache)), "reset: clear conditioning cache");
   *r->err_host = 0;
   RV_CUDA(r, cudaMemcpy(r->plan.seeds, seeds, sizeof(uint64_t) * batch, cudaMemcpyHostToDevice), "reset: seeds");
   RV_CUDA(r, launch_reset(buffer, r->plan.seeds, r->plan.counters, batch, r->plan.cfg.slots,
@@ -205,6 +213,17 @@ static ravel_status check_device_errors(ravel_t* r) {
   return RAVEL_OK;
 }
 
+// A context installed by ravel_set_context since the last step: make `st`
+// wait for its copy and switch the device state to it.
+static ravel_status apply_pending_swap(ravel_t* r, cudaStream_t st) {
+  if (!r->swap_pending) return RAVEL_OK;
+  RV_CUDA(r, cudaStreamWaitEvent(st, r->ev_ctx_ready, 0), "wait for context");
+  RV_CUDA(r, launch_flip(r->plan.ctx_state, r->pending_slot, r->pending_len, st), "context flip");
+  r->active_host = r->pending_slot;
+  r->swap_pending = false;
+  return RAVEL_OK;
+}
+
 ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
                              const float* delta, float* released, float* velocity, void* stream) {
   if (!r || !buffer || !slot_times || !delta || !released) return fail(r, RAVEL_EINVAL, "roll_step: null argument");
@@ -215,12 +234,8 @@ ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times,
   if (s != RAVEL_OK) return s;
   RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
   cudaStream_t st = (cudaStream_t)stream;
-  if (r->swap_pending) {
-    RV_CUDA(r, cudaStreamWaitEvent(st, r->ev_ctx_ready, 0), "roll_step: wait for context");
-    RV_CUDA(r, launch_flip(r->plan.ctx_state, r->pending_slot, r->pending_len, st), "roll_step: flip");
-    r->active_host = r->pending_slot;
-    r->swap_pending = false;
-  }
+  s = apply_pending_swap(r, st);
+  if (s != RAVEL_OK) return s;
   StepIO io{buffer, slot_times, obs_tokens, delta, released, velocity};
   if (!r->gexec || r->graph_batch != r->batch || memcmp(&io, &r->graph_io, sizeof io) != 0) {
     if (r->gexec) {
@@ -246,6 +261,63 @@ ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times,
     r->graph_kernels = nk;
   }
   RV_CUDA(r, cudaGraphLaunch(r->gexec, st), "graph launch");
+  RV_CUDA(r, cudaEventRecord(r->ev_step_done, st), "record step");
+  RV_CUDA(r, cudaMemcpyAsync(r->err_host, r->plan.err, sizeof(int), cudaMemcpyDeviceToHost, st), "error mirror");
+  r->any_step = true;
+  return RAVEL_OK;
+}
+
+ravel_status ravel_denoise_chunk(ravel_t* r, float* chunk, int n_steps, const void* obs_tokens, const float* delta,
+                                 float* velocity, void* stream) {
+  if (!r || !chunk || !delta) return fail(r, RAVEL_EINVAL, "denoise_chunk: null argument");
+  if (n_steps < 1 || n_steps > 64) return fail(r, RAVEL_EINVAL, "denoise_chunk: n_steps outside [1, 64]");
+  if (r->plan.cfg.fop_tokens > 0 && !obs_tokens) return fail(r, RAVEL_EINVAL, "denoise_chunk: obs_tokens is null");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "denoise_chunk: call ravel_reset first");
+  if (!r->have_ctx) return fail(r, RAVEL_ENOCONTEXT, "denoise_chunk: no context set");
+  ravel_status s = check_device_errors(r);
+  if (s != RAVEL_OK) return s;
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  cudaStream_t st = (cudaStream_t)stream;
+  s = apply_pending_swap(r, st);
+  if (s != RAVEL_OK) return s;
+  StepIO io{chunk, r->plan.dn_times, obs_tokens, delta, nullptr, velocity};
+  if (!r->dn_gexec || r->dn_batch != r->batch || r->dn_steps != n_steps || memcmp(&io, &r->dn_io, sizeof io) != 0) {
+    if (r->dn_gexec) {
+      RV_CUDA(r, cudaStreamSynchronize(st), "denoise_chunk: sync before re-capture");
+      cudaGraphExecDestroy(r->dn_gexec);
+      r->dn_gexec = nullptr;
+    }
+    const ravel_config& c = r->plan.cfg;
+    cudaGraph_t graph = nullptr;
+    RV_CUDA(r, cudaStreamBeginCapture(r->cap_stream, cudaStreamCaptureModeThreadLocal), "capture begin");
+    // a fresh chunk of H Gaussian actions, then n_steps passes at one flow
+    // time each, t_n = 1 - n / n_steps, stepping to t_{n+1} (t_{n_steps} = 0)
+    cudaError_t e = launch_chunk_noise(chunk, r->plan.seeds, r->plan.counters, r->batch, c.slots, c.action_dim,
+                                       r->cap_stream);
+    for (int n = 0; n < n_steps && e == cudaSuccess; ++n) {
+      const float t_now = (float)(1.0 - (double)n / n_steps);
+      const float t_next = n + 1 < n_steps ? (float)(1.0 - (double)(n + 1) / n_steps) : 0.f;
+      e = launch_fill_times(r->plan.dn_times, c.slots, t_now, r->cap_stream);
+      if (e == cudaSuccess) {
+        const DenoisePass dn{t_now, t_next};
+        int nk = 0;
+        e = enqueue_step(r->plan, r->batch, io, r->cap_stream, &nk, nullptr, &dn);
+      }
+    }
+    cudaError_t e2 = cudaStreamEndCapture(r->cap_stream, &graph);
+    if (e != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      return cuda_fail(r, e, "denoise_chunk: enqueue");
+    }
+    RV_CUDA(r, e2, "capture end");
+    e = cudaGraphInstantiateWithFlags(&r->dn_gexec, graph, 0);
+    cudaGraphDestroy(graph);
+    RV_CUDA(r, e, "graph instantiate");
+    r->dn_io = io;
+    r->dn_batch = r->batch;
+    r->dn_steps = n_steps;
+  }
+  RV_CUDA(r, cudaGraphLaunch(r->dn_gexec, st), "graph launch");
   RV_CUDA(r, cudaEventRecord(r->ev_step_done, st), "record step");
   RV_CUDA(r, cudaMemcpyAsync(r->err_host, r->plan.err, sizeof(int), cudaMemcpyDeviceToHost, st), "error mirror");
   r->any_step = true;
@@ -301,12 +373,8 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
   if (s != RAVEL_OK) return s;
   RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
   cudaStream_t st = (cudaStream_t)stream;
-  if (r->swap_pending) {
-    RV_CUDA(r, cudaStreamWaitEvent(st, r->ev_ctx_ready, 0), "profile_step: wait for context");
-    RV_CUDA(r, launch_flip(r->plan.ctx_state, r->pending_slot, r->pending_len, st), "profile_step: flip");
-    r->active_host = r->pending_slot;
-    r->swap_pending = false;
-  }
+  s = apply_pending_swap(r, st);
+  if (s != RAVEL_OK) return s;
   // hold the stream for a few ms so that every launch below is queued before
   // the first one starts: the events then time the kernels, not the host
   RV_CUDA(r, launch_delay(5000000ull, st), "profile_step: delay");

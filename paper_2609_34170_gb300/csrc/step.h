@@ -43,7 +43,13 @@ struct StepPlan {
   double* omega = nullptr;   // [D/2] angular frequencies of the embedding
   void* H1 = nullptr;     // [H+Bmax][D]  first MLP layer (SiLU)
   void* HC = nullptr;     // [H+Bmax][D]  MLP outputs h_t, h_delta
-  float* modv = nullptr;  // [H+Bmax][mod_dim]  h @ W_mod (bias added in the norms)
+  float* modv = nullptr;  // [H+Bmax+kCondCache][mod_dim]  h @ W_mod (bias added in the norms):
+                          // slot-time rows, this step's offset rows, cached offset rows
+  CondCache* cond = nullptr;   // steady-state conditioning cache (kernels.h)
+  float* cond_tkey = nullptr;  // [H]
+  int* cond_drow = nullptr;    // [Bmax]
+  int* cond_commit = nullptr;  // [2 Bmax]
+  bool cond_cache = true;
   float* x = nullptr;     // [Bmax*H][D]  residual stream
   void* Y = nullptr;      // [Bmax*(H+F)][D]  normed rows (actions, then FOP tokens)
   void* QKV = nullptr;    // [Bmax*(H+F)][nqkv]
@@ -62,6 +68,7 @@ struct StepPlan {
   TcWorkspace tcws{};       // split-K workspace of the tensor-core GEMM
   int num_sms = 0;
   bool use_tc = false;      // bf16 projections on tcgen05
+  float* dn_times = nullptr;   // [H] flow times of a synchronous denoising pass (all equal)
   uint64_t* seeds = nullptr;
   uint64_t* counters = nullptr;
   int* err = nullptr;
@@ -75,7 +82,7 @@ void plan_destroy(StepPlan* p);
 // Kernel kinds of one step (per-launch profiling labels).
 enum KernelKind {
   KK_EMBED = 0, KK_GEMM_COND, KK_GEMM_MOD, KK_IN_PROJ, KK_NORM, KK_GEMM_QKV, KK_ATTENTION, KK_GEMM_O,
-  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COUNT
+  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_COUNT
 };
 const char* kernel_kind_name(int k);
 
@@ -89,10 +96,17 @@ struct LaunchTrace {
 // the shapes allow, SIMT otherwise).
 cudaError_t run_gemm(const StepPlan& p, const GemmArgs& g, cudaStream_t st);
 
+// One pass of the full-horizon (synchronous) denoising: every slot at flow
+// time t_now, Euler step t_now - t_next, no release / shift / append.
+struct DenoisePass {
+  float t_now, t_next;
+};
+
 // Enqueue one rolling step for `B` robots on `st` (no synchronisation, graph
 // capture safe when trace == nullptr).  *n_kernels receives the number of
-// kernel launches.
+// kernel launches.  With `dn`, the same expert pass ends in the synchronous
+// denoising update instead of the rolling tail.
 cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_t st, int* n_kernels,
-                         LaunchTrace* trace = nullptr);
+                         LaunchTrace* trace = nullptr, const DenoisePass* dn = nullptr);
 
 }  // namespace ravel

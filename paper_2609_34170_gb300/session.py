@@ -34,6 +34,7 @@ class RollingSession:
         Bn, H, A = len(seeds), self.cfg.slots, self.cfg.action_dim
         self.batch = Bn
         self.buffer = t.empty((Bn, H, A), device=self.device, dtype=t.float32)
+        self.chunk = t.empty((Bn, H, A), device=self.device, dtype=t.float32)
         self.released = t.empty((Bn, A), device=self.device, dtype=t.float32)
         self.velocity = t.empty((Bn, H, A), device=self.device, dtype=t.float32)
         # persistent step inputs: the step graph is captured on their addresses
@@ -57,6 +58,19 @@ class RollingSession:
         B.ravel_roll_step(self.handle, self.buffer, self.slot_times, self.obs if self.cfg.fop_tokens else None,
                           self.delta, self.released, self.velocity if want_velocity else None, stream)
         return self.released
+
+    def denoise_chunk(self, n_steps: int, obs, delta, want_velocity: bool = False, stream=None):
+        """Full-horizon denoising of a fresh chunk (the paper's synchronous
+        baseline): returns the [B, H, A] chunk tensor (t = 0)."""
+        t = self.torch
+        if not hasattr(self, "chunk"):
+            self.chunk = t.empty_like(self.buffer)
+        if self.cfg.fop_tokens:
+            self.obs.copy_(self.to_dev(obs))
+        self.delta.copy_(self.to_dev(delta, t.float32))
+        B.ravel_denoise_chunk(self.handle, self.chunk, n_steps, self.obs if self.cfg.fop_tokens else None, self.delta,
+                              self.velocity if want_velocity else None, stream)
+        return self.chunk
 
     def counters(self) -> np.ndarray:
         return B.ravel_get_state(self.handle, self.batch)
