@@ -272,7 +272,7 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
       for (int q = 0; q < 8; ++q) {
         const int ng = tile_n * TC_BM + fg * 8 + q;   // gate row; its up row is ng + 64
         const float bg = p.bias ? p.bias[ng] : 0.f, bu = p.bias ? p.bias[ng + 64] : 0.f;
-        o[q] = gelu_tanh_f(srow[fg * 8 + q] + bg) * (srow[64 + fg * 8 + q] + bu);
+        o[q] = gelu_tanh_bf16out(srow[fg * 8 + q] + bg) * (srow[64 + fg * 8 + q] + bu);
       }
       bf16* dst = (bf16*)p.out + (size_t)m * p.ldo + f0;
       if (f0 + 8 <= nf && ((uintptr_t)dst & 15) == 0) {
@@ -384,10 +384,10 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
         const float4* u4 = (const float4*)(xch + c * STG_LD + 64 + fg * 8);
         const float4 ga = g4[0], gb = g4[1], ua = u4[0], ub = u4[1];
         *(uint4*)((bf16*)box + c * 64 + fg * 8) =
-            make_uint4(pack_bf16x2(gelu_tanh_f(ga.x) * ua.x, gelu_tanh_f(ga.y) * ua.y),
-                       pack_bf16x2(gelu_tanh_f(ga.z) * ua.z, gelu_tanh_f(ga.w) * ua.w),
-                       pack_bf16x2(gelu_tanh_f(gb.x) * ub.x, gelu_tanh_f(gb.y) * ub.y),
-                       pack_bf16x2(gelu_tanh_f(gb.z) * ub.z, gelu_tanh_f(gb.w) * ub.w));
+            make_uint4(pack_bf16x2(gelu_tanh_bf16out(ga.x) * ua.x, gelu_tanh_bf16out(ga.y) * ua.y),
+                       pack_bf16x2(gelu_tanh_bf16out(ga.z) * ua.z, gelu_tanh_bf16out(ga.w) * ua.w),
+                       pack_bf16x2(gelu_tanh_bf16out(gb.x) * ub.x, gelu_tanh_bf16out(gb.y) * ub.y),
+                       pack_bf16x2(gelu_tanh_bf16out(gb.z) * ub.z, gelu_tanh_bf16out(gb.w) * ub.w));
       }
     }
   } else if (kind == EK_BF16) {
@@ -508,6 +508,11 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     if (TMA_OUT) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
+  }
+  // A launch that may be skipped at run time (p.skip) issues nothing before
+  // it has read its flag after the wait; every other launch streams its first
+  // weight tiles now, while the previous kernel is still finishing.
+  auto issue_weight_prologue = [&]() {
     if (p.oneshot) {
       // every weight k-tile of this CTA in one box; the token k-tiles follow
       // after the wait into the same barrier
@@ -525,27 +530,15 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       if (p.splits > 1)
         for (int kb = kb0_first + npre; kb < kb1_first; ++kb) prefetch_l2_2d(&tmW, kb * TC_BK, tn0 * TC_BM);
     }
-  }
+  };
+  if (threadIdx.x == 0 && !p.skip) issue_weight_prologue();
   // everything below may read what earlier kernels wrote; TMEM is taken only
   // now, so a CTA waiting here never holds columns its predecessor needs
   pdl_wait();
-  if (p.skip && *p.skip) {
-    // nothing to compute (the flag is the same for every CTA): the token
-    // tiles of the stages loaded before the wait are fetched as well, so that
-    // each barrier completes as armed, and the CTA leaves once they landed
-    if (threadIdx.x == 0 && has_work) {
-      if (p.oneshot) {
-        tma_load_3d(&tmX, &full[0], b_s, 0, tm0 * BN, kb0_first, pol_x);
-        if (!mbar_wait(&full[0], 0)) raise_error(p.err, ERR_TIMEOUT);
-      } else {
-        for (int i = 0; i < npre; ++i)
-          tma_load_2d(&tmX, &full[i], b_s + (size_t)i * b_bytes, (kb0_first + i) * TC_BK, tm0 * BN, pol_x);
-        for (int i = 0; i < npre; ++i)
-          if (!mbar_wait(&full[i], 0)) raise_error(p.err, ERR_TIMEOUT);
-      }
-    }
-    cta_sync();
-    return;
+  if (p.skip) {
+    // nothing is in flight yet; the flag is the same for every CTA
+    if (*p.skip) return;
+    if (threadIdx.x == 0) issue_weight_prologue();
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -969,28 +962,23 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"(&tmO) : "memory");
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol_w));
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol_x));
-    // the first stages' weight halves, before the wait on the previous kernel
+  }
+  // the first stages' weight halves, before the wait on the previous kernel
+  // (after it, for a launch that may be skipped at run time)
+  auto issue_weight_prologue = [&]() {
     for (int i = 0; i < npre; ++i) {
       if (leader) mbar_expect_tx(&full[i], stage_tx);
       tma_load_2d_pair(&tmW, full0 + 8u * (uint32_t)i, a_s + (size_t)i * TC_A_BYTES, i * TC_BK,
                        (2 * tn0 + (int)rank) * TC_BM, pol_w);
     }
-  }
+  };
+  if (threadIdx.x == 0 && !p.skip) issue_weight_prologue();
   pdl_wait();
-  if (p.skip && *p.skip) {
-    // nothing to compute: both CTAs fetch the token halves of the stages
-    // loaded before the wait (completing on the even CTA's barriers), the even
-    // CTA waits for them, and neither leaves before the other
-    if (threadIdx.x == 0) {
-      for (int i = 0; i < npre; ++i)
-        tma_load_2d_pair(&tmX, full0 + 8u * (uint32_t)i, b_s + (size_t)i * bh_bytes, i * TC_BK,
-                         tm0 * BN + (int)rank * BNh, pol_x);
-      if (leader)
-        for (int i = 0; i < npre; ++i)
-          if (!mbar_wait(&full[i], 0)) raise_error(p.err, ERR_TIMEOUT);
-    }
-    cluster_sync();
-    return;
+  if (p.skip) {
+    // nothing has been issued yet and the flag is the same for both CTAs of
+    // the pair: they leave together, with no copy or arrival in flight
+    if (*p.skip) return;
+    if (threadIdx.x == 0) issue_weight_prologue();
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
