@@ -199,13 +199,58 @@ def euler_roll(buffer, velocity, slot_times, seeds, counters):
     return released, new, counters + np.uint64(1)
 
 
+def to_relative(buffer, slot_times, state, rel_mask):
+    """Absolute buffer -> the expert's relative coordinates (App. "LIBERO and
+    RoboTwin 2.0": absolute targets are stored, and converted to actions
+    relative to the latest robot state before each expert update; the paired
+    noise stays in model coordinates).  A slot at flow time t holds
+    a = t eps + (1 - t) a_hat, so expressing a_hat relative to the state s
+    moves it by -(1 - t) s on the relative dimensions (rel_mask = 1)."""
+    shift = (1.0 - _f64(slot_times))[None, :, None] * (_f64(rel_mask)[None, None, :] * _f64(state)[:, None, :])
+    return _f64(buffer) - shift
+
+
+def to_absolute(buffer_rel, slot_times, state, rel_mask):
+    """The inverse of to_relative at the given flow times."""
+    shift = (1.0 - _f64(slot_times))[None, :, None] * (_f64(rel_mask)[None, None, :] * _f64(state)[:, None, :])
+    return _f64(buffer_rel) + shift
+
+
 def roll_step(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, seeds, counters,
-              mask: str = "full"):
+              mask: str = "full", state=None, rel_mask=None):
     """One rolling action-expert step.  Returns (released, new buffer, new
-    counters, velocity)."""
-    v = expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, mask)
-    released, new, counters = euler_roll(buffer, v, slot_times, seeds, counters)
-    return released, new, counters, v
+    counters, velocity).
+
+    With ``state`` [B, A] and ``rel_mask`` [A] (1 = a dimension the expert
+    predicts relative to the robot state, 0 = absolute, e.g. a gripper), the
+    buffer holds absolute coordinates: it is converted to relative ones at the
+    slots' times, the expert and the Euler update act there, and every slot is
+    converted back at its new time t_{j-1} (the released slot at t = 0 becomes
+    its absolute target).  The appended noise slot (t = 1) needs no shift."""
+    if state is None:
+        v = expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, mask)
+        released, new, counters = euler_roll(buffer, v, slot_times, seeds, counters)
+        return released, new, counters, v
+    rel = to_relative(buffer, slot_times, state, rel_mask)
+    v = expert_velocity(cfg, W, rel, slot_times, ctx_k, ctx_v, prefix_len, fop, delta, mask)
+    return (*roll_relative(rel, v, slot_times, seeds, counters, state, rel_mask), v)
+
+
+def roll_relative(rel, velocity, slot_times, seeds, counters, state, rel_mask):
+    """Eq. 3 in relative coordinates, then each slot back to absolute ones at
+    its new time (slot j moves from t_j to t_{j-1}, t_{-1} = 0), then the
+    release / shift / append.  Returns (released, new buffer, new counters)."""
+    t = _f64(slot_times)
+    t_new = np.concatenate([[0.0], t[:-1]])
+    a_rel = _f64(rel) + slot_dt(slot_times)[None, :, None] * _f64(velocity)
+    a = to_absolute(a_rel, t_new, state, rel_mask)
+    B, H, A = a.shape
+    released = a[:, 0].copy()
+    counters = np.asarray(counters, dtype=np.uint64)
+    fresh = np.stack([action_noise(int(seeds[b]), counters[b], A) for b in range(B)]) \
+        if B else np.zeros((0, A), np.float32)
+    new = np.concatenate([a[:, 1:], _f64(fresh)[:, None, :]], axis=1)
+    return released, new, counters + np.uint64(1)
 
 
 def denoise_chunk(cfg, W, seeds, counters, n_steps: int, ctx_k, ctx_v, prefix_len, fop, delta,

@@ -431,3 +431,60 @@ def test_denoise_chunk_one_step_is_one_expert_pass_at_t1():
                    for b in range(cfg.batch)]).astype(np.float64)
     vel = expert.expert_velocity(cfg, W, a0, np.ones(cfg.slots, np.float32), k, v, P, z, d)
     np.testing.assert_allclose(chunk, a0 + vel, rtol=1e-12, atol=1e-14)
+
+
+# ----------------------------------------------------------------------------- relative <-> absolute buffer
+
+
+def test_relative_coordinates_keep_absolute_targets_while_the_state_moves():
+    # The expert predicts relative to the latest robot state (App. "LIBERO and
+    # RoboTwin 2.0"); the buffer stores absolute targets.  With the ideal
+    # single-target field written in relative coordinates -- the target
+    # relative to THIS step's state -- every released action must be its
+    # absolute target, although the state changes at every step; the gripper
+    # dimension (rel_mask 0) is absolute throughout.
+    cfg = TINY.replace(batch=2, slots=6, action_dim=4)
+    H = cfg.slots
+    t = synth.staggered_times(H).astype(np.float64)
+    rng = np.random.default_rng(11)
+    steps = 4 * H
+    targets = rng.standard_normal((steps + H, 2, 4))       # absolute targets of action n
+    states = rng.standard_normal((steps, 2, 4)) * 3.0       # a different robot state every step
+    rel_mask = np.array([1.0, 1.0, 1.0, 0.0])
+    seeds = synth.robot_seeds(31, 2)
+    buf, cnt = expert.reset(cfg, seeds)
+    buf = buf.astype(np.float64)
+    out = []
+    for s in range(steps):
+        rel = expert.to_relative(buf, t.astype(np.float32), states[s], rel_mask)
+        tgt_rel = np.stack([targets[s + j] for j in range(H)], axis=1) - rel_mask * states[s][:, None, :]
+        v = (tgt_rel - rel) / t[None, :, None]
+        released, buf, cnt = expert.roll_relative(rel, v, t.astype(np.float32), seeds, cnt, states[s], rel_mask)
+        out.append(released)
+    np.testing.assert_allclose(np.array(out), targets[:steps], rtol=0, atol=1e-10)
+    # ... while keeping the stored targets relative (no conversion) breaks it
+    buf, cnt = expert.reset(cfg, seeds)
+    buf = buf.astype(np.float64)
+    for s in range(H + 2):
+        tgt_rel = np.stack([targets[s + j] for j in range(H)], axis=1) - rel_mask * states[s][:, None, :]
+        released, buf, cnt = expert.euler_roll(buf, (tgt_rel - buf) / t[None, :, None], t.astype(np.float32), seeds, cnt)
+    assert np.max(np.abs(released - targets[H + 1])) > 0.1
+
+
+def test_relative_step_with_zero_mask_is_the_absolute_step():
+    cfg = TINY
+    W, buf, t, k, v, P, z, d, cnt = _inputs(cfg)
+    seeds = synth.robot_seeds(7, cfg.batch)
+    state = np.random.default_rng(2).standard_normal((cfg.batch, cfg.action_dim))
+    a = expert.roll_step(cfg, W, buf, t, k, v, P, z, d, seeds, cnt)
+    b = expert.roll_step(cfg, W, buf, t, k, v, P, z, d, seeds, cnt, state=state, rel_mask=np.zeros(cfg.action_dim))
+    for x, y in zip(a, b):
+        np.testing.assert_allclose(np.asarray(x, np.float64), np.asarray(y, np.float64), rtol=1e-13, atol=1e-14)
+    # with a mask, the expert sees the buffer shifted by (1 - t_j) s on those dimensions
+    m = np.array([1.0] * (cfg.action_dim - 1) + [0.0])
+    rel, new, _, vel = expert.roll_step(cfg, W, buf, t, k, v, P, z, d, seeds, cnt, state=state, rel_mask=m)
+    want_v = expert.expert_velocity(cfg, W, buf - (1 - t.astype(np.float64))[None, :, None] * (m * state)[:, None, :],
+                                    t, k, v, P, z, d)
+    np.testing.assert_allclose(vel, want_v, rtol=1e-12, atol=1e-14)
+    # slot 0 moves from t_0 to 0: a' = a + dt (v + m s), dt = t_0
+    np.testing.assert_allclose(rel, buf[:, 0] + t[0] * (vel[:, 0] + m * state), rtol=1e-12, atol=1e-13)
