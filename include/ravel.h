@@ -150,6 +150,31 @@ ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int pre
 ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
                              const float* delta, float* released, float* velocity, void* stream);
 
+/* The rolling step for an expert that predicts actions relative to the robot
+ * state while the buffer keeps absolute targets (App. "LIBERO and RoboTwin
+ * 2.0": absolute targets are stored, converted to actions relative to the
+ * latest state before each expert update and back afterwards; the paired
+ * noise stays in model coordinates).  Same arguments and effects as
+ * ravel_roll_step, plus
+ *   state   device float32 [B, A]: the latest robot state in the action
+ *           coordinates (non-null)
+ * A slot at flow time t holds a = t eps + (1 - t) a_hat, so on the relative
+ * dimensions (ravel_set_relative_dims) the expert sees a - (1 - t_j) state,
+ * the Euler step happens there, and each slot returns to absolute
+ * coordinates at its new time t_{j-1}: a' = a + dt_j (v_j + mask * state).
+ * The released slot (t = 0) is an absolute action; the appended slot is pure
+ * noise (t = 1) and needs no shift.  With h > 1 actions per slot
+ * (action_dim = h * the robot's action size) the mask repeats per action. */
+ravel_status ravel_roll_step_rel(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                                 const float* delta, const float* state, float* released, float* velocity,
+                                 void* stream);
+
+/* Which action dimensions the expert predicts relative to the robot state:
+ * mask host float32 [A], 1 = relative (for example joint or pose targets),
+ * 0 = absolute (for example a gripper command).  A new handle has none.
+ * Synchronous. */
+ravel_status ravel_set_relative_dims(ravel_t* r, const float* mask);
+
 /* The full-horizon (synchronous) denoising that the paper compares rolling
  * inference with (Experiments, synchronous simulation: ten full-horizon
  * denoising steps per policy query; Table 1): every robot draws a fresh chunk

@@ -66,6 +66,8 @@ def load(path: str | None = None):
         "ravel_set_context": (i, [vp, vp, vp, i, vp]),
         "ravel_roll_step": (i, [vp, vp, vp, vp, vp, vp, vp, vp]),
         "ravel_denoise_chunk": (i, [vp, vp, i, vp, vp, vp, vp]),
+        "ravel_roll_step_rel": (i, [vp, vp, vp, vp, vp, vp, vp, vp, vp]),
+        "ravel_set_relative_dims": (i, [vp, vp]),
         "ravel_get_state": (i, [vp, vp]),
         "ravel_set_state": (i, [vp, vp]),
         "ravel_step_kernel_count": (i, [vp]),
@@ -165,6 +167,20 @@ def ravel_roll_step(h, buffer, slot_times, obs_tokens, delta, released, velocity
         h, _dptr(buffer, f32, "buffer"), _dptr(slot_times, f32, "slot_times"), _dptr(obs_tokens, name="obs_tokens"),
         _dptr(delta, f32, "delta"), _dptr(released, f32, "released"), _dptr(velocity, f32, "velocity"),
         _stream_ptr(stream)), "ravel_roll_step")
+
+
+def ravel_roll_step_rel(h, buffer, slot_times, obs_tokens, delta, state, released, velocity=None, stream=None):
+    import torch
+    f32 = torch.float32
+    _check(h, load().ravel_roll_step_rel(
+        h, _dptr(buffer, f32, "buffer"), _dptr(slot_times, f32, "slot_times"), _dptr(obs_tokens, name="obs_tokens"),
+        _dptr(delta, f32, "delta"), _dptr(state, f32, "state"), _dptr(released, f32, "released"),
+        _dptr(velocity, f32, "velocity"), _stream_ptr(stream)), "ravel_roll_step_rel")
+
+
+def ravel_set_relative_dims(h, mask):
+    m = np.ascontiguousarray(mask, dtype=np.float32)
+    _check(h, load().ravel_set_relative_dims(h, m.ctypes.data), "ravel_set_relative_dims")
 
 
 def ravel_denoise_chunk(h, chunk, n_steps: int, obs_tokens, delta, velocity=None, stream=None):

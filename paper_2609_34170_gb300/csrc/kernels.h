@@ -119,8 +119,11 @@ struct NormArgs {
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 
 // ---- action in-projection: x[b*H+j][c] = sum_a buf[b][j][a] in_w[a][c] + in_b[c] ----
+// With `state` ([B][A], or null) the buffer holds absolute coordinates and
+// the expert sees a - (1 - t_j) rel_mask * state_b (the relative ones).
 cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b,
-                           float* x, cudaStream_t st);
+                           float* x, cudaStream_t st, const float* state = nullptr, const float* rel_mask = nullptr,
+                           const float* slot_times = nullptr, int H = 1);
 
 // ---- GeGLU on the interleaved gate/up GEMM output --------------------------------
 cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cudaStream_t st);
@@ -170,6 +173,8 @@ struct TailArgs {
   const uint64_t* seeds;     // [B]
   uint64_t* counters;        // [B], advanced by one
   int B, H, A;
+  const float* state = nullptr;      // optional [B][A]: absolute buffer, relative expert (see launch_in_proj):
+  const float* rel_mask = nullptr;   // [A]; a' = a + dt (v + rel_mask * state)
 };
 cudaError_t launch_tail(const TailArgs& a, cudaStream_t st);
 

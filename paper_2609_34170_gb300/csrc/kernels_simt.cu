@@ -469,12 +469,20 @@ cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st) {
 // ============================================================================ in-proj
 
 __global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, const float* __restrict__ in_w,
-                               const float* __restrict__ in_b, float* __restrict__ x) {
+                               const float* __restrict__ in_b, float* __restrict__ x, const float* __restrict__ state,
+                               const float* __restrict__ rel_mask, const float* __restrict__ slot_times, int H) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ float arow[];   // the action row of this slot
   const int r = blockIdx.y;
-  for (int i = threadIdx.x; i < A; i += blockDim.x) arow[i] = buf[(size_t)r * A + i];
+  for (int i = threadIdx.x; i < A; i += blockDim.x) {
+    float a = buf[(size_t)r * A + i];
+    if (state) {   // relative coordinates of the expert: a - (1 - t_j) m s_b
+      const int b = r / H, j = r % H;
+      a = __fsub_rn(a, __fmul_rn(__fsub_rn(1.f, slot_times[j]), __fmul_rn(rel_mask[i], state[(size_t)b * A + i])));
+    }
+    arow[i] = a;
+  }
   __syncthreads();
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= D) return;
@@ -484,10 +492,10 @@ __global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, cons
 }
 
 cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b, float* x,
-                           cudaStream_t st) {
+                           cudaStream_t st, const float* state, const float* rel_mask, const float* slot_times, int H) {
   if (BH <= 0) return cudaSuccess;
   return launch_kernel(in_proj_kernel, dim3((D + 255) / 256, BH), dim3(256), A * sizeof(float), st, 1, buf, A, D,
-                       in_w, in_b, x);
+                       in_w, in_b, x, state, rel_mask, slot_times, H);
 }
 
 // ============================================================================ GeGLU
@@ -670,7 +678,10 @@ __global__ void tail_kernel(TailArgs a) {
     const float t1 = a.slot_times[j];
     const float t0 = j ? a.slot_times[j - 1] : 0.f;
     const float dt = __fsub_rn(t1, t0);
-    sa[i] = fmaf(dt, v[i], buf[i]);
+    // absolute buffer, relative expert: the slot also moves by dt m s as its
+    // flow time drops from t_j to t_{j-1}
+    const float vv = a.state ? fmaf(a.rel_mask[i % A], a.state[(size_t)b * A + i % A], v[i]) : v[i];
+    sa[i] = fmaf(dt, vv, buf[i]);
     if (a.vel_out) a.vel_out[(size_t)b * H * A + i] = v[i];
   }
   __syncthreads();

@@ -224,8 +224,9 @@ static ravel_status apply_pending_swap(ravel_t* r, cudaStream_t st) {
   return RAVEL_OK;
 }
 
-ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
-                             const float* delta, float* released, float* velocity, void* stream) {
+static ravel_status roll_step_impl(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                                   const float* delta, const float* state, float* released, float* velocity,
+                                   void* stream) {
   if (!r || !buffer || !slot_times || !delta || !released) return fail(r, RAVEL_EINVAL, "roll_step: null argument");
   if (r->plan.cfg.fop_tokens > 0 && !obs_tokens) return fail(r, RAVEL_EINVAL, "roll_step: obs_tokens is null");
   if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "roll_step: call ravel_reset first");
@@ -236,7 +237,7 @@ ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times,
   cudaStream_t st = (cudaStream_t)stream;
   s = apply_pending_swap(r, st);
   if (s != RAVEL_OK) return s;
-  StepIO io{buffer, slot_times, obs_tokens, delta, released, velocity};
+  StepIO io{buffer, slot_times, obs_tokens, delta, released, velocity, state};
   if (!r->gexec || r->graph_batch != r->batch || memcmp(&io, &r->graph_io, sizeof io) != 0) {
     if (r->gexec) {
       RV_CUDA(r, cudaStreamSynchronize(st), "roll_step: sync before re-capture");
@@ -264,6 +265,27 @@ ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times,
   RV_CUDA(r, cudaEventRecord(r->ev_step_done, st), "record step");
   RV_CUDA(r, cudaMemcpyAsync(r->err_host, r->plan.err, sizeof(int), cudaMemcpyDeviceToHost, st), "error mirror");
   r->any_step = true;
+  return RAVEL_OK;
+}
+
+ravel_status ravel_roll_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                             const float* delta, float* released, float* velocity, void* stream) {
+  return roll_step_impl(r, buffer, slot_times, obs_tokens, delta, nullptr, released, velocity, stream);
+}
+
+ravel_status ravel_roll_step_rel(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
+                                 const float* delta, const float* state, float* released, float* velocity,
+                                 void* stream) {
+  if (!state) return fail(r, RAVEL_EINVAL, "roll_step_rel: state is null");
+  return roll_step_impl(r, buffer, slot_times, obs_tokens, delta, state, released, velocity, stream);
+}
+
+ravel_status ravel_set_relative_dims(ravel_t* r, const float* mask) {
+  if (!r || !mask) return fail(r, RAVEL_EINVAL, "set_relative_dims: null argument");
+  RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
+  RV_CUDA(r, cudaDeviceSynchronize(), "set_relative_dims: sync");
+  RV_CUDA(r, cudaMemcpy(r->plan.rel_mask, mask, sizeof(float) * r->plan.cfg.action_dim, cudaMemcpyHostToDevice),
+          "set_relative_dims: copy");
   return RAVEL_OK;
 }
 

@@ -142,6 +142,7 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->tcws.ws, p->tcws.ws_bytes);
   AL(p->tcws.counters, p->tcws.n_counters * sizeof(int));
   AL(p->dn_times, (size_t)H * sizeof(float));
+  AL(p->rel_mask, (size_t)A * sizeof(float));
   AL(p->seeds, Bm * sizeof(uint64_t));
   AL(p->counters, Bm * sizeof(uint64_t));
   AL(p->err, sizeof(int));
@@ -297,7 +298,8 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   RUN(KK_GEMM_MOD, gemm(p.HC, D, p.mod_w, H + B, p.mod_dim, D, EPI_STORE, p.modv, p.mod_dim, DT_F32, nullptr, 0, skip));
   RUN(KK_COND_CACHE, launch_cond_commit(ca, st));
   // residual stream
-  RUN(KK_IN_PROJ, launch_in_proj(io.buffer, B * H, A, D, p.in_w, p.in_b, p.x, st));
+  RUN(KK_IN_PROJ, launch_in_proj(io.buffer, B * H, A, D, p.in_w, p.in_b, p.x, st, io.state, p.rel_mask, io.slot_times,
+                                 H));
   const int FF = io.obs ? F : 0;      // FOP tokens present in this step
   const int RPR = H + FF;              // normed / QKV rows per robot: H slots, then the FOP tokens
   const int BH = B * H, BY = B * RPR;
@@ -330,8 +332,8 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
                   c.max_prefix, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim, c.mask_mode, p.O, p.qdim, p.err};
       RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
     }
-    RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x, D,
-             DT_F32, nullptr, p.split_cap[1]));
+    RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x,
+                        D, DT_F32, nullptr, p.split_cap[1]));
     NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
     RUN(KK_NORM, launch_ada_norm(n2, dt, st));
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
@@ -352,7 +354,8 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   if (dn) {
     RUN(KK_TAIL, launch_denoise_tail(io.buffer, p.V, io.velocity, B, H, A, dn->t_now, dn->t_next, st));
   } else {
-    TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A};
+    TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A, io.state,
+                p.rel_mask};
     RUN(KK_TAIL, launch_tail(ta, st));
   }
 #undef RUN

@@ -20,6 +20,7 @@ struct StepIO {
   const float* delta;
   float* released;
   float* velocity;
+  const float* state = nullptr;   // [B][A] latest robot state: absolute buffer, relative expert
 };
 
 struct StepPlan {
@@ -69,6 +70,7 @@ struct StepPlan {
   int num_sms = 0;
   bool use_tc = false;      // bf16 projections on tcgen05
   float* dn_times = nullptr;   // [H] flow times of a synchronous denoising pass (all equal)
+  float* rel_mask = nullptr;   // [A] 1 = a dimension the expert predicts relative to the robot state
   uint64_t* seeds = nullptr;
   uint64_t* counters = nullptr;
   int* err = nullptr;

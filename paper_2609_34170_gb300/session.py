@@ -49,15 +49,30 @@ class RollingSession:
         self._ctx = (k, v)   # keep alive until the side-stream copy has run
         B.ravel_set_context(self.handle, k, v, int(prefix_len or k.shape[3]), side_stream)
 
-    def step(self, slot_times, obs, delta, want_velocity: bool = False, stream=None):
+    def step(self, slot_times, obs, delta, want_velocity: bool = False, stream=None, state=None):
+        """One rolling step; with `state` ([B, A]) the buffer holds absolute
+        targets and the expert works relative to that state (see
+        ravel_roll_step_rel and set_relative_dims)."""
         t = self.torch
         self.slot_times.copy_(self.to_dev(slot_times, t.float32))
         if self.cfg.fop_tokens:
             self.obs.copy_(self.to_dev(obs))
         self.delta.copy_(self.to_dev(delta, t.float32))
-        B.ravel_roll_step(self.handle, self.buffer, self.slot_times, self.obs if self.cfg.fop_tokens else None,
-                          self.delta, self.released, self.velocity if want_velocity else None, stream)
+        obs_arg = self.obs if self.cfg.fop_tokens else None
+        vel_arg = self.velocity if want_velocity else None
+        if state is None:
+            B.ravel_roll_step(self.handle, self.buffer, self.slot_times, obs_arg, self.delta, self.released, vel_arg,
+                              stream)
+        else:
+            if not hasattr(self, "state"):
+                self.state = t.zeros((self.batch, self.cfg.action_dim), device=self.device, dtype=t.float32)
+            self.state.copy_(self.to_dev(state, t.float32))
+            B.ravel_roll_step_rel(self.handle, self.buffer, self.slot_times, obs_arg, self.delta, self.state,
+                                  self.released, vel_arg, stream)
         return self.released
+
+    def set_relative_dims(self, mask):
+        B.ravel_set_relative_dims(self.handle, mask)
 
     def denoise_chunk(self, n_steps: int, obs, delta, want_velocity: bool = False, stream=None):
         """Full-horizon denoising of a fresh chunk (the paper's synchronous
