@@ -115,6 +115,36 @@ def attention(q, k, v, valid=None):
     return p @ v
 
 
+def adapter_of_layer(cfg, layer: int) -> int:
+    """Index of the FOP adapter in ``layer``, or -1: with adapters every k
+    layers, layers k-1, 2k-1, ... carry one."""
+    k = getattr(cfg, "fop_adapter_every", 0)
+    return (layer + 1) // k - 1 if k and (layer + 1) % k == 0 else -1
+
+
+def gated_cross_attention(cfg, W, i, x, fop):
+    """FOP adapter i (Sec. 3.2: the FOP tokens are injected into selected
+    expert layers through gated cross-attention adapters): the action rows
+    attend to the FOP tokens only,
+        q = (RMSNorm(x) (1 + a_gamma_i)) W_q,  [k | v] = (RMSNorm(z) (1 + a_zgamma_i)) W_kv,
+    grouped-query heads as in the self-attention, and the result enters the
+    residual stream through a tanh gate:  tanh(a_gate_i) * attn W_o.
+    Returns that increment [B, H, D]."""
+    B, H, D = x.shape
+    F = fop.shape[1]
+    Hq, Hkv, hd = cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim
+    G = Hq // Hkv
+    q = ((rmsnorm(x) * (1.0 + _f64(W["a_gamma"][i]))) @ _f64(W["a_wq"][i])).reshape(B, H, Hq, hd)
+    kv = (rmsnorm(_f64(fop)) * (1.0 + _f64(W["a_zgamma"][i]))) @ _f64(W["a_wkv"][i])
+    k = kv[..., :Hkv * hd].reshape(B, F, Hkv, hd)
+    v = kv[..., Hkv * hd:].reshape(B, F, Hkv, hd)
+    o = np.empty((B, H, Hq, hd))
+    for b in range(B):
+        for h in range(Hq):
+            o[b, :, h] = attention(q[b, :, h], k[b, :, h // G], v[b, :, h // G])
+    return np.tanh(float(W["a_gate"][i])) * (o.reshape(B, H, Hq * hd) @ _f64(W["a_wo"][i]))
+
+
 def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, delta,
                     mask: str = "full", trace: dict | None = None):
     """v_theta(A, t, c, delta) for B robots: [B, H, A] float64 (Eq. 3's velocity).
@@ -126,7 +156,8 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
     D, L = cfg.width, cfg.layers
     Hq, Hkv, hd = cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim
     G = Hq // Hkv
-    F = fop.shape[1]
+    adapters = getattr(cfg, "fop_adapter_every", 0) > 0
+    F = 0 if adapters else fop.shape[1]   # FOP keys of the self-attention
     P = int(prefix_len)
 
     cond = conditioning(cfg, W, _f64(slot_times), _f64(delta))
@@ -145,7 +176,7 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
         wqkv = _f64(W["w_qkv"][l])
         sc, sh = mod_slice(cfg, mod, l, 0)
         y = ada_rmsnorm(x, sc, sh)                                  # [B, H, D]
-        yf = zn * (1.0 + _f64(W["fop_gamma"][l]))                  # [B, F, D]
+        yf = (zn * (1.0 + _f64(W["fop_gamma"][l])))[:, :F]         # [B, F, D]
         qkv = y @ wqkv                                              # [B, H, NQKV]
         kvf = yf @ wqkv[:, Hq * hd:]                                # [B, F, 2 Hkv hd]
         q = qkv[..., :Hq * hd].reshape(B, H, Hq, hd)
@@ -161,6 +192,8 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
                 for h in range(g * G, (g + 1) * G):
                     o[b, :, h] = attention(q[b, :, h], keys, vals, valid)
         x = x + o.reshape(B, H, Hq * hd) @ _f64(W["w_o"][l])
+        if adapter_of_layer(cfg, l) >= 0:
+            x = x + gated_cross_attention(cfg, W, adapter_of_layer(cfg, l), x, fop)
         sc2, sh2 = mod_slice(cfg, mod, l, 1)
         y2 = ada_rmsnorm(x, sc2, sh2)
         hmid = gelu_tanh(y2 @ _f64(W["w_gate"][l])) * (y2 @ _f64(W["w_up"][l]))

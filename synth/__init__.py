@@ -52,6 +52,14 @@ class ExpertConfig:
     fop_tokens: int
     batch: int
     dtype: str  # "fp32" or "bf16"
+    # 0: FOP tokens are extra keys / values of every layer's self-attention;
+    # k > 0: they enter layers k-1, 2k-1, ... through gated cross-attention
+    # adapters instead (and are not keys of the self-attention)
+    fop_adapter_every: int = 0
+
+    @property
+    def n_adapters(self) -> int:
+        return self.layers // self.fop_adapter_every if self.fop_adapter_every else 0
 
     @property
     def n_qkv(self) -> int:
@@ -136,6 +144,10 @@ def weight_names(cfg: ExpertConfig) -> dict[str, tuple[int, ...]]:
         "w_up": (L, D, cfg.mlp_dim),
         "w_down": (L, cfg.mlp_dim, D),
         "out_w": (D, A), "out_b": (A,),
+        **({} if not cfg.n_adapters else {
+            "a_gamma": (cfg.n_adapters, D), "a_zgamma": (cfg.n_adapters, D),
+            "a_wq": (cfg.n_adapters, D, cfg.q_dim), "a_wkv": (cfg.n_adapters, D, 2 * cfg.n_kv_heads * cfg.head_dim),
+            "a_wo": (cfg.n_adapters, cfg.q_dim, D), "a_gate": (cfg.n_adapters,)}),
     }
 
 

@@ -488,3 +488,56 @@ def test_relative_step_with_zero_mask_is_the_absolute_step():
     np.testing.assert_allclose(vel, want_v, rtol=1e-12, atol=1e-14)
     # slot 0 moves from t_0 to 0: a' = a + dt (v + m s), dt = t_0
     np.testing.assert_allclose(rel, buf[:, 0] + t[0] * (vel[:, 0] + m * state), rtol=1e-12, atol=1e-13)
+
+
+# ----------------------------------------------------------------------------- gated cross-attention FOP adapters
+
+
+ADAPT = TINY.replace(layers=4, fop_adapter_every=2)      # adapters in layers 1 and 3
+
+
+def test_adapter_with_closed_gates_is_the_network_without_fop():
+    # tanh(0) = 0: every adapter adds nothing, and in adapter mode the FOP
+    # tokens are no keys of the self-attention -- so the expert is the one
+    # that never sees them
+    W, buf, t, k, v, P, z, d, _ = _inputs(ADAPT)
+    W0 = dict(W, a_gate=np.zeros_like(W["a_gate"]))
+    a = expert.expert_velocity(ADAPT, W0, buf, t, k, v, P, z, d)
+    nofop = ADAPT.replace(fop_adapter_every=0, fop_tokens=0)
+    Wn = {n: W[n] for n in synth.weight_names(nofop)}
+    b = expert.expert_velocity(nofop, Wn, buf, t, k, v, P, z[:, :0], d)
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-14)
+    # open gates change the result, and do not depend on the order of the FOP tokens
+    W1 = dict(W, a_gate=np.full_like(W["a_gate"], 0.8))
+    c = expert.expert_velocity(ADAPT, W1, buf, t, k, v, P, z, d)
+    assert np.max(np.abs(c - a)) > 1e-4
+    perm = np.random.default_rng(1).permutation(ADAPT.fop_tokens)
+    np.testing.assert_allclose(expert.expert_velocity(ADAPT, W1, buf, t, k, v, P, z[:, perm], d), c,
+                               rtol=1e-11, atol=1e-13)
+
+
+def test_adapter_closed_form_one_layer():
+    # one layer with its adapter; W_q^a = 0 makes the cross-attention uniform
+    # over the F FOP tokens, and zero self-attention / MLP outputs leave
+    #   x1 = x0 + tanh(g) * (mean_f (sqrt(D) z_f / |z_f| (1 + a_zgamma)) W_v^a) W_o^a
+    # per head (|z| ~ 100: eps negligible), written out here from the definition
+    cfg = TINY.replace(layers=1, fop_adapter_every=1)
+    D, Hq, Hkv, hd, F = cfg.width, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.fop_tokens
+    G = Hq // Hkv
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    z = z.astype(np.float64) * 100.0
+    g = 2.0     # tanh(2) = 0.964, unlike sigmoid(2) or 2 itself
+    W1 = dict(W, a_wq=np.zeros_like(W["a_wq"]), w_o=np.zeros_like(W["w_o"]), w_gate=np.zeros_like(W["w_gate"]),
+              a_gate=np.array([g]), a_zgamma=W["a_zgamma"].astype(np.float64) * 20.0)
+    tr = {}
+    expert.expert_velocity(cfg, W1, buf, t, k, v, P, z, d, trace=tr)
+    x0 = buf.astype(np.float64) @ W["in_w"] + W["in_b"]
+    wv = W["a_wkv"][0].astype(np.float64)[:, Hkv * hd:]
+    o = np.zeros((cfg.batch, Hq * hd))
+    for b in range(cfg.batch):
+        yz = np.sqrt(D) * z[b] / np.linalg.norm(z[b], axis=1, keepdims=True) * (1.0 + W1["a_zgamma"][0])
+        vf = yz @ wv
+        for h in range(Hq):
+            o[b, h * hd:(h + 1) * hd] = vf[:, (h // G) * hd:(h // G + 1) * hd].mean(0)
+    want = x0 + np.tanh(g) * (o @ W["a_wo"][0].astype(np.float64))[:, None, :]
+    np.testing.assert_allclose(tr["x"][0], want, rtol=1e-9, atol=1e-9)
