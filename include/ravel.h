@@ -75,6 +75,15 @@ typedef struct {
                        all FOP tokens and all H slots; RAVEL_MASK_SLOT_ISOLATED
                        (a test mode): action query j sees the prefix, the FOP
                        tokens and slot j only */
+  int fop_adapter_every; /* 0: the FOP tokens are extra keys / values of every
+                       layer's self-attention; k in [1, layers]: they are no
+                       keys of the self-attention and enter layers k-1, 2k-1,
+                       ... through gated cross-attention adapters (Sec. 3.2:
+                       "injected into selected action-expert layers through
+                       gated cross-attention adapters"), each after its
+                       layer's self-attention block:
+                       x += tanh(a_gate) MHA(q = RMSNorm(x)(1 + a_gamma) a_wq,
+                       [k | v] = RMSNorm(z)(1 + a_zgamma) a_wkv) a_wo */
 } ravel_config;
 
 /*
@@ -103,6 +112,11 @@ typedef struct {
   const float *w_qkv, *w_o, *w_gate, *w_up, *w_down;
   const float *out_w, *out_b;
   int on_device;
+  /* FOP adapters (cfg.fop_adapter_every > 0; NA = layers / fop_adapter_every
+   * adapters, stacked): a_gamma, a_zgamma [NA, D]; a_wq [NA, D, Hq hd];
+   * a_wkv [NA, D, 2 Hkv hd] (K heads, then V heads); a_wo [NA, Hq hd, D];
+   * a_gate [NA].  NULL when there are no adapters. */
+  const float *a_gamma, *a_zgamma, *a_wq, *a_wkv, *a_wo, *a_gate;
 } ravel_weights;
 
 typedef struct ravel_ctx ravel_t;

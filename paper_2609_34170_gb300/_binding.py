@@ -24,15 +24,19 @@ STATUS = ["RAVEL_OK", "RAVEL_EINVAL", "RAVEL_ESHAPE", "RAVEL_ENOMEM", "RAVEL_ECU
 class RavelConfig(C.Structure):
     _fields_ = [(n, C.c_int) for n in (
         "layers", "width", "n_q_heads", "n_kv_heads", "head_dim", "mlp_dim", "slots", "action_dim",
-        "max_prefix", "fop_tokens", "max_batch", "dtype", "mask_mode")]
+        "max_prefix", "fop_tokens", "max_batch", "dtype", "mask_mode", "fop_adapter_every")]
 
 
 WEIGHT_FIELDS = ("t_w1", "t_b1", "t_w2", "t_b2", "d_w1", "d_b1", "d_w2", "d_b2", "mod_w", "mod_b",
                  "in_w", "in_b", "fop_gamma", "w_qkv", "w_o", "w_gate", "w_up", "w_down", "out_w", "out_b")
 
 
+ADAPTER_FIELDS = ("a_gamma", "a_zgamma", "a_wq", "a_wkv", "a_wo", "a_gate")
+
+
 class RavelWeights(C.Structure):
-    _fields_ = [(n, C.c_void_p) for n in WEIGHT_FIELDS] + [("on_device", C.c_int)]
+    _fields_ = ([(n, C.c_void_p) for n in WEIGHT_FIELDS] + [("on_device", C.c_int)]
+                + [(n, C.c_void_p) for n in ADAPTER_FIELDS])
 
 
 class RavelError(RuntimeError):
@@ -118,11 +122,14 @@ def ravel_create(cfg, weights: dict, device: int = 0, max_batch: int | None = No
     L = load()
     c = RavelConfig(cfg.layers, cfg.width, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.mlp_dim, cfg.slots,
                     cfg.action_dim, max_prefix or cfg.prefix, cfg.fop_tokens, max_batch or cfg.batch,
-                    RAVEL_BF16 if cfg.dtype == "bf16" else RAVEL_FP32, mask_mode)
+                    RAVEL_BF16 if cfg.dtype == "bf16" else RAVEL_FP32, mask_mode,
+                    getattr(cfg, "fop_adapter_every", 0))
     on_dev = None
     keep = []
     w = RavelWeights()
-    for n in WEIGHT_FIELDS:
+    for n in WEIGHT_FIELDS + ADAPTER_FIELDS:
+        if n not in weights:   # adapter tensors of a network without adapters
+            continue
         a = weights[n]
         if isinstance(a, np.ndarray):
             a = np.ascontiguousarray(a, dtype=np.float32)

@@ -115,6 +115,8 @@ struct NormArgs {
   const void* fop; int F; const float* gamma;
   void* Y; int row_pitch;
   const int* drow = nullptr;    // optional: row of modv holding robot b's offset part (default H + b)
+  const float* act_gain = nullptr;   // optional [D]: action rows y = x rsqrt(mean(x^2)+eps) (1 + act_gain),
+                                     // without modulation (the query rows of a FOP adapter)
 };
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 
@@ -162,6 +164,13 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st);
 // bf16 context V [L][B][Hkv][P][hd] -> slot layout Vt [L][Bmax][Hkv][hd][pst]
 cudaError_t launch_transpose_ctx_v(const void* src, void* dst, int L, int B, int Bmax, int Hkv, int P, int hd,
                                    int pst, cudaStream_t st);
+
+// ---- gated cross-attention of a FOP adapter ------------------------------------------
+// out[b*H + j][h*hd + c] = tanh(gate[0]) * sum_f softmax_f(q . k_f / sqrt(hd)) v_f[c] over the
+// F FOP tokens of robot b: q from Q [B*H][Hq*hd], k / v from KV [B*F][2*Hkv*hd] (K heads, then
+// V heads), query head h reading KV head h / (Hq / Hkv).  F <= 64.
+cudaError_t launch_fop_xattn(const void* Q, const void* KV, void* out, int B, int H, int F, int Hq, int Hkv, int hd,
+                             const float* gate, Dtype dt, cudaStream_t st);
 
 // ---- rolling tail: Euler, release, shift, append ------------------------------------
 struct TailArgs {

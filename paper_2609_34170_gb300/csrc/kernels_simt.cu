@@ -342,21 +342,22 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, i
     const int c = 4 * threadIdx.x + 1024 * g;
     csc[g] = csh[g] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (c < D) {   // weights: independent of the earlier kernels
-      if (act) {
+      if (act && !a.act_gain) {
         csc[g] = ld4(a.mod_b + a.off + c);
         csh[g] = ld4(a.mod_b + a.off + D + c);
       } else {
-        csc[g] = ld4(a.gamma + c);
+        csc[g] = ld4(act ? a.act_gain + c : a.gamma + c);
       }
     }
   }
   pdl_wait();
-  const float* md = a.modv + (size_t)(a.drow ? a.drow[b] : a.H + b) * a.mod_ld + a.off;
+  const bool modulated = act && !a.act_gain;   // action rows with adaLN modulation
+  const float* md = modulated ? a.modv + (size_t)(a.drow ? a.drow[b] : a.H + b) * a.mod_ld + a.off : nullptr;
   int buf = 0;
   for (int j = j0; j < j1; j += R, buf ^= 1) {
     float4 xv[R][G], ts[R][G], th[R][G];
     float ss[R];
-    if (act && j == j0) {   // M_delta[b] joins the first batch's loads (one round trip)
+    if (modulated && j == j0) {   // M_delta[b] joins the first batch's loads (one round trip)
 #pragma unroll
       for (int g = 0; g < G; ++g) {
         const int c = 4 * threadIdx.x + 1024 * g;
@@ -377,9 +378,11 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, i
         if (jj < j1 && c < D) {
           if (act) {
             xv[rr][g] = ld4(a.x + (size_t)(b * a.H + jj) * D + c);
-            const float* mt = a.modv + (size_t)jj * a.mod_ld + a.off;
-            ts[rr][g] = ld4(mt + c);
-            th[rr][g] = ld4(mt + D + c);
+            if (modulated) {
+              const float* mt = a.modv + (size_t)jj * a.mod_ld + a.off;
+              ts[rr][g] = ld4(mt + c);
+              th[rr][g] = ld4(mt + D + c);
+            }
           } else {
             xv[rr][g] = ld4((const T*)a.fop + (size_t)(b * a.F + jj) * D + c);
           }
@@ -411,7 +414,7 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, i
         const int c = 4 * threadIdx.x + 1024 * g;
         if (c >= D) continue;
         const float4 x = xv[rr][g];
-        if (act) {
+        if (modulated) {
           const float4 sc = add2(csc[g], ts[rr][g]), sh = add2(csh[g], th[rr][g]);
           st4(Y + c, make_float4(x.x * inv * (1.f + sc.x) + sh.x, x.y * inv * (1.f + sc.y) + sh.y,
                                  x.z * inv * (1.f + sc.z) + sh.z, x.w * inv * (1.f + sc.w) + sh.w));
@@ -660,6 +663,69 @@ cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st) 
   return cudaGetLastError();
 }
 
+// ============================================================================ FOP adapter cross-attention
+
+// One CTA per (robot b, query head h); warp w takes slots w, w + 8, ...: the
+// scores of a slot over the F FOP keys (lanes split the head dim), the
+// softmax, and the lanes' head-dim slices of the weighted values.
+template <typename T>
+__global__ void __launch_bounds__(256) fop_xattn_kernel(const T* __restrict__ Q, const T* __restrict__ KV,
+                                                        T* __restrict__ out, int H, int F, int Hq, int Hkv, int hd,
+                                                        const float* __restrict__ gate) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ float xs[];
+  float* Ks = xs;                 // [F][hd]
+  float* Vs = Ks + F * hd;        // [F][hd]
+  float* Ps = Vs + F * hd;        // [8 warps][F]
+  const int b = blockIdx.x / Hq, h = blockIdx.x % Hq, g = h / (Hq / Hkv);
+  const int ldkv = 2 * Hkv * hd, ldq = Hq * hd;
+  for (int i = threadIdx.x; i < F * hd; i += blockDim.x) {
+    const int f = i / hd, c = i % hd;
+    const T* row = KV + (size_t)(b * F + f) * ldkv;
+    Ks[i] = to_f32(row[g * hd + c]);
+    Vs[i] = to_f32(row[Hkv * hd + g * hd + c]);
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float scale = rsqrtf((float)hd), gt = tanhf(gate[0]);
+  float* p = Ps + warp * F;
+  for (int j = warp; j < H; j += 8) {
+    const T* q = Q + (size_t)(b * H + j) * ldq + h * hd;
+    float mx = -INFINITY;
+    for (int f = 0; f < F; ++f) {
+      float d = 0.f;
+      for (int c = lane; c < hd; c += 32) d = fmaf(to_f32(q[c]), Ks[f * hd + c], d);
+      d = warp_sum(d) * scale;
+      if (lane == 0) p[f] = d;
+      mx = fmaxf(mx, d);
+    }
+    __syncwarp();
+    float sum = 0.f;
+    for (int f = 0; f < F; ++f) sum += __expf(p[f] - mx);
+    const float inv = gt / sum;
+    T* o = out + (size_t)(b * H + j) * ldq + h * hd;
+    for (int c = lane; c < hd; c += 32) {
+      float acc = 0.f;
+      for (int f = 0; f < F; ++f) acc = fmaf(__expf(p[f] - mx), Vs[f * hd + c], acc);
+      o[c] = from_f32<T>(acc * inv);
+    }
+    __syncwarp();
+  }
+}
+
+cudaError_t launch_fop_xattn(const void* Q, const void* KV, void* out, int B, int H, int F, int Hq, int Hkv, int hd,
+                             const float* gate, Dtype dt, cudaStream_t st) {
+  if (B <= 0 || H <= 0) return cudaSuccess;
+  if (F < 1 || F > 64 || hd > 256) return cudaErrorInvalidValue;
+  const size_t smem = ((size_t)2 * F * hd + 8 * F) * sizeof(float);
+  if (dt == DT_BF16)
+    return launch_kernel(fop_xattn_kernel<bf16>, dim3(B * Hq), dim3(256), smem, st, 1, (const bf16*)Q,
+                         (const bf16*)KV, (bf16*)out, H, F, Hq, Hkv, hd, gate);
+  return launch_kernel(fop_xattn_kernel<float>, dim3(B * Hq), dim3(256), smem, st, 1, (const float*)Q,
+                       (const float*)KV, (float*)out, H, F, Hq, Hkv, hd, gate);
+}
+
 // ============================================================================ tail
 
 // One CTA per robot: a'_j = a_j + dt_j v_j (Eq. 3), released = a'_0, buffer
@@ -776,6 +842,11 @@ cudaError_t init_simt_kernels() {
     e = cudaFuncSetAttribute(attention_simt_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, att);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tail_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * (int)sizeof(float));
+  const int xa = (2 * 64 * 256 + 8 * 64) * (int)sizeof(float);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(fop_xattn_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, xa);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(fop_xattn_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, xa);
   return e;
 }
 

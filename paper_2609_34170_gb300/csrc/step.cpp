@@ -27,6 +27,10 @@ bool validate_config(const ravel_config& c, std::string* why) {
   if (c.max_prefix < 1 || c.fop_tokens < 0 || c.max_batch < 1) return bad("max_prefix, max_batch >= 1, fop_tokens >= 0");
   if (c.dtype != RAVEL_FP32 && c.dtype != RAVEL_BF16) return bad("dtype must be RAVEL_FP32 or RAVEL_BF16");
   if (c.mask_mode != RAVEL_MASK_FULL && c.mask_mode != RAVEL_MASK_SLOT_ISOLATED) return bad("unknown mask_mode");
+  if (c.fop_adapter_every < 0 || c.fop_adapter_every > c.layers)
+    return bad("fop_adapter_every must be 0 or in [1, layers]");
+  if (c.fop_adapter_every > 0 && (c.fop_tokens < 1 || c.fop_tokens > 64))
+    return bad("FOP adapters need 1 <= fop_tokens <= 64");
   return true;
 }
 
@@ -83,6 +87,10 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
       *errs = "a weight pointer is null";
       return RAVEL_EINVAL;
     }
+  if (c.fop_adapter_every > 0 && (!w.a_gamma || !w.a_zgamma || !w.a_wq || !w.a_wkv || !w.a_wo || !w.a_gate)) {
+    *errs = "an adapter weight pointer is null";
+    return RAVEL_EINVAL;
+  }
   p->cfg = c;
   p->dt = c.dtype == RAVEL_BF16 ? DT_BF16 : DT_F32;
   p->esize = c.dtype == RAVEL_BF16 ? 2 : 4;
@@ -143,6 +151,21 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->tcws.counters, p->tcws.n_counters * sizeof(int));
   AL(p->dn_times, (size_t)H * sizeof(float));
   AL(p->rel_mask, (size_t)A * sizeof(float));
+  p->n_adapters = c.fop_adapter_every > 0 ? L / c.fop_adapter_every : 0;
+  const int NA = p->n_adapters, nkv = 2 * c.n_kv_heads * c.head_dim;
+  if (NA) {
+    AL(p->a_wq, (size_t)NA * p->qdim * D * es);
+    AL(p->a_wkv, (size_t)NA * nkv * D * es);
+    AL(p->a_wo, (size_t)NA * D * p->qdim * es);
+    AL(p->a_gamma, (size_t)NA * D * 4);
+    AL(p->a_zgamma, (size_t)NA * D * 4);
+    AL(p->a_gate, (size_t)NA * 4);
+    AL(p->Ya, (size_t)Bm * H * D * es);
+    AL(p->Za, (size_t)Bm * F * D * es);
+    AL(p->Qa, (size_t)Bm * H * p->qdim * es);
+    AL(p->KVa, (size_t)Bm * F * nkv * es);
+    AL(p->XA, (size_t)Bm * H * p->qdim * es);
+  }
   AL(p->seeds, Bm * sizeof(uint64_t));
   AL(p->counters, Bm * sizeof(uint64_t));
   AL(p->err, sizeof(int));
@@ -206,6 +229,17 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
     pk.transpose(w.w_down + (size_t)l * Fm * D, Fm, D, (char*)p->w_down + (size_t)l * D * Fm * es);
   }
   pk.transpose(w.out_w, D, A, p->out_w);
+  for (int i = 0; i < NA; ++i) {
+    const int nkv2 = 2 * c.n_kv_heads * c.head_dim;
+    pk.transpose(w.a_wq + (size_t)i * D * p->qdim, D, p->qdim, (char*)p->a_wq + (size_t)i * p->qdim * D * es);
+    pk.transpose(w.a_wkv + (size_t)i * D * nkv2, D, nkv2, (char*)p->a_wkv + (size_t)i * nkv2 * D * es);
+    pk.transpose(w.a_wo + (size_t)i * p->qdim * D, p->qdim, D, (char*)p->a_wo + (size_t)i * D * p->qdim * es);
+  }
+  if (NA) {
+    pk.copy_f32(w.a_gamma, (size_t)NA * D, p->a_gamma);
+    pk.copy_f32(w.a_zgamma, (size_t)NA * D, p->a_zgamma);
+    pk.copy_f32(w.a_gate, (size_t)NA, p->a_gate);
+  }
   pk.copy_f32(w.t_b1, D, p->t_b1);
   pk.copy_f32(w.t_b2, D, p->t_b2);
   pk.copy_f32(w.d_b1, D, p->d_b1);
@@ -236,7 +270,7 @@ cudaError_t run_gemm(const StepPlan& p, const GemmArgs& g, cudaStream_t st) {
 const char* kernel_kind_name(int k) {
   static const char* const names[KK_COUNT] = {"embed", "gemm_cond", "gemm_mod", "in_proj", "norm", "gemm_qkv",
                                               "attention", "gemm_o", "gemm_gate_up", "geglu", "gemm_down",
-                                              "gemm_out", "tail", "cond_cache"};
+                                              "gemm_out", "tail", "cond_cache", "adapter"};
   return (k >= 0 && k < KK_COUNT) ? names[k] : "unknown";
 }
 
@@ -300,12 +334,13 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   // residual stream
   RUN(KK_IN_PROJ, launch_in_proj(io.buffer, B * H, A, D, p.in_w, p.in_b, p.x, st, io.state, p.rel_mask, io.slot_times,
                                  H));
-  const int FF = io.obs ? F : 0;      // FOP tokens present in this step
+  const bool adapters = p.n_adapters > 0 && io.obs;
+  const int FF = (io.obs && !adapters) ? F : 0;   // FOP tokens as keys of the self-attention
   const int RPR = H + FF;              // normed / QKV rows per robot: H slots, then the FOP tokens
   const int BH = B * H, BY = B * RPR;
   for (int l = 0; l < L; ++l) {
-    NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, io.obs, F, p.fop_gamma + (size_t)l * D, p.Y, RPR,
-                p.cond_drow};
+    NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, FF ? io.obs : nullptr, F,
+                p.fop_gamma + (size_t)l * D, p.Y, RPR, p.cond_drow};
     RUN(KK_NORM, launch_ada_norm(n1, dt, st));
     const void* wqkv = (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es;
     if (p.use_tc_attn) {
@@ -334,6 +369,23 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     }
     RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x,
                         D, DT_F32, nullptr, p.split_cap[1]));
+    if (adapters && (l + 1) % c.fop_adapter_every == 0) {
+      // gated cross-attention adapter: the action rows attend to the FOP tokens
+      const int ai = (l + 1) / c.fop_adapter_every - 1, nkv = 2 * c.n_kv_heads * c.head_dim;
+      NormArgs na{p.x, B, H, D, nullptr, 0, nullptr, 0, nullptr, 0, nullptr, p.Ya, H};
+      na.act_gain = p.a_gamma + (size_t)ai * D;
+      RUN(KK_ADAPTER, launch_ada_norm(na, dt, st));
+      NormArgs nz{p.x, B, 0, D, nullptr, 0, nullptr, 0, io.obs, F, p.a_zgamma + (size_t)ai * D, p.Za, F};
+      RUN(KK_ADAPTER, launch_ada_norm(nz, dt, st));
+      RUN(KK_ADAPTER, gemm(p.Ya, D, (const char*)p.a_wq + (size_t)ai * p.qdim * D * es, BH, p.qdim, D, EPI_STORE, p.Qa,
+                           p.qdim, dt, nullptr));
+      RUN(KK_ADAPTER, gemm(p.Za, D, (const char*)p.a_wkv + (size_t)ai * nkv * D * es, B * F, nkv, D, EPI_STORE, p.KVa,
+                           nkv, dt, nullptr));
+      RUN(KK_ADAPTER, launch_fop_xattn(p.Qa, p.KVa, p.XA, B, H, F, c.n_q_heads, c.n_kv_heads, c.head_dim,
+                                       p.a_gate + ai, dt, st));
+      RUN(KK_ADAPTER, gemm(p.XA, p.qdim, (const char*)p.a_wo + (size_t)ai * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32,
+                           p.x, D, DT_F32, nullptr));
+    }
     NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
     RUN(KK_NORM, launch_ada_norm(n2, dt, st));
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;

@@ -71,6 +71,12 @@ struct StepPlan {
   bool use_tc = false;      // bf16 projections on tcgen05
   float* dn_times = nullptr;   // [H] flow times of a synchronous denoising pass (all equal)
   float* rel_mask = nullptr;   // [A] 1 = a dimension the expert predicts relative to the robot state
+  // FOP adapters (cfg.fop_adapter_every > 0): packed K-major weights, gains,
+  // gates and their activations
+  int n_adapters = 0;
+  void *a_wq = nullptr, *a_wkv = nullptr, *a_wo = nullptr;
+  float *a_gamma = nullptr, *a_zgamma = nullptr, *a_gate = nullptr;
+  void *Ya = nullptr, *Za = nullptr, *Qa = nullptr, *KVa = nullptr, *XA = nullptr;
   uint64_t* seeds = nullptr;
   uint64_t* counters = nullptr;
   int* err = nullptr;
@@ -84,7 +90,7 @@ void plan_destroy(StepPlan* p);
 // Kernel kinds of one step (per-launch profiling labels).
 enum KernelKind {
   KK_EMBED = 0, KK_GEMM_COND, KK_GEMM_MOD, KK_IN_PROJ, KK_NORM, KK_GEMM_QKV, KK_ATTENTION, KK_GEMM_O,
-  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_COUNT
+  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_ADAPTER, KK_COUNT
 };
 const char* kernel_kind_name(int k);
 
