@@ -64,6 +64,17 @@ cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int
 
 // ---- generic projection GEMM: out[m][n] = sum_k A[m][k] W[n][k] (W K-major) ----
 enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2, EPI_GEGLU = 3 };
+
+// adaRMSNorm of whole rows right after a residual update (see NormArgs for
+// the formula): action row (b, j) = residual row b*H + j, written to
+// Y[b*row_pitch + j]; with fop, FOP row (b, f) written to Y[b*row_pitch + H + f].
+struct RowNorm {
+  const float* modv; int mod_ld; const float* mod_b; int off; const int* drow;
+  int B, H;
+  const void* fop; int F; const float* gamma;
+  void* Y; int row_pitch;
+  int* gbar;                    // {count, generation} of a grid-wide barrier (zero-initialised)
+};
 struct GemmArgs {
   const void* A; int lda;       // [M][K] activations of dtype dt
   const void* W; int ldw;       // [N][K] weights of dtype dt
@@ -79,6 +90,11 @@ struct GemmArgs {
   int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
   int max_splits = 0;           // tcgen05 path: cap on the split-K factor (0: chosen from the shape)
   const int* skip = nullptr;    // optional device flag: nonzero at run time -> the launch computes nothing
+  // optional (EPI_ADD_F32 into the residual stream, bf16 operands, few
+  // tiles): the launch also normalises every updated row (the split
+  // partials meet in global memory, the CTAs pass a grid-wide barrier and
+  // the CTA owning a row sums it, adds it to `out` and writes its norm)
+  const RowNorm* rownorm = nullptr;
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
 
@@ -126,6 +142,12 @@ cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b,
                            float* x, cudaStream_t st, const float* state = nullptr, const float* rel_mask = nullptr,
                            const float* slot_times = nullptr, int H = 1);
+
+// The in-projection (as launch_in_proj) of whole rows with the first layer's
+// adaRMSNorm into rn.Y (action rows and, with rn.fop, FOP rows).
+cudaError_t launch_in_proj_norm(const float* buf, int A, int D, const float* in_w, const float* in_b, float* x,
+                                const float* state, const float* rel_mask, const float* slot_times, const RowNorm& rn,
+                                Dtype dt, cudaStream_t st);
 
 // ---- GeGLU on the interleaved gate/up GEMM output --------------------------------
 cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cudaStream_t st);

@@ -501,6 +501,90 @@ cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* 
                        in_w, in_b, x, state, rel_mask, slot_times, H);
 }
 
+// The in-projection of whole rows with the first layer's adaRMSNorm: one
+// CTA per row; an action row is projected (x, fp32), then normalised with its
+// modulation into Y; a FOP row is normalised with its gain.  (Rows of up to
+// 4096 features: a thread owns features tid, tid + 256, ...)
+template <typename T>
+__global__ void __launch_bounds__(256) in_proj_norm_kernel(const float* __restrict__ buf, int A, int D,
+                                                           const float* __restrict__ in_w,
+                                                           const float* __restrict__ in_b, float* __restrict__ x,
+                                                           const float* __restrict__ state,
+                                                           const float* __restrict__ rel_mask,
+                                                           const float* __restrict__ slot_times, RowNorm rn) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ float arow[];   // the action row of this slot
+  __shared__ float red[32];
+  const int r = blockIdx.x, BH = rn.B * rn.H;
+  float v[16];
+  float ss = 0.f;
+  if (r < BH) {
+    const int b = r / rn.H, j = r % rn.H;
+    for (int i = threadIdx.x; i < A; i += blockDim.x) {
+      float a = buf[(size_t)r * A + i];
+      if (state)   // relative coordinates of the expert: a - (1 - t_j) m s_b
+        a = __fsub_rn(a, __fmul_rn(__fsub_rn(1.f, slot_times[j]), __fmul_rn(rel_mask[i], state[(size_t)b * A + i])));
+      arow[i] = a;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int c = threadIdx.x + 256 * k;
+      v[k] = 0.f;
+      if (c < D) {
+        float acc = in_b[c];
+        for (int i = 0; i < A; ++i) acc = fmaf(arow[i], in_w[(size_t)i * D + c], acc);
+        x[(size_t)r * D + c] = acc;
+        v[k] = acc;
+        ss += acc * acc;
+      }
+    }
+    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
+    const float* mt = rn.modv + (size_t)j * rn.mod_ld + rn.off;
+    const float* md = rn.modv + (size_t)(rn.drow ? rn.drow[b] : rn.H + b) * rn.mod_ld + rn.off;
+    const float* mb = rn.mod_b + rn.off;
+    T* Y = (T*)rn.Y + (size_t)(b * rn.row_pitch + j) * D;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int c = threadIdx.x + 256 * k;
+      if (c < D) {
+        const float sc = mt[c] + md[c] + mb[c], sh = mt[D + c] + md[D + c] + mb[D + c];
+        Y[c] = from_f32<T>(v[k] * inv * (1.f + sc) + sh);
+      }
+    }
+  } else {
+    const int fr = r - BH, b = fr / rn.F, f = fr % rn.F;
+    const T* z = (const T*)rn.fop + (size_t)(b * rn.F + f) * D;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int c = threadIdx.x + 256 * k;
+      v[k] = c < D ? to_f32(z[c]) : 0.f;
+      ss += v[k] * v[k];
+    }
+    const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
+    T* Y = (T*)rn.Y + (size_t)(b * rn.row_pitch + rn.H + f) * D;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int c = threadIdx.x + 256 * k;
+      if (c < D) Y[c] = from_f32<T>(v[k] * inv * (1.f + rn.gamma[c]));
+    }
+  }
+}
+
+cudaError_t launch_in_proj_norm(const float* buf, int A, int D, const float* in_w, const float* in_b, float* x,
+                                const float* state, const float* rel_mask, const float* slot_times, const RowNorm& rn,
+                                Dtype dt, cudaStream_t st) {
+  if (D > 4096) return cudaErrorInvalidValue;
+  const int rows = rn.B * rn.H + (rn.fop ? rn.B * rn.F : 0);
+  if (rows <= 0) return cudaSuccess;
+  if (dt == DT_BF16)
+    return launch_kernel(in_proj_norm_kernel<bf16>, dim3(rows), dim3(256), A * sizeof(float), st, 1, buf, A, D, in_w,
+                         in_b, x, state, rel_mask, slot_times, rn);
+  return launch_kernel(in_proj_norm_kernel<float>, dim3(rows), dim3(256), A * sizeof(float), st, 1, buf, A, D, in_w,
+                       in_b, x, state, rel_mask, slot_times, rn);
+}
+
 // ============================================================================ GeGLU
 
 template <typename T>

@@ -71,6 +71,8 @@ struct StepPlan {
   bool use_tc = false;      // bf16 projections on tcgen05
   float* dn_times = nullptr;   // [H] flow times of a synchronous denoising pass (all equal)
   float* rel_mask = nullptr;   // [A] 1 = a dimension the expert predicts relative to the robot state
+  int* gbar = nullptr;         // {count, generation}: grid-wide barrier of the row-norm GEMMs
+  bool fuse_norm = true;       // residual GEMMs of few tiles also write the next adaRMSNorm
   // FOP adapters (cfg.fop_adapter_every > 0): packed K-major weights, gains,
   // gates and their activations
   int n_adapters = 0;
