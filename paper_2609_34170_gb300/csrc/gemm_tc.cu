@@ -61,7 +61,7 @@ constexpr int STG_LD = 132;                  // SIMT staging pitch (floats): 16 
 constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
 constexpr uint32_t XCH_BYTES = 32 * STG_LD * 4;  // GeGLU transpose tile (TMA epilogue): <= 32 tokens x 128 rows
 
-enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3, RED_ROWS = 4 };
+enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3 };
 // Epilogue kind of an instantiation: outputs through TMA boxes as fp32, bf16
 // (+ the V^T side output), a reduce-add into the fp32 residual stream or the
 // GeGLU pair -- fixed, so that a long persistent launch carries only the code
@@ -108,12 +108,6 @@ struct TcParams {
                         // nobody makes, so the launch gives up after wait_ns and unwinds
   const int* skip;      // optional device flag read after the dependency wait: nonzero -> the launch
                         // completes the copies it started and exits without computing
-  // RED_ROWS: the partials of split sp of tile tn go to ws token-major,
-  // [tn][sp][token m < mpad][128 rows], and after a grid-wide barrier the CTAs
-  // own the residual rows (and the FOP rows of rn) and normalise them
-  RowNorm rn;
-  int mpad;             // token rows of one partial (tiles_m * BN)
-  int nctas;            // CTAs of the grid
 };
 
 // The TMA epilogue kind of a launch (EK_F32 .. EK_GEGLU).
@@ -750,17 +744,6 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
                                  __uint_as_float(raw[4 * qq + 2]), __uint_as_float(raw[4 * qq + 3])));
         }
         __threadfence();
-      } else if constexpr (RED == RED_ROWS) {
-        // token-major partial: a warp stores 32 consecutive rows (128 bytes)
-        // of one token per instruction, so the row owners read contiguous runs
-        float* w = p.ws + (((size_t)tn * p.splits + sp) * p.mpad + m_base) * TC_BM + r;
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          float v[16];
-          tmem_ld16(trow + c0, v);
-#pragma unroll
-          for (int k = 0; k < 16; ++k)
-            if (m_base + c0 + k < p.M) __stcg(w + (size_t)(c0 + k) * TC_BM, v[k]);
-        }
       } else {
         // workspace mode: [split][tile][col][row] partials, last arrival reduces
         const int tiles = gridDim.x * gridDim.y;
@@ -844,126 +827,6 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         int ebuf = 0;
         if constexpr (TMA_OUT) epilogue_tma<EK, 32>(p, &tmO, tn0, tm0 * BN + sp0 * cpr, r, v, brow, stg_raw, xch, ebuf);
         if (threadIdx.x == 64) bulk_wait<0>();
-      }
-    }
-  }
-  if constexpr (RED == RED_ROWS) {
-    // Every CTA has stored its partial (or given up).  CTA c owns rows c,
-    // c + grid, ...: a residual row is x + the splits' partials of its
-    // features (summed in split order) and its adaRMSNorm goes to Y; a FOP row
-    // is normalised as it is.  What a row needs besides the partials (x, the
-    // modulation, the FOP token) does not depend on this launch, so the first
-    // row's inputs are loaded while thread 0 waits at the grid-wide barrier,
-    // which every CTA passes whatever happened before (none waits for a CTA
-    // that left).  The partials then come by asynchronous copies into the
-    // drained operand ring: one L2 round trip per row.
-    const RowNorm& rn = p.rn;
-    const int D = p.N, tid = threadIdx.x - 64, f0 = 8 * tid;
-    const bool on = warp >= 2 && f0 < D;   // D is a multiple of 8, at most 1024
-    const int nrows = p.M + (rn.fop ? rn.B * rn.F : 0);
-    const int cta = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);
-    float* xo = (float*)p.out;
-    float xs[8], sc[8], sh[8];
-    // x, scale and shift of an action row; z, gain and 0 of a FOP row
-    auto load_row = [&](int row) {
-      if (row < p.M) {
-        const int b = row / rn.H, j = row - b * rn.H;
-        const float* mt = rn.modv + (size_t)j * rn.mod_ld + rn.off + f0;
-        const float* md = rn.modv + (size_t)(rn.drow ? rn.drow[b] : rn.H + b) * rn.mod_ld + rn.off + f0;
-        const float* mb = rn.mod_b + rn.off + f0;
-        const float* xr = xo + (size_t)row * p.ldo + f0;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const float4 xv = *(const float4*)(xr + 4 * h);
-          const float4 t0 = *(const float4*)(mt + 4 * h), t1 = *(const float4*)(mt + D + 4 * h);
-          const float4 d0 = *(const float4*)(md + 4 * h), d1 = *(const float4*)(md + D + 4 * h);
-          const float4 b0 = *(const float4*)(mb + 4 * h), b1 = *(const float4*)(mb + D + 4 * h);
-          const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
-          const float s0[4] = {t0.x + d0.x + b0.x, t0.y + d0.y + b0.y, t0.z + d0.z + b0.z, t0.w + d0.w + b0.w};
-          const float h0[4] = {t1.x + d1.x + b1.x, t1.y + d1.y + b1.y, t1.z + d1.z + b1.z, t1.w + d1.w + b1.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            xs[4 * h + e] = xa[e];
-            sc[4 * h + e] = s0[e];
-            sh[4 * h + e] = h0[e];
-          }
-        }
-      } else {
-        const int fr = row - p.M, b = fr / rn.F, f = fr - b * rn.F;
-        const uint4 z = *(const uint4*)((const bf16*)rn.fop + (size_t)(b * rn.F + f) * D + f0);
-        const uint32_t zz[4] = {z.x, z.y, z.z, z.w};
-        const float4 g0 = *(const float4*)(rn.gamma + f0), g1 = *(const float4*)(rn.gamma + f0 + 4);
-        const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          xs[2 * e] = __uint_as_float(zz[e] << 16);
-          xs[2 * e + 1] = __uint_as_float(zz[e] & 0xFFFF0000u);
-        }
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          sc[e] = gg[e];
-          sh[e] = 0.f;
-        }
-      }
-    };
-    if (on && cta < nrows) load_row(cta);
-    if (threadIdx.x == 0) {
-      flags[1] = grid_epoch_sync((unsigned*)rn.gbar, p.nctas, cta == 0) ? 1 : 0;
-      if (!flags[1]) raise_error(p.err, ERR_TIMEOUT);
-    }
-    cta_sync();
-    if (flags[1] && warp >= 2) {
-      float* red = stage;   // [2][4] row sums of the epilogue warps
-      // this thread's partial slots in the ring: [split][half][128] float4
-      float4* own = (float4*)smem + tid;
-      if (on) fence_proxy_async_smem();   // the ring was last used by TMA and the tensor cores
-      const size_t sstride = (size_t)p.mpad * TC_BM;
-      int rb = 0;
-      for (int row = cta; row < nrows; row += p.nctas, rb ^= 1) {
-        if (row != cta && on) load_row(row);
-        const bool act = row < p.M;
-        float v[8];
-        float ss = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = xs[e];
-        if (on && act) {
-          const float* pp = p.ws + (((size_t)(f0 / TC_BM) * p.splits) * p.mpad + row) * TC_BM + f0 % TC_BM;
-          for (int sp2 = 0; sp2 < p.splits; ++sp2) {
-            cp_async16(own + (size_t)(2 * sp2) * TC_BM, pp + sp2 * sstride);
-            cp_async16(own + (size_t)(2 * sp2 + 1) * TC_BM, pp + sp2 * sstride + 4);
-          }
-          cp_async_wait_all();
-          float acc[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-          for (int sp2 = 0; sp2 < p.splits; ++sp2) {
-            const float4 pa = own[(size_t)(2 * sp2) * TC_BM], pb = own[(size_t)(2 * sp2 + 1) * TC_BM];
-            acc[0] += pa.x; acc[1] += pa.y; acc[2] += pa.z; acc[3] += pa.w;
-            acc[4] += pb.x; acc[5] += pb.y; acc[6] += pb.z; acc[7] += pb.w;
-          }
-#pragma unroll
-          for (int e = 0; e < 8; ++e) v[e] += acc[e];
-          *(float4*)(xo + (size_t)row * p.ldo + f0) = make_float4(v[0], v[1], v[2], v[3]);
-          *(float4*)(xo + (size_t)row * p.ldo + f0 + 4) = make_float4(v[4], v[5], v[6], v[7]);
-        }
-        if (on) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) ss += v[e] * v[e];
-        }
-        const int b = act ? row / rn.H : (row - p.M) / rn.F;
-        const int orow = b * rn.row_pitch + (act ? row - b * rn.H : rn.H + (row - p.M) - b * rn.F);
-        ss = warp_sum(ss);
-        if (lane == 0) red[rb * 4 + (warp & 3)] = ss;
-        epi_bar();
-        const float tot = red[rb * 4] + red[rb * 4 + 1] + red[rb * 4 + 2] + red[rb * 4 + 3];
-        const float inv = rsqrtf(tot / (float)D + 1e-6f);
-        if (on) {
-          float y[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) y[e] = v[e] * inv * (1.f + sc[e]) + sh[e];
-          *(uint4*)((bf16*)rn.Y + (size_t)orow * D + f0) = make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]),
-                                                                      pack_bf16x2(y[4], y[5]), pack_bf16x2(y[6], y[7]));
-        }
       }
     }
   }
@@ -1278,7 +1141,6 @@ TcKernel tc_kernel(int red, int ek) {
   RAVEL_TC_K(RED_L2_CLUSTER, EK_TMA_ANY) RAVEL_TC_K(RED_L2_CLUSTER, EK_GENERIC)
   RAVEL_TC_K(RED_DSMEM, EK_TMA_ANY)
   RAVEL_TC_K(RED_WORKSPACE, EK_GENERIC)
-  RAVEL_TC_K(RED_ROWS, EK_GENERIC)
 #undef RAVEL_TC_K
   return nullptr;
 }
@@ -1434,7 +1296,7 @@ cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
   std::vector<const void*> kernels;
-  for (int red = 0; red <= RED_ROWS; ++red)
+  for (int red = 0; red < 4; ++red)
     for (int ek = 0; ek <= EK_TMA_ANY; ++ek)
       if (TcKernel k = tc_kernel(red, ek)) kernels.push_back((const void*)k);
   for (int ek = 0; ek < EK_GENERIC; ++ek) kernels.push_back((const void*)tc_pair_kernel(ek));
@@ -1483,16 +1345,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   int splits = 1;
   if (tiles < num_sms) splits = std::min(num_kb, std::max(1, num_sms / tiles));
   if (g.max_splits > 0) splits = std::min(splits, g.max_splits);
-  // residual update with the rows' adaRMSNorm fused: split partials meet in
-  // global memory behind one grid-wide barrier, which needs every CTA
-  // resident at once (at most one per SM) and whole rows of at most 1024
-  const bool rows = g.rownorm != nullptr;
-  if (rows) {
-    const size_t part = (size_t)tiles * splits * tiles_m * bn * TC_BM * 4;
-    if (g.epi != EPI_ADD_F32 || g.bias || g.N > 1024 || g.N % 8 || g.ldo % 4 || splits < 2 ||
-        tiles * splits > num_sms || part > ws.ws_bytes || !g.rownorm->gbar)
-      return cudaErrorNotSupported;
-  } else if (cluster) {
+  if (cluster) {
     // the splits of a tile form one cluster: a power of two, at most the cluster
     // limit, whose partials fit the workspace and whose column slices are
     // multiples of 4
@@ -1504,7 +1357,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   } else {
     while (splits > 1 && ((size_t)splits * tiles * bn * TC_BM * 4 > ws.ws_bytes || tiles > ws.n_counters)) --splits;
   }
-  int reduce = rows ? RED_ROWS : splits == 1 ? RED_NONE : (cluster ? RED_L2_CLUSTER : RED_WORKSPACE);
+  int reduce = splits == 1 ? RED_NONE : (cluster ? RED_L2_CLUSTER : RED_WORKSPACE);
   {
     // two-SM tiles for a persistent launch whose pair tiles fill at least
     // three quarters of the pairs of SMs
@@ -1533,17 +1386,14 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   stages = std::max(2, std::min(stages, std::max(2, kb_per_item * items)));
   // one-shot: a cluster split whose whole K range fits a ring of up to 200 KB
   // takes its weight and token k-tiles in one box each (K a multiple of 64)
-  const bool oneshot = splits > 1 && (cluster || rows) && g.K % TC_BK == 0 && g.K / TC_BK <= 256 &&
+  const bool oneshot = splits > 1 && cluster && g.K % TC_BK == 0 && g.K / TC_BK <= 256 &&
                        (size_t)kb_per_item * stage_bytes <= (size_t)TC_SMEM_BUDGET;
   if (oneshot) stages = kb_per_item;   // the ring is exactly one box deep
-  size_t ring = ((size_t)stages * stage_bytes + 1023) / 1024 * 1024;
-  // RED_ROWS: the row owners' partial slots ([split][2][128] float4) overlay the ring
-  if (rows) ring = std::max(ring, ((size_t)splits * 2 * TC_BM * 16 + 1023) / 1024 * 1024);
+  const size_t ring = ((size_t)stages * stage_bytes + 1023) / 1024 * 1024;
   // outputs through TMA boxes when the output rows are 16-byte aligned
   const bool out_bf = g.epi == EPI_GEGLU || (g.epi != EPI_ADD_F32 && g.out_dt == DT_BF16);
   const int es = out_bf ? 2 : 4;
-  const bool tma_out = reduce != RED_WORKSPACE && reduce != RED_ROWS && ((uintptr_t)g.out & 15) == 0 &&
-                       ((size_t)g.ldo * es) % 16 == 0;
+  const bool tma_out = reduce != RED_WORKSPACE && ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * es) % 16 == 0;
   int box_m = 0;
   uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, vts_off = 0, rcv_off = 0, bar_off = 0;
   size_t smem = 0;
@@ -1588,11 +1438,6 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
              vts_off, rcv_off, bar_off, kTcTimeoutNs, 0, g.skip};
-  if (rows) {
-    p.rn = *g.rownorm;
-    p.mpad = tiles_m * bn;
-    p.nctas = tiles * splits;
-  }
   // fault injection (tests): a launch without a cluster may be told to wait
   // for an arrival that never comes, with a short limit
   if ((reduce == RED_NONE || reduce == RED_WORKSPACE) && g_withhold.load() > 0 && g_withhold.fetch_sub(1) > 0) {

@@ -65,7 +65,7 @@ cudaError_t launch_embed(const float* slot_times, int H, const float* delta, int
 // ---- generic projection GEMM: out[m][n] = sum_k A[m][k] W[n][k] (W K-major) ----
 enum Epi { EPI_STORE = 0, EPI_STORE_SILU = 1, EPI_ADD_F32 = 2, EPI_GEGLU = 3 };
 
-// adaRMSNorm of whole rows right after a residual update (see NormArgs for
+// adaRMSNorm of whole rows right after the in-projection (see NormArgs for
 // the formula): action row (b, j) = residual row b*H + j, written to
 // Y[b*row_pitch + j]; with fop, FOP row (b, f) written to Y[b*row_pitch + H + f].
 struct RowNorm {
@@ -73,7 +73,6 @@ struct RowNorm {
   int B, H;
   const void* fop; int F; const float* gamma;
   void* Y; int row_pitch;
-  int* gbar;                    // {count, generation} of a grid-wide barrier (zero-initialised)
 };
 struct GemmArgs {
   const void* A; int lda;       // [M][K] activations of dtype dt
@@ -90,11 +89,6 @@ struct GemmArgs {
   int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
   int max_splits = 0;           // tcgen05 path: cap on the split-K factor (0: chosen from the shape)
   const int* skip = nullptr;    // optional device flag: nonzero at run time -> the launch computes nothing
-  // optional (EPI_ADD_F32 into the residual stream, bf16 operands, few
-  // tiles): the launch also normalises every updated row (the split
-  // partials meet in global memory, the CTAs pass a grid-wide barrier and
-  // the CTA owning a row sums it, adds it to `out` and writes its norm)
-  const RowNorm* rownorm = nullptr;
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
 

@@ -61,6 +61,13 @@ static ravel_status cuda_fail(ravel_t* r, cudaError_t e, const char* what) {
   return fail(r, e == cudaErrorMemoryAllocation ? RAVEL_ENOMEM : RAVEL_ECUDA, m);
 }
 
+// an enqueue_step failure, naming the kernel kind whose launch failed
+static ravel_status enqueue_fail(ravel_t* r, cudaError_t e, const char* what) {
+  const int k = enqueue_fail_kind();
+  const std::string m = std::string(what) + (k >= 0 ? std::string(" (") + kernel_kind_name(k) + ")" : std::string());
+  return cuda_fail(r, e, m.c_str());
+}
+
 #define RV_CUDA(r, call, what)                         \
   do {                                                 \
     cudaError_t _e = (call);                           \
@@ -144,7 +151,6 @@ ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* bu
   // a new rollout starts with an empty conditioning cache (its rows are then
   // computed at this batch size only)
   RV_CUDA(r, cudaMemset(r->plan.cond, 0, sizeof(CondCache)), "reset: clear conditioning cache");
-  RV_CUDA(r, cudaMemset(r->plan.gbar, 0, 2 * sizeof(int)), "reset: clear grid barrier");
   *r->err_host = 0;
   RV_CUDA(r, cudaMemcpy(r->plan.seeds, seeds, sizeof(uint64_t) * batch, cudaMemcpyHostToDevice), "reset: seeds");
   RV_CUDA(r, launch_reset(buffer, r->plan.seeds, r->plan.counters, batch, r->plan.cfg.slots,
@@ -252,7 +258,7 @@ static ravel_status roll_step_impl(ravel_t* r, float* buffer, const float* slot_
     cudaError_t e2 = cudaStreamEndCapture(r->cap_stream, &graph);
     if (e != cudaSuccess) {
       if (graph) cudaGraphDestroy(graph);
-      return cuda_fail(r, e, "roll_step: enqueue");
+      return enqueue_fail(r, e, "roll_step: enqueue");
     }
     RV_CUDA(r, e2, "capture end");
     e = cudaGraphInstantiateWithFlags(&r->gexec, graph, 0);
@@ -330,7 +336,7 @@ ravel_status ravel_denoise_chunk(ravel_t* r, float* chunk, int n_steps, const vo
     cudaError_t e2 = cudaStreamEndCapture(r->cap_stream, &graph);
     if (e != cudaSuccess) {
       if (graph) cudaGraphDestroy(graph);
-      return cuda_fail(r, e, "denoise_chunk: enqueue");
+      return enqueue_fail(r, e, "denoise_chunk: enqueue");
     }
     RV_CUDA(r, e2, "capture end");
     e = cudaGraphInstantiateWithFlags(&r->dn_gexec, graph, 0);

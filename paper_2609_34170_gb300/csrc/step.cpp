@@ -151,7 +151,6 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->tcws.counters, p->tcws.n_counters * sizeof(int));
   AL(p->dn_times, (size_t)H * sizeof(float));
   AL(p->rel_mask, (size_t)A * sizeof(float));
-  AL(p->gbar, 2 * sizeof(int));
   p->n_adapters = c.fop_adapter_every > 0 ? L / c.fop_adapter_every : 0;
   const int NA = p->n_adapters, nkv = 2 * c.n_kv_heads * c.head_dim;
   if (NA) {
@@ -268,6 +267,11 @@ cudaError_t run_gemm(const StepPlan& p, const GemmArgs& g, cudaStream_t st) {
   return launch_gemm_simt(g, p.dt, st);
 }
 
+int& enqueue_fail_kind() {
+  static thread_local int k = -1;
+  return k;
+}
+
 const char* kernel_kind_name(int k) {
   static const char* const names[KK_COUNT] = {"embed", "gemm_cond", "gemm_mod", "in_proj", "norm", "gemm_qkv",
                                               "attention", "gemm_o", "gemm_gate_up", "geglu", "gemm_down",
@@ -279,6 +283,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
                          LaunchTrace* trace, const DenoisePass* dn) {
   const ravel_config& c = p.cfg;
   const int D = c.width, L = c.layers, H = c.slots, A = c.action_dim, F = c.fop_tokens, Fm = c.mlp_dim;
+  enqueue_fail_kind() = -1;
   const size_t es = p.esize;
   const Dtype dt = p.dt;
   int nk = 0;
@@ -298,6 +303,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       e = (call);                       \
       ++nk;                             \
       mark(kind);                       \
+      if (e != cudaSuccess) enqueue_fail_kind() = (kind); \
     }                                   \
   } while (0)
   auto gemm = [&](const void* Aop, int lda, const void* W, int M, int N, int K, Epi epi, void* out, int ldo,
@@ -338,7 +344,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   if (fuse_in) {
     const int FF0 = (io.obs && !(p.n_adapters > 0)) ? F : 0;
     const RowNorm rn0{p.modv, p.mod_dim, p.mod_b, 0, p.cond_drow, B, H, FF0 ? io.obs : nullptr, F, p.fop_gamma, p.Y,
-                      H + FF0, p.gbar};
+                      H + FF0};
     RUN(KK_IN_PROJ, launch_in_proj_norm(io.buffer, A, D, p.in_w, p.in_b, p.x, io.state, p.rel_mask, io.slot_times,
                                         rn0, dt, st));
   } else {
@@ -349,24 +355,10 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   const int FF = (io.obs && !adapters) ? F : 0;   // FOP tokens as keys of the self-attention
   const int RPR = H + FF;              // normed / QKV rows per robot: H slots, then the FOP tokens
   const int BH = B * H, BY = B * RPR;
-  // A residual GEMM of few tiles (split K) may also write the adaRMSNorm that
-  // follows it: its CTAs own whole rows after a grid-wide barrier.  Returns
-  // whether it launched so; otherwise nothing was launched.
-  auto gemm_rownorm = [&](GemmArgs g, const RowNorm& rn, int kind) {
-    if (e != cudaSuccess || !p.use_tc || !p.fuse_norm || !tc_gemm_supported(g)) return false;
-    g.rownorm = &rn;
-    const cudaError_t r = launch_gemm_tc(g, p.tcws, p.num_sms, st);
-    if (r == cudaErrorNotSupported) return false;
-    e = r;
-    ++nk;
-    mark(kind);
-    return true;
-  };
-  bool y_ready = fuse_in;   // Y already holds this layer's first norm (in-projection or previous down GEMM)
   for (int l = 0; l < L; ++l) {
     NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, FF ? io.obs : nullptr, F,
                 p.fop_gamma + (size_t)l * D, p.Y, RPR, p.cond_drow};
-    if (!y_ready) RUN(KK_NORM, launch_ada_norm(n1, dt, st));
+    if (l > 0 || !fuse_in) RUN(KK_NORM, launch_ada_norm(n1, dt, st));
     const void* wqkv = (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es;
     if (p.use_tc_attn) {
       // QKV projection also writes V transposed (keys contiguous) for the tensor-core attention
@@ -392,16 +384,9 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
                   c.max_prefix, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim, c.mask_mode, p.O, p.qdim, p.err};
       RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
     }
-    const bool adapter_layer = adapters && (l + 1) % c.fop_adapter_every == 0;
-    GemmArgs go{p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, p.qdim, BH, D, p.qdim, EPI_ADD_F32, p.x,
-                D, DT_F32, nullptr};
-    go.max_splits = p.split_cap[1];
-    // (an adapter's update comes between the O projection and the second norm)
-    const RowNorm rn2{p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, p.cond_drow, B, H, nullptr, 0, nullptr, p.Y, H,
-                      p.gbar};
-    const bool n2_done = !adapter_layer && gemm_rownorm(go, rn2, KK_GEMM_O);
-    if (!n2_done) RUN(KK_GEMM_O, run_gemm(p, go, st));
-    if (adapter_layer) {
+    RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x,
+                        D, DT_F32, nullptr, p.split_cap[1]));
+    if (adapters && (l + 1) % c.fop_adapter_every == 0) {
       // gated cross-attention adapter: the action rows attend to the FOP tokens
       const int ai = (l + 1) / c.fop_adapter_every - 1, nkv = 2 * c.n_kv_heads * c.head_dim;
       NormArgs na{p.x, B, H, D, nullptr, 0, nullptr, 0, nullptr, 0, nullptr, p.Ya, H};
@@ -419,7 +404,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
                            p.x, D, DT_F32, nullptr));
     }
     NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
-    if (!n2_done) RUN(KK_NORM, launch_ada_norm(n2, dt, st));
+    RUN(KK_NORM, launch_ada_norm(n2, dt, st));
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
     GemmArgs gu{p.Y, D, wgu, D, BH, 2 * Fm, D, EPI_GEGLU, p.Hm, Fm, dt, nullptr};
     gu.max_splits = p.split_cap[2];
@@ -429,20 +414,11 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       RUN(KK_GEMM_GATE_UP, gemm(p.Y, D, wgu, BH, 2 * Fm, D, EPI_STORE, p.GU, 2 * Fm, DT_F32, nullptr));
       RUN(KK_GEGLU, launch_geglu(p.GU, BH, Fm, p.Hm, dt, st));
     }
-    GemmArgs gd{p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, Fm, BH, D, Fm, EPI_ADD_F32, p.x, D, DT_F32,
-                nullptr};
-    gd.max_splits = p.split_cap[3];
-    // the next layer's first norm (with its FOP rows), or the final norm
-    const RowNorm rn1 = l + 1 < L
-                            ? RowNorm{p.modv, p.mod_dim, p.mod_b, 4 * (l + 1) * D, p.cond_drow, B, H,
-                                      FF ? io.obs : nullptr, F, p.fop_gamma + (size_t)(l + 1) * D, p.Y, RPR, p.gbar}
-                            : RowNorm{p.modv, p.mod_dim, p.mod_b, 4 * L * D, p.cond_drow, B, H, nullptr, 0, nullptr,
-                                      p.Y, H, p.gbar};
-    y_ready = gemm_rownorm(gd, rn1, KK_GEMM_DOWN);
-    if (!y_ready) RUN(KK_GEMM_DOWN, run_gemm(p, gd, st));
+    RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D,
+                           DT_F32, nullptr, p.split_cap[3]));
   }
   NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
-  if (!y_ready) RUN(KK_NORM, launch_ada_norm(nf, dt, st));
+  RUN(KK_NORM, launch_ada_norm(nf, dt, st));
   RUN(KK_GEMM_OUT, gemm(p.Y, D, p.out_w, BH, A, D, EPI_STORE, p.V, A, DT_F32, p.out_b));
   if (dn) {
     RUN(KK_TAIL, launch_denoise_tail(io.buffer, p.V, io.velocity, B, H, A, dn->t_now, dn->t_next, st));

@@ -71,8 +71,7 @@ struct StepPlan {
   bool use_tc = false;      // bf16 projections on tcgen05
   float* dn_times = nullptr;   // [H] flow times of a synchronous denoising pass (all equal)
   float* rel_mask = nullptr;   // [A] 1 = a dimension the expert predicts relative to the robot state
-  int* gbar = nullptr;         // {count, generation}: grid-wide barrier of the row-norm GEMMs
-  bool fuse_norm = true;       // residual GEMMs of few tiles also write the next adaRMSNorm
+  bool fuse_norm = true;       // bf16: the in-projection also writes the first layer's first norm
   // FOP adapters (cfg.fop_adapter_every > 0): packed K-major weights, gains,
   // gates and their activations
   int n_adapters = 0;
@@ -95,6 +94,8 @@ enum KernelKind {
   KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_ADAPTER, KK_COUNT
 };
 const char* kernel_kind_name(int k);
+// The kernel kind whose launch failed last in enqueue_step on this thread (-1: none)
+int& enqueue_fail_kind();
 
 // Optional per-launch trace: an event recorded after every launch.
 struct LaunchTrace {

@@ -287,43 +287,6 @@ __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// Grid-wide barrier on a counter that only grows.  A launch adds exactly
-// kGridEpoch to it in total (the CTA with first = true adds
-// kGridEpoch - (nctas - 1), every other CTA 1), so between launches the
-// counter is a multiple of kGridEpoch, and a CTA reading it before its own
-// arrival finds the current multiple; it then waits for the next one.  One
-// thread per CTA, after a CTA-wide barrier that orders the CTA's stores
-// before the arrival; every CTA of the grid must be resident.  False after
-// kTcTimeoutNs without the last arrival.  (Unsigned wrap-around is harmless:
-// kGridEpoch divides 2^32.)
-constexpr unsigned kGridEpoch = 1u << 16;
-__device__ __forceinline__ bool grid_epoch_sync(unsigned* count, int nctas, bool first) {
-  unsigned cur;
-  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(cur) : "l"(count) : "memory");
-  const unsigned target = (cur & ~(kGridEpoch - 1)) + kGridEpoch;
-  __threadfence();
-  const unsigned inc = first ? kGridEpoch - (unsigned)(nctas - 1) : 1u;
-  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(count), "r"(inc) : "memory");
-  const unsigned long long t0 = globaltimer();
-  while (true) {
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(cur) : "l"(count) : "memory");
-    if ((int)(cur - target) >= 0) return true;
-    if (globaltimer() - t0 > kTcTimeoutNs) return false;
-  }
-}
-
-// 16-byte asynchronous copy global -> shared (through L2 only), and the wait
-// for all of this thread's copies
-__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
-// orders this thread's later generic-proxy accesses to shared memory after
-// the async proxy's earlier ones (TMA writes, tensor-core operand reads)
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
 // ---- thread-block clusters: rank, barrier, distributed shared memory
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
