@@ -185,7 +185,9 @@ __device__ __forceinline__ void xch_combine(uint32_t og, uint32_t ml, int r, int
 
 __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_constant__ AtMaps maps, AtParams p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  // 1024-byte aligned; derived from smem_raw by pointer arithmetic so that the
+  // compiler keeps it (and everything indexed from it) in the shared window
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int SK = p.k_slots, SV = p.v_slots;   // K and V^T ring depths
   const uint32_t k_bytes = (uint32_t)p.nblk * AT_KBLK;
   uint8_t* q_s = smem;
@@ -615,11 +617,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           else tmem_ld16_async(lane_base + o_col + 16 * chn, nxt);
         }
         if (snd) {
-#pragma unroll
-          for (int h = 0; h < 4; ++h) {   // groups of 8 columns
-            if (8 * h >= cw) break;
-            const int gidx = (cw / 8) * ch + h;
-            const int dst = gidx / ngs, gl = gidx - dst * ngs;
+          // groups of 8 columns: group g of the row goes to rank g / ngs, slot
+          // g % ngs there (one division per chunk, then a running count)
+          const int gidx0 = (cw / 8) * ch;
+          int dst = gidx0 / ngs, gl = gidx0 - dst * ngs;
+          auto send8 = [&](int h) {
             uint4 w;
             w.x = pack_bf16x2(__uint_as_float(cur[8 * h]) * inv, __uint_as_float(cur[8 * h + 1]) * inv);
             w.y = pack_bf16x2(__uint_as_float(cur[8 * h + 2]) * inv, __uint_as_float(cur[8 * h + 3]) * inv);
@@ -628,6 +630,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
             if (!has) w = make_uint4(0u, 0u, 0u, 0u);   // no key: the accumulator was never written
             st_async_u4(mapa_shared(o0 + (uint32_t)gl * (AT_BM * 16), (uint32_t)dst), w,
                         mapa_shared(bar0, (uint32_t)dst));
+            const bool wrap = ++gl == ngs;
+            gl = wrap ? 0 : gl;
+            dst += wrap ? 1 : 0;
+          };
+          send8(0);
+          send8(1);
+          if (cw == 32) {
+            send8(2);
+            send8(3);
           }
         }
         if (jj + 1 < nch) {

@@ -343,6 +343,25 @@ __device__ __forceinline__ bf16* vt_stage(const TcParams& p, uint8_t* boxes) {
 // shared memory (token-major, as the output), and thread 64 sends the box
 // with one TMA store (EPI_ADD_F32: TMA reduce-add into the residual stream);
 // rows past M and columns past N are clipped by the tensor map.
+// f(i) for i < n (n <= NV, a multiple of G), unrolled: without a bound
+// check when n == NV, else one per group of G (the epilogue warps run one per
+// scheduler, so every compare and branch in these loops is exposed latency)
+template <int NV, int G = 4, typename F>
+__device__ __forceinline__ void for_upto(int n, F&& f) {
+  static_assert(NV % G == 0, "whole groups");
+  if (n == NV) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) f(i);
+  } else {
+#pragma unroll
+    for (int g = 0; g < NV; g += G) {
+      if (g >= n) break;
+#pragma unroll
+      for (int i = g; i < g + G; ++i) f(i);
+    }
+  }
+}
+
 template <int EK, int NV = 16>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* tmO, int tile_n, int m0, int r,
                                              const float* v, float brow, uint8_t* boxes, float* xch, int& ebuf) {
@@ -360,21 +379,13 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   const bool vtile = kind == EK_BF16 && p.vt && (tile_n + 1) * TC_BM > p.v_col0;
   if (vtile) {   // this thread's row of the chunk, feature-major, for the V^T side output below
     uint32_t* vrow = (uint32_t*)(vt_stage(p, boxes) + (size_t)r * vpitch);
-#pragma unroll
-    for (int i = 0; i < NV; i += 2) {
-      if (i >= bm) break;
-      vrow[i / 2] = pack_bf16x2(v[i] + brow, v[i + 1] + brow);
-    }
+    for_upto<NV / 2, 2>((bm + 1) / 2, [&](int h) { vrow[h] = pack_bf16x2(v[2 * h] + brow, v[2 * h + 1] + brow); });
   }
   if (kind == EK_GEGLU) {
     // tile rows 0..63 are gate features, 64..127 the matching up features:
     // transpose through xch so that every thread then forms 8 outputs of one
     // token (the GELUs spread over all 128 threads)
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      if (i >= bm) break;
-      xch[i * STG_LD + r] = v[i] + brow;
-    }
+    for_upto<NV>(bm, [&](int i) { xch[i * STG_LD + r] = v[i] + brow; });
     epi_bar();
 #pragma unroll
     for (int h = 0; h < NV / 16; ++h) {
@@ -391,37 +402,17 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
       }
     }
   } else if (kind == EK_BF16) {
-    // (each loop stops at the box width: a short slice runs, and fetches,
-    // only its own iterations)
     bf16* o = (bf16*)box;
-    if (p.epi == EPI_STORE_SILU) {
-#pragma unroll
-      for (int i = 0; i < NV; ++i) {
-        if (i >= bm) break;
-        o[i * TC_BM + r] = __float2bfloat16_rn(silu_f(v[i] + brow));
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < NV; ++i) {
-        if (i >= bm) break;
-        o[i * TC_BM + r] = __float2bfloat16_rn(v[i] + brow);
-      }
-    }
+    if (p.epi == EPI_STORE_SILU)
+      for_upto<NV>(bm, [&](int i) { o[i * TC_BM + r] = __float2bfloat16_rn(silu_f(v[i] + brow)); });
+    else
+      for_upto<NV>(bm, [&](int i) { o[i * TC_BM + r] = __float2bfloat16_rn(v[i] + brow); });
   } else {
     float* o = (float*)box;
-    if (kind == EK_F32 && p.epi == EPI_STORE_SILU) {
-#pragma unroll
-      for (int i = 0; i < NV; ++i) {
-        if (i >= bm) break;
-        o[i * TC_BM + r] = silu_f(v[i] + brow);
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < NV; ++i) {
-        if (i >= bm) break;
-        o[i * TC_BM + r] = v[i] + brow;
-      }
-    }
+    if (kind == EK_F32 && p.epi == EPI_STORE_SILU)
+      for_upto<NV>(bm, [&](int i) { o[i * TC_BM + r] = silu_f(v[i] + brow); });
+    else
+      for_upto<NV>(bm, [&](int i) { o[i * TC_BM + r] = v[i] + brow; });
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   epi_bar();
@@ -458,7 +449,9 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                    const __grid_constant__ CUtensorMap tmO, TcParams p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  // 1024-byte aligned; derived from smem_raw by pointer arithmetic so that the
+  // compiler keeps it (and everything indexed from it) in the shared window
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int BN = p.bn, S = p.stages;
   const uint32_t b_bytes = (uint32_t)BN * TC_BK * 2;
   uint8_t* a_s = smem;
@@ -709,18 +702,15 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
           tmem_wait_ld();
 #pragma unroll
           for (int qq = 0; qq < 4; ++qq) tmem_reg_fence16(raw + 16 * qq);
-#pragma unroll
-          for (int qq = 0; qq < 16; ++qq) {
-            if (qq >= 4 * nq) break;
+          for_upto<16>(4 * nq, [&](int qq) {
             st_async_f4(mapa_shared(rcv0 + (uint32_t)gl * (TC_BM * 16), (uint32_t)dst),
                         make_float4(__uint_as_float(raw[4 * qq]), __uint_as_float(raw[4 * qq + 1]),
                                     __uint_as_float(raw[4 * qq + 2]), __uint_as_float(raw[4 * qq + 3])),
                         mapa_shared(bar0, (uint32_t)dst));
-            if (++gl == ngs) {
-              gl = 0;
-              ++dst;
-            }
-          }
+            const bool wrap = ++gl == ngs;   // next rank: a select, not a branch
+            gl = wrap ? 0 : gl;
+            dst += wrap ? 1 : 0;
+          });
         }
       } else if constexpr (RED == RED_L2_CLUSTER) {
         // this split's fp32 partial to the workspace as [col/4][row][4]: each
@@ -904,7 +894,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmO, TcParams p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  // 1024-byte aligned; derived from smem_raw by pointer arithmetic so that the
+  // compiler keeps it (and everything indexed from it) in the shared window
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int BN = p.bn, BNh = BN / 2, S = p.stages;
   const uint32_t bh_bytes = (uint32_t)BNh * TC_BK * 2;
   const uint32_t stage_tx = 2u * (TC_A_BYTES + bh_bytes);   // both CTAs' halves of a stage
