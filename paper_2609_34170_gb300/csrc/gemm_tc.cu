@@ -53,6 +53,7 @@ namespace {
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
 constexpr int TC_THREADS = 192;
+constexpr int TC_PAIR_THREADS = 320;   // pair kernel: TMA, MMA and two sets of four epilogue warps
 constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;
 constexpr int TC_SMEM_BUDGET = 200 * 1024;   // operand ring
 constexpr int TC_SMEM_MAX = 227 * 1024;
@@ -108,6 +109,7 @@ struct TcParams {
                         // nobody makes, so the launch gives up after wait_ns and unwinds
   const int* skip;      // optional device flag read after the dependency wait: nonzero -> the launch
                         // completes the copies it started and exits without computing
+  uint32_t set_bytes;   // pair kernel: bytes from epilogue set 0's boxes / exchange / V^T tile to set 1's
 };
 
 // The TMA epilogue kind of a launch (EK_F32 .. EK_GEGLU).
@@ -136,6 +138,11 @@ __device__ __forceinline__ bool work_item(const TcParams& p, int i, int& tn, int
 }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+// the 128 threads of epilogue warp set `set` (the pair kernel runs two sets)
+__device__ __forceinline__ void epi_bar_set(int set) {
+  if (set) asm volatile("bar.sync 2, 128;" ::: "memory");
+  else asm volatile("bar.sync 1, 128;" ::: "memory");
+}
 
 // v[4g + e] += sum over splits s = 0..S-1 (in order) of the partial of this
 // thread's row at column group g (g < NG); b0 points at split 0, group 0;
@@ -366,10 +373,14 @@ template <int EK, int NV = 16>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* tmO, int tile_n, int m0, int r,
                                              const float* v, float brow, uint8_t* boxes, float* xch, int& ebuf) {
   const int bm = p.box_m;   // <= NV
+  // epilogue warp set (threads 64..191: 0; 192..319: 1, pair kernel only) and
+  // the thread of the set that issues and waits for its TMA stores
+  const int set = threadIdx.x >= 192 ? 1 : 0;
+  const bool issuer = threadIdx.x == 64 + 128 * set;
   // the box written two chunks ago must have been read by its TMA store (and
   // every thread is done with the V^T tile of the previous chunk)
-  if (threadIdx.x == 64) bulk_wait_read<1>();
-  epi_bar();
+  if (issuer) bulk_wait_read<1>();
+  epi_bar_set(set);
   uint8_t* box = boxes + (size_t)ebuf * p.box_bytes;
   const int vpitch = bm + 10;   // bf16 per V^T tile row: an odd number of words, no bank conflicts
   // V^T side output through a transposed staging tile (below); one path for
@@ -386,7 +397,7 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
     // transpose through xch so that every thread then forms 8 outputs of one
     // token (the GELUs spread over all 128 threads)
     for_upto<NV>(bm, [&](int i) { xch[i * STG_LD + r] = v[i] + brow; });
-    epi_bar();
+    epi_bar_set(set);
 #pragma unroll
     for (int h = 0; h < NV / 16; ++h) {
       const int c = (r >> 3) + 16 * h, fg = r & 7;
@@ -415,8 +426,8 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
       for_upto<NV>(bm, [&](int i) { o[i * TC_BM + r] = v[i] + brow; });
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  epi_bar();
-  if (threadIdx.x == 64) {
+  epi_bar_set(set);
+  if (issuer) {
     if (kind == EK_ADD) tma_reduce_add_2d(tmO, box, tile_n * TC_BM, m0);
     else tma_store_2d(tmO, box, kind == EK_GEGLU ? tile_n * 64 : tile_n * TC_BM, m0);
     bulk_commit();
@@ -890,7 +901,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
 // both CTAs run the epilogue of their own rows, whose drained accumulators
 // the even CTA's `acc_empty` counts (256 arrivals).
 template <int EK>
-__global__ void __launch_bounds__(TC_THREADS, 1)
+__global__ void __launch_bounds__(TC_PAIR_THREADS, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmO, TcParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -907,7 +918,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   uint64_t* full = (uint64_t*)(smem + p.bar_off);   // the even CTA's count both halves
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;      // [2]
-  uint64_t* acc_empty = acc_full + 2;  // [2] the even CTA's: 256 arrivals
+  uint64_t* acc_empty = acc_full + 2;  // [2] the even CTA's: 512 arrivals (256 epilogue threads per CTA)
   uint32_t* tmem_slot = (uint32_t*)(acc_empty + 2);
   int* flags = (int*)(tmem_slot + 1);  // [0] abort, [2] stages issued, [3] stages consumed
 
@@ -938,7 +949,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 256);
+      mbar_init(&acc_empty[b], 512);
     }
     flags[0] = flags[1] = flags[2] = flags[3] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1044,9 +1055,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     __syncwarp();
   } else {
-    // epilogue warps 2..5 of both CTAs: TMEM lane quarter q, this CTA's tile row r
+    // epilogue warps 2..9 of both CTAs: TMEM lane quarter q, this CTA's tile
+    // row r; set 0 (warps 2..5) takes the 32-token chunks 0, 2, 4, ..., set 1
+    // (warps 6..9) chunks 1, 3, 5, ..., each with its own boxes and barrier
     const int q = warp & 3;
     const int r = q * 32 + lane;
+    const int set = warp >= 6 ? 1 : 0;
+    uint8_t* sboxes = stg_raw + (size_t)set * p.set_bytes;
+    float* sxch = (float*)((uint8_t*)xch + (size_t)set * p.set_bytes);
     int ebuf = 0;
     int tn2, tm;
     for (int i = 0; item(i, tn2, tm); ++i) {
@@ -1062,25 +1078,26 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const int m_base = tm * BN;
       const int n = tile_n * TC_BM + r;
       const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
-      // 32-token chunks (BN is a multiple of 32): half the barriers and box
-      // hand-offs per token of 16-token chunks
+      // 32-token chunks (BN is a multiple of 32, at least 128): this set's
+      // every other chunk, the next one's TMEM load in flight meanwhile
       uint32_t nxt[32];
-      tmem_ld32_async(trow, nxt);
+      const int cf = 32 * set;
+      tmem_ld32_async(trow + cf, nxt);
       tmem_wait_ld();
       tmem_reg_fence16(nxt);
       tmem_reg_fence16(nxt + 16);
-      for (int c0 = 0; c0 < BN; c0 += 32) {
+      for (int c0 = cf; c0 < BN; c0 += 64) {
         float v[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(nxt[k]);
-        const bool more = c0 + 32 < BN;
+        const bool more = c0 + 64 < BN;
         if (more) {
-          tmem_ld32_async(trow + c0 + 32, nxt);
-        } else {   // this CTA's accumulator drained: tell the MMA issuer
+          tmem_ld32_async(trow + c0 + 64, nxt);
+        } else {   // this thread is done with the accumulator: tell the MMA issuer
           tc_fence_before();
           mbar_arrive_remote(acc_empty0 + 8u * (uint32_t)b);
         }
-        epilogue_tma<EK, 32>(p, &tmO, tile_n, m_base + c0, r, v, brow, stg_raw, xch, ebuf);
+        epilogue_tma<EK, 32>(p, &tmO, tile_n, m_base + c0, r, v, brow, sboxes, sxch, ebuf);
         if (more) {
           tmem_wait_ld();
           tmem_reg_fence16(nxt);
@@ -1088,7 +1105,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
       }
     }
-    if (threadIdx.x == 64) bulk_wait<0>();
+    if (threadIdx.x == 64 + 128 * set) bulk_wait<0>();   // this set's stores are complete
   }
   tc_fence_before();
   cta_sync();
@@ -1253,7 +1270,9 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
   const size_t stg_bytes = 2 * (size_t)box_bytes;
   const size_t xch_bytes = g.epi == EPI_GEGLU ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
   const size_t vts_bytes = g.vt ? ((size_t)TC_BM * (box_m + 10) * 2 + 1023) / 1024 * 1024 : 0;
-  const size_t fixed = 1024 + stg_bytes + xch_bytes + vts_bytes + 256;
+  // each of the two epilogue warp sets has its own boxes, exchange tile and V^T tile
+  const size_t set_bytes = stg_bytes + xch_bytes + vts_bytes;
+  const size_t fixed = 1024 + 2 * set_bytes + 256;
   const int stage_bytes = TC_A_BYTES + (bn / 2) * TC_BK * 2;
   const int stages = std::min(8, (int)((TC_SMEM_MAX - fixed) / stage_bytes));
   if (stages < 2) return cudaErrorInvalidConfiguration;
@@ -1261,7 +1280,7 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
   const uint32_t stg_off = (uint32_t)ring;
   const uint32_t xch_off = stg_off + (uint32_t)stg_bytes;
   const uint32_t vts_off = xch_off + (uint32_t)xch_bytes;
-  const uint32_t bar_off = vts_off + (uint32_t)vts_bytes;
+  const uint32_t bar_off = stg_off + 2 * (uint32_t)set_bytes;
   const size_t smem = 1024 + bar_off + (size_t)(2 * stages + 4) * 8 + 4 + 16 + 64;
   if (smem > (size_t)TC_SMEM_MAX) return cudaErrorInvalidConfiguration;
   CUtensorMap mw, mx, mo;
@@ -1275,9 +1294,10 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
              (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
              g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, 1, 0, box_m, box_bytes, stg_off, xch_off,
              vts_off, 0, bar_off, kTcTimeoutNs, 0, g.skip};
+  p.set_bytes = (uint32_t)set_bytes;
   const int npairs = std::min(num_tiles, slots);
-  return launch_kernel_cluster(tc_pair_kernel(ek), dim3(2 * npairs), dim3(TC_THREADS), smem, st, dim3(2, 1, 1), mw, mx,
-                               mo, p);
+  return launch_kernel_cluster(tc_pair_kernel(ek), dim3(2 * npairs), dim3(TC_PAIR_THREADS), smem, st, dim3(2, 1, 1),
+                               mw, mx, mo, p);
 }
 
 }  // namespace
