@@ -442,12 +442,12 @@ cudaError_t launch_ada_norm_t(const NormArgs& a, cudaStream_t st) {
   }
   const int G = (a.D + 1023) / 1024;
   const int R = (G >= 4) ? 1 : 4 / G;
-  // rows per block: enough blocks for every SM, in whole batches of R rows
-  // rows per block: all rows (action + FOP) over about three resident blocks
-  // per SM, in whole batches of R rows -- few serial batches per block
+  // rows per block: one batch of R rows, so that every block's loads are in
+  // flight at once (a block that walks several batches pays one L2 round
+  // trip per batch); up to 8 blocks of 256 threads are resident per SM
   const int nf = a.fop ? a.F : 0;
   const int total = a.B * (a.H + nf);
-  int rb_all = (total + 3 * g_norm_sms - 1) / (3 * g_norm_sms);
+  int rb_all = (total + 8 * g_norm_sms - 1) / (8 * g_norm_sms);
   rb_all = (rb_all + R - 1) / R * R;
   auto rows_per_block = [&](int rows_per_robot) { return std::max(R, std::min(rb_all, rows_per_robot)); };
   const int rb_act = rows_per_block(a.H), nb_act = (a.H + rb_act - 1) / rb_act;
