@@ -224,6 +224,8 @@ int ravel_step_kernel_count(const ravel_t* r);
  * [cap] (kind id, see ravel_kernel_kind_name); *n_launches receives the
  * number of launches (entries beyond cap are dropped).  The stream is first
  * held for ~5 ms so that all launches are queued before the first one starts.
+ * The step's launches are followed by 16 launches of an empty kernel, timed
+ * the same way (kind "launch_gap"): the overhead every interval holds.
  * Synchronous. */
 ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_times, const void* obs_tokens,
                                 const float* delta, float* released, float* velocity, void* stream,

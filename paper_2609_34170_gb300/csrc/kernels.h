@@ -143,6 +143,9 @@ cudaError_t launch_in_proj_norm(const float* buf, int A, int D, const float* in_
                                 const float* state, const float* rel_mask, const float* slot_times, const RowNorm& rn,
                                 Dtype dt, cudaStream_t st);
 
+// An empty kernel (one thread): the launch overhead of a timed eager replay.
+cudaError_t launch_noop(cudaStream_t st);
+
 // ---- GeGLU on the interleaved gate/up GEMM output --------------------------------
 cudaError_t launch_geglu(const float* GU, int M, int Fm, void* Hm, Dtype dt, cudaStream_t st);
 

@@ -585,6 +585,10 @@ cudaError_t launch_in_proj_norm(const float* buf, int A, int D, const float* in_
                        in_b, x, state, rel_mask, slot_times, rn);
 }
 
+__global__ void noop_kernel() {}
+
+cudaError_t launch_noop(cudaStream_t st) { return launch_kernel(noop_kernel, dim3(1), dim3(1), 0, st, 1); }
+
 // ============================================================================ GeGLU
 
 template <typename T>

@@ -414,6 +414,18 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
   int nk = 0;
   StepIO io{buffer, slot_times, obs_tokens, delta, released, velocity};
   if (e == cudaSuccess) e = enqueue_step(r->plan, r->batch, io, st, &nk, &tr);
+  // then 16 empty kernels timed the same way: the per-launch overhead that
+  // every interval above also holds (kind KK_LAUNCH_GAP)
+  for (int i = 0; i < 16 && e == cudaSuccess; ++i) {
+    e = launch_noop(st);
+    cudaEvent_t ev;
+    if (e == cudaSuccess) e = cudaEventCreate(&ev);
+    if (e == cudaSuccess) {
+      tr.events.push_back(ev);
+      tr.kinds.push_back(KK_LAUNCH_GAP);
+      e = cudaEventRecord(ev, st);
+    }
+  }
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   int n = 0;
   cudaEvent_t prev = start;

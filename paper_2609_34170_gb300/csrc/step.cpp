@@ -275,7 +275,7 @@ int& enqueue_fail_kind() {
 const char* kernel_kind_name(int k) {
   static const char* const names[KK_COUNT] = {"embed", "gemm_cond", "gemm_mod", "in_proj", "norm", "gemm_qkv",
                                               "attention", "gemm_o", "gemm_gate_up", "geglu", "gemm_down",
-                                              "gemm_out", "tail", "cond_cache", "adapter"};
+                                              "gemm_out", "tail", "cond_cache", "adapter", "launch_gap"};
   return (k >= 0 && k < KK_COUNT) ? names[k] : "unknown";
 }
 

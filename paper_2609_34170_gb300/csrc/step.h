@@ -91,7 +91,9 @@ void plan_destroy(StepPlan* p);
 // Kernel kinds of one step (per-launch profiling labels).
 enum KernelKind {
   KK_EMBED = 0, KK_GEMM_COND, KK_GEMM_MOD, KK_IN_PROJ, KK_NORM, KK_GEMM_QKV, KK_ATTENTION, KK_GEMM_O,
-  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_ADAPTER, KK_COUNT
+  KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_ADAPTER,
+  KK_LAUNCH_GAP,   // an empty kernel timed like the step's launches (ravel_profile_step)
+  KK_COUNT
 };
 const char* kernel_kind_name(int k);
 // The kernel kind whose launch failed last in enqueue_step on this thread (-1: none)
