@@ -118,13 +118,19 @@ def kind_work(kind, cfg, B, P):
         return (md * D + (H + B) * D) * es + (H + B) * md * 4, 2 * (H + B) * D * md
     if kind == "norm":
         # average over a step's norm launches: L - 1 first norms with the FOP
-        # rows (layer 0's is written by the in-projection), L second norms
-        # and the final norm; each reads x, the slot and robot modulation rows
-        # and the shift/scale bias, and writes Y (+ the FOP rows' z and gain)
+        # rows (layer 0's is written by the in-projection) and L second norms
+        # (the final norm is part of head_tail); each reads x, the slot and
+        # robot modulation rows and the shift/scale bias, and writes Y (+ the
+        # FOP rows' z and gain)
         L = cfg.layers
         plain = BH * D * 4 + (H + B) * 2 * D * 4 + 2 * D * 4 + BH * D * es
         fop = plain + 2 * B * F * D * es + D * 4
-        return ((L - 1) * fop + (L + 1) * plain) / (2 * L), 0
+        return ((L - 1) * fop + L * plain) / (2 * L - 1), 0
+    if kind == "head_tail":
+        # final norm (x, modulation rows, bias), W_out and b_out, the buffer
+        # read and written, the released actions and the velocity rows
+        return (BH * D * 4 + (H + B) * 2 * D * 4 + 2 * D * 4 + A * D * es + A * 4 + 2 * BH * A * 4 + B * A * 4
+                + BH * A * 4), 2 * BH * D * A
     if kind == "attention":
         kv = B * cfg.n_kv_heads * P * cfg.head_dim * 2 * es
         return kv + (BY * nqkv + BH * qd) * es, 4 * B * cfg.n_q_heads * H * (P + F + H) * cfg.head_dim

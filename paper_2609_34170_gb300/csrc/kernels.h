@@ -206,6 +206,19 @@ struct TailArgs {
 };
 cudaError_t launch_tail(const TailArgs& a, cudaStream_t st);
 
+// The final adaRMSNorm, the velocity head and the tail in one launch (bf16
+// weights, A <= 32): rows_per_cta slots of one robot per CTA write v = the
+// head of their normed rows into a.vel; the robot's last CTA runs the tail.
+struct HeadArgs {
+  const float* x; int D;                       // residual stream [B*H][D]
+  const float* modv; int mod_ld; const float* mod_b; int off; const int* drow;   // as NormArgs
+  const void* w; const float* b;               // W_out [A][D] bf16, b_out [A]
+  float* v;                                    // [B*H][A] velocity (= a.vel)
+  int* cnt;                                    // [B] zero-initialised counters
+  int rows_per_cta;
+};
+cudaError_t launch_head_tail(const HeadArgs& h, const TailArgs& a, cudaStream_t st);
+
 // Synchronous (full-horizon) denoising: buffer += (t_now - t_next) * vel for
 // every slot (vel_out optional copy); times[0..H-1] = t; a fresh chunk
 // buffer[b][j] = noise(seeds[b], counters[b] + j), counters[b] += H.

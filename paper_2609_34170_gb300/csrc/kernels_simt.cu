@@ -819,11 +819,9 @@ cudaError_t launch_fop_xattn(const void* Q, const void* KV, void* out, int B, in
 // One CTA per robot: a'_j = a_j + dt_j v_j (Eq. 3), released = a'_0, buffer
 // slots shift forward, the last slot receives the Gaussian action of index
 // counters[b], and the counter advances.
-__global__ void tail_kernel(TailArgs a) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ float sa[];   // [H][A]
-  const int b = blockIdx.x;
+// Euler step, release, shift and noise append of robot b (Eq. 3 and the roll
+// after it), by the whole block; sa: H*A floats of shared memory.
+__device__ void tail_robot(const TailArgs& a, int b, float* sa) {
   const int H = a.H, A = a.A;
   float* buf = a.buffer + (size_t)b * H * A;
   const float* v = a.vel + (size_t)b * H * A;
@@ -834,9 +832,10 @@ __global__ void tail_kernel(TailArgs a) {
     const float dt = __fsub_rn(t1, t0);
     // absolute buffer, relative expert: the slot also moves by dt m s as its
     // flow time drops from t_j to t_{j-1}
-    const float vv = a.state ? fmaf(a.rel_mask[i % A], a.state[(size_t)b * A + i % A], v[i]) : v[i];
+    const float vi = __ldcg(v + i);   // (written by other CTAs of the fused head kernel)
+    const float vv = a.state ? fmaf(a.rel_mask[i % A], a.state[(size_t)b * A + i % A], vi) : vi;
     sa[i] = fmaf(dt, vv, buf[i]);
-    if (a.vel_out) a.vel_out[(size_t)b * H * A + i] = v[i];
+    if (a.vel_out) a.vel_out[(size_t)b * H * A + i] = vi;
   }
   __syncthreads();
   for (int i = threadIdx.x; i < H * A; i += blockDim.x) {
@@ -856,10 +855,126 @@ __global__ void tail_kernel(TailArgs a) {
   if (threadIdx.x == 0) a.counters[b] = n + 1;
 }
 
+__global__ void tail_kernel(TailArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ float sa[];   // [H][A]
+  tail_robot(a, blockIdx.x, sa);
+}
+
 cudaError_t launch_tail(const TailArgs& a, cudaStream_t st) {
   if (a.B <= 0) return cudaSuccess;
   const size_t smem = (size_t)a.H * a.A * sizeof(float);
   return launch_kernel(tail_kernel, dim3(a.B), dim3(256), smem, st, 1, a);
+}
+
+// The step's last three stages in one launch (bf16 mode, A <= 32): the final
+// adaRMSNorm of each action row (Eq. 2's modulation, offset fin_off), the
+// velocity head v = Y W_out^T + b_out on the bf16-rounded normed row (as the
+// separate norm + GEMM compute it), and, by the CTA of each robot that
+// finishes last, the Euler step, release, shift and noise append (tail_robot).
+// A CTA owns rows_per_cta slots of one robot; the robot's CTAs count their
+// finished rows on cnt[b] (reset by the last one, so it is zero between
+// launches), the classic last-block pattern: no CTA waits for another.
+template <bool FULL>   // FULL: A == 32
+__global__ void __launch_bounds__(256) head_tail_kernel(HeadArgs h, TailArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[8][33];     // per-warp sums: [warp][output] (+ the norm's row sum in [w][32])
+  __shared__ int last;
+  extern __shared__ float sa[];    // [H][A], the last CTA's tail
+  const int nb = (a.H + h.rows_per_cta - 1) / h.rows_per_cta;
+  const int b = blockIdx.x / nb, j0 = (blockIdx.x % nb) * h.rows_per_cta;
+  const int j1 = min(a.H, j0 + h.rows_per_cta);
+  const int D = h.D, A = a.A, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* md = h.modv + (size_t)(h.drow ? h.drow[b] : a.H + b) * h.mod_ld + h.off;
+  const float* mb = h.mod_b + h.off;
+  for (int j = j0; j < j1; ++j) {
+    const float* xr = h.x + (size_t)(b * a.H + j) * D;
+    const float* mt = h.modv + (size_t)j * h.mod_ld + h.off;
+    // sum of squares of the row (4 features per thread per pass)
+    float ss = 0.f;
+    for (int f = 4 * threadIdx.x; f < D; f += 4 * blockDim.x) {
+      const float4 xv = *(const float4*)(xr + f);
+      ss += xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w;
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) red[warp][32] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w][32];
+    const float inv = rsqrtf(tot / (float)D + 1e-6f);
+    // this thread's partial products for all 32 outputs
+    float acc[32];
+#pragma unroll
+    for (int o = 0; o < 32; ++o) acc[o] = 0.f;
+    for (int f = 4 * threadIdx.x; f < D; f += 4 * blockDim.x) {
+      const float4 xv = *(const float4*)(xr + f);
+      const float4 t0 = *(const float4*)(mt + f), t1 = *(const float4*)(mt + D + f);
+      const float4 d0 = *(const float4*)(md + f), d1 = *(const float4*)(md + D + f);
+      const float4 b0 = *(const float4*)(mb + f), b1 = *(const float4*)(mb + D + f);
+      const float xs[4] = {xv.x, xv.y, xv.z, xv.w};
+      const float sc[4] = {t0.x + d0.x + b0.x, t0.y + d0.y + b0.y, t0.z + d0.z + b0.z, t0.w + d0.w + b0.w};
+      const float sh[4] = {t1.x + d1.x + b1.x, t1.y + d1.y + b1.y, t1.z + d1.z + b1.z, t1.w + d1.w + b1.w};
+      float y[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) y[e] = __bfloat162float(__float2bfloat16_rn(xs[e] * inv * (1.f + sc[e]) + sh[e]));
+#pragma unroll
+      for (int o = 0; o < 32; ++o) {
+        if (FULL || o < A) {
+          const uint2 wq = *(const uint2*)((const bf16*)h.w + (size_t)o * D + f);   // 4 bf16 of W_out row o
+          acc[o] = fmaf(y[0], __uint_as_float(wq.x << 16), acc[o]);
+          acc[o] = fmaf(y[1], __uint_as_float(wq.x & 0xFFFF0000u), acc[o]);
+          acc[o] = fmaf(y[2], __uint_as_float(wq.y << 16), acc[o]);
+          acc[o] = fmaf(y[3], __uint_as_float(wq.y & 0xFFFF0000u), acc[o]);
+        }
+      }
+    }
+    // warp: lane o ends with the warp's sum of output o (each step keeps half
+    // of the outputs and adds the partner's half)
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      const bool up = (lane & off) != 0;
+#pragma unroll
+      for (int i = 0; i < off; ++i) {
+        const float send = up ? acc[i] : acc[i + off];
+        const float keep = up ? acc[i + off] : acc[i];
+        acc[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+      }
+    }
+    red[warp][lane] = acc[0];
+    __syncthreads();
+    if (threadIdx.x < A) {
+      float v = h.b[threadIdx.x];
+#pragma unroll
+      for (int w = 0; w < 8; ++w) v += red[w][threadIdx.x];
+      h.v[(size_t)(b * a.H + j) * A + threadIdx.x] = v;
+    }
+    __syncthreads();   // red is reused by the next row
+  }
+  // the robot's last CTA to finish runs the tail
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int done = atomicAdd(h.cnt + b, 1);
+    last = done == nb - 1;
+    if (last) h.cnt[b] = 0;
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  tail_robot(a, b, sa);
+}
+
+cudaError_t launch_head_tail(const HeadArgs& h, const TailArgs& a, cudaStream_t st) {
+  if (a.B <= 0) return cudaSuccess;
+  const size_t smem = (size_t)a.H * a.A * sizeof(float);
+  if (a.A > 32 || h.D % 4 || smem > 48 * 1024) return cudaErrorNotSupported;
+  const int nb = (a.H + h.rows_per_cta - 1) / h.rows_per_cta;
+  if (a.A == 32)
+    return launch_kernel(head_tail_kernel<true>, dim3(a.B * nb), dim3(256), smem, st, 1, h, a);
+  return launch_kernel(head_tail_kernel<false>, dim3(a.B * nb), dim3(256), smem, st, 1, h, a);
 }
 
 // Full-horizon denoising (the synchronous baseline): every slot takes the

@@ -151,6 +151,7 @@ ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* bu
   // a new rollout starts with an empty conditioning cache (its rows are then
   // computed at this batch size only)
   RV_CUDA(r, cudaMemset(r->plan.cond, 0, sizeof(CondCache)), "reset: clear conditioning cache");
+  RV_CUDA(r, cudaMemset(r->plan.head_cnt, 0, sizeof(int) * r->plan.cfg.max_batch), "reset: clear head counters");
   *r->err_host = 0;
   RV_CUDA(r, cudaMemcpy(r->plan.seeds, seeds, sizeof(uint64_t) * batch, cudaMemcpyHostToDevice), "reset: seeds");
   RV_CUDA(r, launch_reset(buffer, r->plan.seeds, r->plan.counters, batch, r->plan.cfg.slots,

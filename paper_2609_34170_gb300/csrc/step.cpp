@@ -168,6 +168,7 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   }
   AL(p->seeds, Bm * sizeof(uint64_t));
   AL(p->counters, Bm * sizeof(uint64_t));
+  AL(p->head_cnt, Bm * sizeof(int));
   AL(p->err, sizeof(int));
 #undef AL
   p->tcws.err = p->err;
@@ -275,7 +276,8 @@ int& enqueue_fail_kind() {
 const char* kernel_kind_name(int k) {
   static const char* const names[KK_COUNT] = {"embed", "gemm_cond", "gemm_mod", "in_proj", "norm", "gemm_qkv",
                                               "attention", "gemm_o", "gemm_gate_up", "geglu", "gemm_down",
-                                              "gemm_out", "tail", "cond_cache", "adapter", "launch_gap"};
+                                              "gemm_out", "tail", "cond_cache", "adapter", "head_tail",
+                                              "launch_gap"};
   return (k >= 0 && k < KK_COUNT) ? names[k] : "unknown";
 }
 
@@ -416,6 +418,16 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     }
     RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D,
                            DT_F32, nullptr, p.split_cap[3]));
+  }
+  if (!dn && dt == DT_BF16 && A <= 32 && D % 4 == 0) {
+    // final norm, velocity head and tail in one launch, about eight CTAs per SM
+    TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A, io.state,
+                p.rel_mask};
+    const int rpc = std::max(1, (B * H + 8 * p.num_sms - 1) / (8 * p.num_sms));
+    HeadArgs hd{p.x, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, p.cond_drow, p.out_w, p.out_b, p.V, p.head_cnt, rpc};
+    RUN(KK_HEAD_TAIL, launch_head_tail(hd, ta, st));
+    if (n_kernels) *n_kernels = nk;
+    return e;
   }
   NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
   RUN(KK_NORM, launch_ada_norm(nf, dt, st));

@@ -49,6 +49,7 @@ struct StepPlan {
   CondCache* cond = nullptr;   // steady-state conditioning cache (kernels.h)
   float* cond_tkey = nullptr;  // [H]
   int* cond_drow = nullptr;    // [Bmax]
+  int* head_cnt = nullptr;     // [Bmax] finished-row counters of the fused head kernel (zero between launches)
   int* cond_commit = nullptr;  // [2 Bmax]
   bool cond_cache = true;
   float* x = nullptr;     // [Bmax*H][D]  residual stream
@@ -92,6 +93,7 @@ void plan_destroy(StepPlan* p);
 enum KernelKind {
   KK_EMBED = 0, KK_GEMM_COND, KK_GEMM_MOD, KK_IN_PROJ, KK_NORM, KK_GEMM_QKV, KK_ATTENTION, KK_GEMM_O,
   KK_GEMM_GATE_UP, KK_GEGLU, KK_GEMM_DOWN, KK_GEMM_OUT, KK_TAIL, KK_COND_CACHE, KK_ADAPTER,
+  KK_HEAD_TAIL,    // final norm + velocity head + tail in one launch (bf16)
   KK_LAUNCH_GAP,   // an empty kernel timed like the step's launches (ravel_profile_step)
   KK_COUNT
 };
