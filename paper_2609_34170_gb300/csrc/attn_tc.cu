@@ -137,16 +137,22 @@ __device__ __forceinline__ float2 lds_f2(uint32_t a) {
   return v;
 }
 
-// Merge of this thread's row over the SP splits' shares received in shared
-// memory (O groups [s][g][row] of 8 bf16 from `og`, (m, l) [s][row] from
-// `ml`, both shared-memory addresses of row 0): head-dim groups g < ngs of
-// slice q, columns q*8*ngs + 8g, stored as bf16 (columns past hd skipped).
+// Merge of row r, head-dim group gq, over the SP splits' shares received in
+// shared memory (O groups [s][g][row] of 8 bf16 from `og`, (m, l) [s][row]
+// from `ml`, both shared-memory addresses of row 0): columns d0 + 8 gq .. +7
+// of slice q, stored as bf16 (a group past hd is skipped).
 //   O = sum_s 2^(m_s - M) l_s Ohat_s / sum_s 2^(m_s - M) l_s
 template <int SP>
-__device__ __forceinline__ void xch_combine(uint32_t og, uint32_t ml, int r, int ngs, int d0, int hd, bf16* orow) {
+__device__ __forceinline__ void xch_combine_group(uint32_t og, uint32_t ml, int r, int ngs, int gq, int d0, int hd,
+                                                  bf16* orow) {
+  const int d = d0 + 8 * gq;
+  if (d >= hd) return;
   float2 v[SP];
 #pragma unroll
   for (int s2 = 0; s2 < SP; ++s2) v[s2] = lds_f2(ml + (uint32_t)(s2 * AT_BM + r) * 8u);
+  uint4 u[SP];
+#pragma unroll
+  for (int s2 = 0; s2 < SP; ++s2) u[s2] = lds_u4(og + ((uint32_t)(s2 * ngs + gq) * AT_BM + r) * 16u);
   float M = -INFINITY;
 #pragma unroll
   for (int s2 = 0; s2 < SP; ++s2) M = fmaxf(M, v[s2].x);
@@ -158,29 +164,21 @@ __device__ __forceinline__ void xch_combine(uint32_t og, uint32_t ml, int r, int
     L += w[s2];
   }
   const float inv = L > 0.f ? 1.f / L : 0.f;
+  float acc[8];
 #pragma unroll
-  for (int s2 = 0; s2 < SP; ++s2) w[s2] *= inv;
-  for (int gq = 0; gq < ngs; ++gq) {
-    const int d = d0 + 8 * gq;
-    if (d >= hd) break;
-    uint4 u[SP];
+  for (int k = 0; k < 8; ++k) acc[k] = 0.f;
 #pragma unroll
-    for (int s2 = 0; s2 < SP; ++s2) u[s2] = lds_u4(og + ((uint32_t)(s2 * ngs + gq) * AT_BM + r) * 16u);
-    float acc[8];
+  for (int s2 = 0; s2 < SP; ++s2) {
+    const float ws = w[s2] * inv;
+    const uint32_t uu[4] = {u[s2].x, u[s2].y, u[s2].z, u[s2].w};
 #pragma unroll
-    for (int k = 0; k < 8; ++k) acc[k] = 0.f;
-#pragma unroll
-    for (int s2 = 0; s2 < SP; ++s2) {
-      const uint32_t uu[4] = {u[s2].x, u[s2].y, u[s2].z, u[s2].w};
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        acc[2 * k] = fmaf(w[s2], __uint_as_float(uu[k] << 16), acc[2 * k]);
-        acc[2 * k + 1] = fmaf(w[s2], __uint_as_float(uu[k] & 0xFFFF0000u), acc[2 * k + 1]);
-      }
+    for (int k = 0; k < 4; ++k) {
+      acc[2 * k] = fmaf(ws, __uint_as_float(uu[k] << 16), acc[2 * k]);
+      acc[2 * k + 1] = fmaf(ws, __uint_as_float(uu[k] & 0xFFFF0000u), acc[2 * k + 1]);
     }
-    *(uint4*)(orow + d) = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]),
-                                     pack_bf16x2(acc[4], acc[5]), pack_bf16x2(acc[6], acc[7]));
   }
+  *(uint4*)(orow + d) = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]),
+                                   pack_bf16x2(acc[4], acc[5]), pack_bf16x2(acc[6], acc[7]));
 }
 
 __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_constant__ AtMaps maps, AtParams p) {
@@ -690,23 +688,27 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     // split's share has arrived (the wait also keeps this CTA alive until no
     // store into its shared memory is in flight):
     //   O = sum_s 2^(m_s - M) l_s Ohat_s / sum_s 2^(m_s - M) l_s,  Ohat_s = O_s / l_s.
-    if (warp >= 2) {
-      const int r = (warp & 3) * 32 + lane;
+    // Every warp takes part (the producer and MMA warps are idle by now):
+    // work item (row r, 8-column group gq) of this rank's slice.
+    {
       const bool ok = __all_sync(0xffffffffu, mbar_wait_cluster(rcv_bar, 0));
       if (!ok) {
         if (lane == 0) raise_error(p.err, ERR_TIMEOUT);
-      } else if (r < vrows) {
-        const int ngs = cps / 8;
+      } else {
+        const int ngs = cps / 8, items = vrows * ngs;
         const uint32_t og = smem_u32(smem);
         const uint32_t ml = og + (uint32_t)(p.splits * ngs * AT_BM) * 16u;
-        const int t = r / p.G, hh = r % p.G;
-        const int j = qt * p.TQ + t;
-        bf16* orow = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
-        switch (p.splits) {
-          case 2: xch_combine<2>(og, ml, r, ngs, split * cps, p.hd, orow); break;
-          case 4: xch_combine<4>(og, ml, r, ngs, split * cps, p.hd, orow); break;
-          case 8: xch_combine<8>(og, ml, r, ngs, split * cps, p.hd, orow); break;
-          default: xch_combine<16>(og, ml, r, ngs, split * cps, p.hd, orow); break;
+        for (int it = threadIdx.x; it < items; it += AT_THREADS) {
+          const int r = it % vrows, gq = it / vrows;
+          const int t = r / p.G, hh = r % p.G;
+          const int j = qt * p.TQ + t;
+          bf16* orow = p.out + (size_t)(b * p.H + j) * p.ld_out + (size_t)(g * p.G + hh) * p.hd;
+          switch (p.splits) {
+            case 2: xch_combine_group<2>(og, ml, r, ngs, gq, split * cps, p.hd, orow); break;
+            case 4: xch_combine_group<4>(og, ml, r, ngs, gq, split * cps, p.hd, orow); break;
+            case 8: xch_combine_group<8>(og, ml, r, ngs, gq, split * cps, p.hd, orow); break;
+            default: xch_combine_group<16>(og, ml, r, ngs, gq, split * cps, p.hd, orow); break;
+          }
         }
       }
     }
