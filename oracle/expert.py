@@ -150,7 +150,9 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
     """v_theta(A, t, c, delta) for B robots: [B, H, A] float64 (Eq. 3's velocity).
 
     buffer [B, H, A]; slot_times [H]; ctx_k / ctx_v [L, B, Hkv, >=prefix_len, hd];
-    fop [B, F, D]; delta [B].  ``trace`` (optional dict) receives intermediates.
+    fop [B, F, D]; delta [B].  prefix_len: one valid prefix length for every
+    robot, or one per robot ([B]: robots whose contexts arrived at different
+    times, Sec. 3.2).  ``trace`` (optional dict) receives intermediates.
     """
     B, H, A = buffer.shape
     D, L = cfg.width, cfg.layers
@@ -158,19 +160,21 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
     G = Hq // Hkv
     adapters = getattr(cfg, "fop_adapter_every", 0) > 0
     F = 0 if adapters else fop.shape[1]   # FOP keys of the self-attention
-    P = int(prefix_len)
+    Pb = np.broadcast_to(np.asarray(prefix_len, dtype=np.int64), (B,))
 
     cond = conditioning(cfg, W, _f64(slot_times), _f64(delta))
     mod = modulation(cfg, W, cond)
     x = _f64(buffer) @ _f64(W["in_w"]) + _f64(W["in_b"])         # residual stream [B, H, D]
     zn = rmsnorm(_f64(fop))                                        # [B, F, D]
 
-    nk = P + F + H
-    valid = np.ones((H, nk), dtype=bool)
-    if mask == "slot_isolated":
-        valid[:, P + F:] = np.eye(H, dtype=bool)
-    elif mask != "full":
+    if mask not in ("full", "slot_isolated"):
         raise ValueError(mask)
+
+    def valid_of(P):   # [H, P + F + H]: which keys each slot sees
+        valid = np.ones((H, P + F + H), dtype=bool)
+        if mask == "slot_isolated":
+            valid[:, P + F:] = np.eye(H, dtype=bool)
+        return valid
 
     for l in range(L):
         wqkv = _f64(W["w_qkv"][l])
@@ -186,6 +190,8 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
         vf = kvf[..., Hkv * hd:].reshape(B, F, Hkv, hd)
         o = np.empty((B, H, Hq, hd))
         for b in range(B):
+            P = int(Pb[b])
+            valid = valid_of(P)
             for g in range(Hkv):
                 keys = np.concatenate([_f64(ctx_k[l, b, g, :P]), kf[b, :, g], ka[b, :, g]])
                 vals = np.concatenate([_f64(ctx_v[l, b, g, :P]), vf[b, :, g], va[b, :, g]])

@@ -192,6 +192,22 @@ def test_batch_independence():
         np.testing.assert_allclose(full[b], one[0], rtol=1e-12, atol=1e-14)
 
 
+def test_per_robot_prefix_lengths_are_independent_robots():
+    # robots whose contexts arrived at different times attend to prefixes of
+    # their own lengths (Sec. 3.2); each robot must equal a one-robot call with
+    # its own length (fails if one robot's length is applied to all, or if a
+    # robot's keys beyond its length leak in)
+    cfg = TINY.replace(batch=3)
+    W, buf, t, k, v, P, z, d, _ = _inputs(cfg)
+    lens = np.array([P, 3, 1])
+    full = expert.expert_velocity(cfg, W, buf, t, k, v, lens, z, d)
+    for b in range(3):
+        one = expert.expert_velocity(cfg.replace(batch=1), W, buf[b:b + 1], t, k[:, b:b + 1], v[:, b:b + 1],
+                                     int(lens[b]), z[b:b + 1], d[b:b + 1])
+        np.testing.assert_allclose(full[b], one[0], rtol=1e-12, atol=1e-14)
+    assert np.abs(full[1] - expert.expert_velocity(cfg, W, buf, t, k, v, P, z, d)[1]).max() > 1e-6
+
+
 def test_slot_permutation_equivariance():
     # full mask, no positional encoding: slots are told apart only by their times
     cfg = TINY
