@@ -147,8 +147,27 @@ ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* bu
  * its stream wait for the copy and then switches to the new context.  The
  * caller may reuse k / v once the side stream has passed this call.
  * 1 <= prefix_len <= max_prefix, else RAVEL_ESHAPE.  A second call before a
- * step has consumed the first returns RAVEL_EBUSY. */
+ * step has consumed the first returns RAVEL_EBUSY.  Every robot has its own
+ * half of the double buffer: this call is ravel_set_context_robots for all
+ * robots of the batch. */
 ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int prefix_len, void* side_stream);
+
+/* Install new VLM contexts for some robots only (Sec. 3.2: each robot's
+ * context is refreshed whenever its own VLM pass completes, so robots run
+ * with contexts of different ages and lengths):
+ *   robots  host int [n], distinct robot indices < B
+ *   k, v    device arrays [L, n, Hkv, prefix_len, hd] of the handle's dtype,
+ *           entry i for robot robots[i]
+ * Each listed robot's context goes into its own inactive half on
+ * `side_stream` (after the last enqueued step and any earlier pending copy);
+ * at the next step those robots switch to it with this prefix length while the
+ * others keep theirs.  Robots still without a context make a step return
+ * RAVEL_ENOCONTEXT.  RAVEL_EBUSY if a listed robot's previous context has not
+ * yet been consumed by a step; RAVEL_EINVAL for a repeated or out-of-range
+ * index; RAVEL_ESHAPE for n outside [1, B] or prefix_len outside
+ * [1, max_prefix]. */
+ravel_status ravel_set_context_robots(ravel_t* r, const int* robots, int n, const void* k, const void* v,
+                                      int prefix_len, void* side_stream);
 
 /* One rolling step (Eq. 3 plus release / shift / append) for the current
  * batch, enqueued on `stream` as one CUDA-graph launch:

@@ -68,6 +68,7 @@ def load(path: str | None = None):
         "ravel_destroy": (None, [vp]),
         "ravel_reset": (i, [vp, i, vp, vp, vp]),
         "ravel_set_context": (i, [vp, vp, vp, i, vp]),
+        "ravel_set_context_robots": (i, [vp, vp, i, vp, vp, i, vp]),
         "ravel_roll_step": (i, [vp, vp, vp, vp, vp, vp, vp, vp]),
         "ravel_denoise_chunk": (i, [vp, vp, i, vp, vp, vp, vp]),
         "ravel_roll_step_rel": (i, [vp, vp, vp, vp, vp, vp, vp, vp, vp]),
@@ -165,6 +166,13 @@ def ravel_reset(h, batch: int, seeds, buffer, stream=None):
 def ravel_set_context(h, k, v, prefix_len: int, side_stream=None):
     _check(h, load().ravel_set_context(h, _dptr(k, name="k"), _dptr(v, name="v"), prefix_len,
                                        _stream_ptr(side_stream)), "ravel_set_context")
+
+
+def ravel_set_context_robots(h, robots, k, v, prefix_len: int, side_stream=None):
+    """New contexts for the listed robots only (k, v [L, len(robots), Hkv, prefix_len, hd])."""
+    idx = np.ascontiguousarray(np.asarray(robots, dtype=np.int32))
+    _check(h, load().ravel_set_context_robots(h, idx.ctypes.data, int(idx.size), _dptr(k, name="k"), _dptr(v, name="v"),
+                                              prefix_len, _stream_ptr(side_stream)), "ravel_set_context_robots")
 
 
 def ravel_roll_step(h, buffer, slot_times, obs_tokens, delta, released, velocity=None, stream=None):

@@ -213,8 +213,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   const int qt = blockIdx.x, bg = blockIdx.y, split = blockIdx.z;
   const int b = bg / p.Hkv, g = bg % p.Hkv;
   const int rows_per_robot = p.H + p.F;
-  const int slot = p.ctx_state[0];
-  const int P = p.ctx_state[1];
+  const int slot = p.ctx_state[2 * b];       // this robot's active context
+  const int P = p.ctx_state[2 * b + 1];
   const int C = p.n_pre + p.n_kv;
   const int c0 = (int)((long)split * C / p.splits), c1 = (int)((long)(split + 1) * C / p.splits);
   const uint32_t ncols = (128 + p.hdp <= 256) ? 256u : 512u;
@@ -910,15 +910,16 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   return e;
 }
 
-// Context V [L][B][Hkv][P][hd] -> slot Vt [L][Bmax][Hkv][hd][pst] (keys contiguous).
-__global__ void transpose_ctx_v_kernel(const bf16* __restrict__ src, bf16* __restrict__ dst, int B, int Bmax,
-                                       int Hkv, int P, int hd, int pst) {
+// Context V [L][n][Hkv][P][hd] of the listed robots -> their slots
+// Vt [L][Bmax][Hkv][hd][pst] (keys contiguous).
+__global__ void transpose_ctx_v_kernel(const bf16* __restrict__ src, int src_n, int i0, bf16* __restrict__ dst0,
+                                       bf16* __restrict__ dst1, int Bmax, int Hkv, int P, int hd, int pst, CtxList f) {
   __shared__ bf16 tile[32][33];
-  const int z = blockIdx.z;                 // (l * B + b) * Hkv + g
-  const int g = z % Hkv, lb = z / Hkv;
-  const int bb = lb % B, l = lb / B;
-  const bf16* s = src + (size_t)z * P * hd;
-  bf16* d = dst + ((size_t)(l * Bmax + bb) * Hkv + g) * hd * pst;
+  const int z = blockIdx.z;                 // (l * f.n + i) * Hkv + g
+  const int g = z % Hkv, li = z / Hkv;
+  const int i = li % f.n, l = li / f.n;
+  const bf16* s = src + ((size_t)(l * src_n + i0 + i) * Hkv + g) * P * hd;
+  bf16* d = (f.slot[i] ? dst1 : dst0) + ((size_t)(l * Bmax + f.robot[i]) * Hkv + g) * hd * pst;
   const int p0 = blockIdx.x * 32, d0 = blockIdx.y * 32;
   for (int i = threadIdx.y; i < 32; i += blockDim.y) {
     const int pp = p0 + i, dd = d0 + threadIdx.x;
@@ -931,10 +932,12 @@ __global__ void transpose_ctx_v_kernel(const bf16* __restrict__ src, bf16* __res
   }
 }
 
-cudaError_t launch_transpose_ctx_v(const void* src, void* dst, int L, int B, int Bmax, int Hkv, int P, int hd,
-                                   int pst, cudaStream_t st) {
-  dim3 grid((P + 31) / 32, (hd + 31) / 32, L * B * Hkv), block(32, 8);
-  transpose_ctx_v_kernel<<<grid, block, 0, st>>>((const bf16*)src, (bf16*)dst, B, Bmax, Hkv, P, hd, pst);
+cudaError_t launch_transpose_ctx_v(const void* src, int src_n, int i0, void* dst0, void* dst1, int L, int Bmax,
+                                   int Hkv, int P, int hd, int pst, const CtxList& f, cudaStream_t st) {
+  if (f.n <= 0) return cudaSuccess;
+  dim3 grid((P + 31) / 32, (hd + 31) / 32, L * f.n * Hkv), block(32, 8);
+  transpose_ctx_v_kernel<<<grid, block, 0, st>>>((const bf16*)src, src_n, i0, (bf16*)dst0, (bf16*)dst1, Bmax, Hkv, P,
+                                                 hd, pst, f);
   return cudaGetLastError();
 }
 

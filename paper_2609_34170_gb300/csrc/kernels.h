@@ -180,9 +180,12 @@ struct AttnTcArgs {
 cudaError_t init_attention_tc();
 bool attention_tc_supported(int hd, int G);
 cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st);
-// bf16 context V [L][B][Hkv][P][hd] -> slot layout Vt [L][Bmax][Hkv][hd][pst]
-cudaError_t launch_transpose_ctx_v(const void* src, void* dst, int L, int B, int Bmax, int Hkv, int P, int hd,
-                                   int pst, cudaStream_t st);
+// bf16 context V [L][src_n][Hkv][P][hd] (list entry i at source position
+// i0 + i) -> the listed robots' slots Vt_{f.slot[i]} [L][Bmax][Hkv][hd][pst]
+// (keys contiguous)
+struct CtxList;
+cudaError_t launch_transpose_ctx_v(const void* src, int src_n, int i0, void* dst0, void* dst1, int L, int Bmax,
+                                   int Hkv, int P, int hd, int pst, const CtxList& f, cudaStream_t st);
 
 // ---- gated cross-attention of a FOP adapter ------------------------------------------
 // out[b*H + j][h*hd + c] = tanh(gate[0]) * sum_f softmax_f(q . k_f / sqrt(hd)) v_f[c] over the
@@ -235,7 +238,20 @@ cudaError_t launch_reset(float* buffer, const uint64_t* seeds, uint64_t* counter
 // Busy-wait on the device for `ns` nanoseconds (globaltimer), then return.
 cudaError_t launch_delay(unsigned long long ns, cudaStream_t st);
 
-// ctx_state = {slot, prefix_len}
-cudaError_t launch_flip(int* ctx_state, int slot, int prefix_len, cudaStream_t st);
+// Per-robot context updates: robot[i] switches to slot[i] with prefix length
+// len[i] (flip), or receives its new context rows in slot[i] (scatter).
+constexpr int kCtxListMax = 256;
+struct CtxList {
+  int n;
+  int robot[kCtxListMax];
+  int slot[kCtxListMax];
+  int len[kCtxListMax];
+};
+// ctx_state [Bmax][2] = {slot, prefix length} per robot
+cudaError_t launch_flip(int* ctx_state, const CtxList& f, cudaStream_t st);
+// src [L][src_n][Hkv][P] rows of row_bytes, list entry i at source position
+// i0 + i -> dst_{f.slot[i]} [L][Bmax][Hkv][Pmax] rows of robot f.robot[i]
+cudaError_t launch_ctx_scatter(const void* src, int src_n, int i0, void* dst0, void* dst1, int L, int Bmax, int Hkv,
+                               int P, int Pmax, size_t row_bytes, const CtxList& f, cudaStream_t st);
 
 }  // namespace ravel

@@ -634,8 +634,8 @@ __global__ void __launch_bounds__(ATT_THREADS) attention_simt_kernel(AttnArgs a)
   const int G = a.Hq / a.Hkv;
   const int nrows = a.H * G;
   const int r0 = blockIdx.y * ATT_QT;
-  const int slot = a.ctx_state[0];
-  const int P = a.ctx_state[1];
+  const int slot = a.ctx_state[2 * b];       // this robot's active context
+  const int P = a.ctx_state[2 * b + 1];
   if (P < 0 || P > a.Pmax) {
     if (threadIdx.x == 0) raise_error(a.err, ERR_PREFIX_LEN);
     return;
@@ -1089,13 +1089,43 @@ cudaError_t launch_delay(unsigned long long ns, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-__global__ void flip_kernel(int* s, int slot, int len) {
-  s[0] = slot;
-  s[1] = len;
+__global__ void flip_kernel(int* s, CtxList f) {
+  for (int i = threadIdx.x; i < f.n; i += blockDim.x) {
+    s[2 * f.robot[i]] = f.slot[i];
+    s[2 * f.robot[i] + 1] = f.len[i];
+  }
 }
 
-cudaError_t launch_flip(int* ctx_state, int slot, int prefix_len, cudaStream_t st) {
-  flip_kernel<<<1, 1, 0, st>>>(ctx_state, slot, prefix_len);
+cudaError_t launch_flip(int* ctx_state, const CtxList& f, cudaStream_t st) {
+  if (f.n <= 0) return cudaSuccess;
+  flip_kernel<<<1, 128, 0, st>>>(ctx_state, f);
+  return cudaGetLastError();
+}
+
+// Context rows of the listed robots into their slots: source [L][src_n][Hkv]
+// [P][row] with the list's robots at positions i0 .. i0 + f.n - 1 of each
+// layer, destination [slot][L][Bmax][Hkv][Pmax][row] (16-byte words).
+__global__ void ctx_scatter_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst0, uint4* __restrict__ dst1,
+                                   int src_n, int i0, int Bmax, int Hkv, int P, int Pmax, int row_words, CtxList f) {
+  const int z = blockIdx.y;                  // (l * f.n + i) * Hkv + g
+  const int g = z % Hkv, li = z / Hkv;
+  const int i = li % f.n, l = li / f.n;
+  const size_t words = (size_t)P * row_words;
+  const uint4* s = src + ((size_t)(l * src_n + i0 + i) * Hkv + g) * words;
+  uint4* d = (f.slot[i] ? dst1 : dst0) + (((size_t)l * Bmax + f.robot[i]) * Hkv + g) * (size_t)Pmax * row_words;
+  for (size_t w = (size_t)blockIdx.x * blockDim.x + threadIdx.x; w < words; w += (size_t)gridDim.x * blockDim.x)
+    d[w] = s[w];
+}
+
+cudaError_t launch_ctx_scatter(const void* src, int src_n, int i0, void* dst0, void* dst1, int L, int Bmax, int Hkv,
+                               int P, int Pmax, size_t row_bytes, const CtxList& f, cudaStream_t st) {
+  if (f.n <= 0 || P <= 0) return cudaSuccess;
+  if (row_bytes % 16 || ((uintptr_t)src | (uintptr_t)dst0 | (uintptr_t)dst1) % 16) return cudaErrorMisalignedAddress;
+  const int row_words = (int)(row_bytes / 16);
+  const size_t words = (size_t)P * row_words;
+  dim3 grid((unsigned)std::min<size_t>((words + 255) / 256, 64), (unsigned)(L * f.n * Hkv));
+  ctx_scatter_kernel<<<grid, 256, 0, st>>>((const uint4*)src, (uint4*)dst0, (uint4*)dst1, src_n, i0, Bmax, Hkv, P,
+                                           Pmax, row_words, f);
   return cudaGetLastError();
 }
 

@@ -27,11 +27,14 @@ const char* const kStatusText[] = {
 struct ravel_ctx {
   StepPlan plan;               // sizes, device buffers, weights (step.h)
   int device = 0;
-  // context double buffer
-  int active_host = 0;         // slot the device will use after pending flips
-  bool have_ctx = false;
-  bool swap_pending = false;
-  int pending_slot = 0, pending_len = 0;
+  // context double buffer, per robot
+  std::vector<int> ctx_active;    // [B] slot the device will use after pending flips
+  std::vector<int> ctx_len;       // [B] its prefix length
+  std::vector<char> ctx_have;     // [B] the robot has a context
+  std::vector<int> ctx_pend;      // [B] pending slot (-1: none)
+  std::vector<int> ctx_pend_len;  // [B]
+  bool have_ctx = false;          // every robot of the batch has a context
+  bool swap_pending = false;      // some robot has a pending swap
   bool any_step = false;
   cudaEvent_t ev_step_done = nullptr, ev_ctx_ready = nullptr;
   // rollout state
@@ -161,51 +164,91 @@ ravel_status ravel_reset(ravel_t* r, int batch, const uint64_t* seeds, float* bu
     // contexts are laid out per robot: a new batch needs a new context
     r->have_ctx = false;
     r->swap_pending = false;
+    r->ctx_active.assign(batch, 0);
+    r->ctx_len.assign(batch, 0);
+    r->ctx_have.assign(batch, 0);
+    r->ctx_pend.assign(batch, -1);
+    r->ctx_pend_len.assign(batch, 0);
   }
   r->batch = batch;
   return RAVEL_OK;
 }
 
-ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int prefix_len, void* side_stream) {
-  if (!r || !k || !v) return fail(r, RAVEL_EINVAL, "set_context: null argument");
-  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, "set_context: call ravel_reset first");
+// Copies robots[0..n) 's new contexts (K, V [L][n][Hkv][prefix_len][hd]) into
+// each robot's inactive slot on the side stream and marks their swaps pending.
+static ravel_status set_context_impl(ravel_t* r, const int* robots, int n, const void* k, const void* v,
+                                     int prefix_len, void* side_stream, const char* what) {
+  const std::string w(what);
+  if (!r || !k || !v || (n > 0 && !robots)) return fail(r, RAVEL_EINVAL, w + ": null argument");
+  if (r->batch == 0) return fail(r, RAVEL_ENOTREADY, w + ": call ravel_reset first");
+  if (n < 1 || n > r->batch) return fail(r, RAVEL_ESHAPE, w + ": robot count outside [1, batch]");
   if (prefix_len < 1 || prefix_len > r->plan.cfg.max_prefix)
-    return fail(r, RAVEL_ESHAPE, "set_context: prefix_len outside [1, max_prefix]");
-  if (r->swap_pending) return fail(r, RAVEL_EBUSY, "set_context: previous context not yet consumed by a step");
+    return fail(r, RAVEL_ESHAPE, w + ": prefix_len outside [1, max_prefix]");
+  std::vector<char> seen(r->batch, 0);
+  for (int i = 0; i < n; ++i) {
+    if (robots[i] < 0 || robots[i] >= r->batch || seen[robots[i]])
+      return fail(r, RAVEL_EINVAL, w + ": robot index out of range or repeated");
+    seen[robots[i]] = 1;
+  }
+  for (int i = 0; i < n; ++i)
+    if (r->ctx_pend[robots[i]] >= 0)
+      return fail(r, RAVEL_EBUSY, w + ": previous context of a robot not yet consumed by a step");
   RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
   cudaStream_t side = (cudaStream_t)side_stream;
-  const int target = r->have_ctx ? 1 - r->active_host : 0;
-  // the inactive slot was last read by steps already enqueued: wait for them
-  if (r->any_step) RV_CUDA(r, cudaStreamWaitEvent(side, r->ev_step_done, 0), "set_context: wait");
+  // the inactive slots were last read by steps already enqueued, and an
+  // earlier pending copy (maybe on another stream) must finish first: the
+  // step waits for the last copy's event only
+  if (r->any_step) RV_CUDA(r, cudaStreamWaitEvent(side, r->ev_step_done, 0), (w + ": wait").c_str());
+  if (r->swap_pending) RV_CUDA(r, cudaStreamWaitEvent(side, r->ev_ctx_ready, 0), (w + ": order").c_str());
   const StepPlan& p = r->plan;
   const ravel_config& c = p.cfg;
   const size_t es = p.esize;
-  const size_t row = (size_t)prefix_len * c.head_dim * es;        // one (l, b, g) block of the source
-  const size_t dpitch = (size_t)c.max_prefix * c.head_dim * es;  // the same block in the slot
-  const size_t per_layer_src = (size_t)r->batch * c.n_kv_heads;
-  if (p.use_tc_attn) {
-    // the tensor-core attention reads V transposed (keys contiguous)
-    RV_CUDA(r, launch_transpose_ctx_v(v, p.ctx_v[target], c.layers, r->batch, c.max_batch, c.n_kv_heads, prefix_len,
-                                      c.head_dim, p.pst, side),
-            "set_context: transpose V");
-  }
-  for (int which = 0; which < (p.use_tc_attn ? 1 : 2); ++which) {
-    const char* src = (const char*)(which ? v : k);
-    char* dst = (char*)(which ? p.ctx_v[target] : p.ctx_k[target]);
-    for (int l = 0; l < c.layers; ++l) {
-      RV_CUDA(r,
-              cudaMemcpy2DAsync(dst + (size_t)l * c.max_batch * c.n_kv_heads * dpitch, dpitch,
-                                src + (size_t)l * per_layer_src * row, row, row, per_layer_src,
-                                cudaMemcpyDeviceToDevice, side),
-              "set_context: copy");
+  for (int i0 = 0; i0 < n; i0 += kCtxListMax) {
+    CtxList f{};
+    f.n = std::min(kCtxListMax, n - i0);
+    for (int i = 0; i < f.n; ++i) {
+      const int b = robots[i0 + i];
+      f.robot[i] = b;
+      f.slot[i] = r->ctx_have[b] ? 1 - r->ctx_active[b] : 0;
+      f.len[i] = prefix_len;
+    }
+    RV_CUDA(r, launch_ctx_scatter(k, n, i0, p.ctx_k[0], p.ctx_k[1], c.layers, c.max_batch, c.n_kv_heads, prefix_len,
+                                  c.max_prefix, (size_t)c.head_dim * es, f, side),
+            (w + ": copy K").c_str());
+    if (p.use_tc_attn) {
+      // the tensor-core attention reads V transposed (keys contiguous)
+      RV_CUDA(r, launch_transpose_ctx_v(v, n, i0, p.ctx_v[0], p.ctx_v[1], c.layers, c.max_batch, c.n_kv_heads,
+                                        prefix_len, c.head_dim, p.pst, f, side),
+              (w + ": transpose V").c_str());
+    } else {
+      RV_CUDA(r, launch_ctx_scatter(v, n, i0, p.ctx_v[0], p.ctx_v[1], c.layers, c.max_batch, c.n_kv_heads, prefix_len,
+                                    c.max_prefix, (size_t)c.head_dim * es, f, side),
+              (w + ": copy V").c_str());
+    }
+    for (int i = 0; i < f.n; ++i) {
+      r->ctx_pend[f.robot[i]] = f.slot[i];
+      r->ctx_pend_len[f.robot[i]] = prefix_len;
+      r->ctx_have[f.robot[i]] = 1;
     }
   }
-  RV_CUDA(r, cudaEventRecord(r->ev_ctx_ready, side), "set_context: record");
+  RV_CUDA(r, cudaEventRecord(r->ev_ctx_ready, side), (w + ": record").c_str());
   r->swap_pending = true;
-  r->pending_slot = target;
-  r->pending_len = prefix_len;
-  r->have_ctx = true;
+  bool all = true;
+  for (int b = 0; b < r->batch; ++b) all = all && r->ctx_have[b];
+  r->have_ctx = all;
   return RAVEL_OK;
+}
+
+ravel_status ravel_set_context(ravel_t* r, const void* k, const void* v, int prefix_len, void* side_stream) {
+  if (!r) return RAVEL_EINVAL;
+  std::vector<int> all(r->batch);
+  for (int b = 0; b < r->batch; ++b) all[b] = b;
+  return set_context_impl(r, all.data(), r->batch, k, v, prefix_len, side_stream, "set_context");
+}
+
+ravel_status ravel_set_context_robots(ravel_t* r, const int* robots, int n, const void* k, const void* v,
+                                      int prefix_len, void* side_stream) {
+  return set_context_impl(r, robots, n, k, v, prefix_len, side_stream, "set_context_robots");
 }
 
 static ravel_status check_device_errors(ravel_t* r) {
@@ -226,8 +269,22 @@ static ravel_status check_device_errors(ravel_t* r) {
 static ravel_status apply_pending_swap(ravel_t* r, cudaStream_t st) {
   if (!r->swap_pending) return RAVEL_OK;
   RV_CUDA(r, cudaStreamWaitEvent(st, r->ev_ctx_ready, 0), "wait for context");
-  RV_CUDA(r, launch_flip(r->plan.ctx_state, r->pending_slot, r->pending_len, st), "context flip");
-  r->active_host = r->pending_slot;
+  CtxList f{};
+  for (int b = 0; b < r->batch; ++b) {
+    if (r->ctx_pend[b] < 0) continue;
+    f.robot[f.n] = b;
+    f.slot[f.n] = r->ctx_pend[b];
+    f.len[f.n] = r->ctx_pend_len[b];
+    ++f.n;
+    r->ctx_active[b] = r->ctx_pend[b];
+    r->ctx_len[b] = r->ctx_pend_len[b];
+    r->ctx_pend[b] = -1;
+    if (f.n == kCtxListMax) {
+      RV_CUDA(r, launch_flip(r->plan.ctx_state, f, st), "context flip");
+      f.n = 0;
+    }
+  }
+  RV_CUDA(r, launch_flip(r->plan.ctx_state, f, st), "context flip");
   r->swap_pending = false;
   return RAVEL_OK;
 }
@@ -385,9 +442,13 @@ ravel_status ravel_debug_inject(ravel_t* r, int fault, int count, void* stream) 
   if (!r) return RAVEL_EINVAL;
   if (!r->have_ctx) return fail(r, RAVEL_ENOCONTEXT, "debug_inject: no context set");
   RV_CUDA(r, cudaSetDevice(r->device), "cudaSetDevice");
-  // the device state {active slot, prefix length}: a length past max_prefix
-  RV_CUDA(r, launch_flip(r->plan.ctx_state, r->active_host, r->plan.cfg.max_prefix + 1000, (cudaStream_t)stream),
-          "debug_inject: state write");
+  // robot 0's device state {active slot, prefix length}: a length past max_prefix
+  CtxList f{};
+  f.n = 1;
+  f.robot[0] = 0;
+  f.slot[0] = r->ctx_active[0];
+  f.len[0] = r->plan.cfg.max_prefix + 1000;
+  RV_CUDA(r, launch_flip(r->plan.ctx_state, f, (cudaStream_t)stream), "debug_inject: state write");
   return RAVEL_OK;
 }
 

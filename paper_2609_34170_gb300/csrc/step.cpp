@@ -125,7 +125,7 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
     AL(p->ctx_k[s], ctx_bytes);
     AL(p->ctx_v[s], ctx_bytes);
   }
-  AL(p->ctx_state, 2 * sizeof(int));
+  AL(p->ctx_state, (size_t)Bm * 2 * sizeof(int));   // per robot {active slot, prefix length}
   const size_t rows_c = (size_t)H + Bm, rows_a = (size_t)Bm * H, rows_y = (size_t)Bm * (H + F);
   AL(p->E, rows_c * D * es); AL(p->H1, rows_c * D * es); AL(p->HC, rows_c * D * es);
   AL(p->omega, (size_t)(D / 2) * sizeof(double));

@@ -49,6 +49,12 @@ class RollingSession:
         self._ctx = (k, v)   # keep alive until the side-stream copy has run
         B.ravel_set_context(self.handle, k, v, int(prefix_len or k.shape[3]), side_stream)
 
+    def set_context_robots(self, robots, k, v, prefix_len: int | None = None, side_stream=None):
+        """New contexts for the listed robots only: k, v [L, len(robots), Hkv, P, hd]."""
+        k, v = self.to_dev(k), self.to_dev(v)
+        self._ctx_robots = (k, v)   # keep alive until the side-stream copy has run
+        B.ravel_set_context_robots(self.handle, robots, k, v, int(prefix_len or k.shape[3]), side_stream)
+
     def step(self, slot_times, obs, delta, want_velocity: bool = False, stream=None, state=None):
         """One rolling step; with `state` ([B, A]) the buffer holds absolute
         targets and the expert works relative to that state (see
