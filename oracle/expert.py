@@ -44,14 +44,21 @@ def _f64(a):
 
 
 def sinusoidal(x, width: int) -> np.ndarray:
-    """Sinusoidal embedding [N, width] of scalars x [N]: first half sin(x w_i),
-    second half cos(x w_i), w_i = 2 pi / p_i, periods p_i geometric from 4e-3
-    (i = 0) to 4.0 (i = width/2 - 1)."""
+    """Sinusoidal embedding [..., width] of scalars x [...]: first half
+    sin(x w_i), second half cos(x w_i), w_i = 2 pi / p_i, periods p_i
+    geometric from 4e-3 (i = 0) to 4.0 (i = width/2 - 1)."""
     half = width // 2
     i = np.arange(half, dtype=np.float64)
     period = 4e-3 * (4.0 / 4e-3) ** (i / (half - 1))
-    ang = _f64(x)[:, None] * (2.0 * np.pi / period)[None, :]
-    return np.concatenate([np.sin(ang), np.cos(ang)], axis=1)
+    ang = _f64(x)[..., None] * (2.0 * np.pi / period)
+    return np.concatenate([np.sin(ang), np.cos(ang)], axis=-1)
+
+
+def per_slot(slot_times):
+    """Slot times [H] (shared by every robot) or [B, H] (one schedule per
+    robot) as a [1 or B, H, 1] array for per-slot arithmetic."""
+    t = _f64(slot_times)
+    return t[None, :, None] if t.ndim == 1 else t[:, :, None]
 
 
 def silu(x):
@@ -81,11 +88,12 @@ def mlp2(e, w1, b1, w2, b2):
 def conditioning(cfg, W, slot_times, delta):
     """cond[b, j] = MLP_t(emb(t_j)) + MLP_d(emb(delta_b))  (App. A.1: the offset
     MLP's embedding is added to the flow-timestep embedding; every slot keeps
-    its own t_j and all slots share delta_b).  Returns [B, H, D]."""
+    its own t_j and all slots share delta_b).  slot_times [H], or [B, H] when
+    every robot runs its own schedule (t_bj).  Returns [B, H, D]."""
     D = cfg.width
-    ht = mlp2(sinusoidal(slot_times, D), W["t_w1"], W["t_b1"], W["t_w2"], W["t_b2"])   # [H, D]
+    ht = mlp2(sinusoidal(slot_times, D), W["t_w1"], W["t_b1"], W["t_w2"], W["t_b2"])   # [H, D] or [B, H, D]
     hd = mlp2(sinusoidal(delta, D), W["d_w1"], W["d_b1"], W["d_w2"], W["d_b2"])        # [B, D]
-    return hd[:, None, :] + ht[None, :, :]
+    return hd[:, None, :] + (ht[None, :, :] if ht.ndim == 2 else ht)
 
 
 def modulation(cfg, W, cond):
@@ -149,7 +157,7 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
                     mask: str = "full", trace: dict | None = None):
     """v_theta(A, t, c, delta) for B robots: [B, H, A] float64 (Eq. 3's velocity).
 
-    buffer [B, H, A]; slot_times [H]; ctx_k / ctx_v [L, B, Hkv, >=prefix_len, hd];
+    buffer [B, H, A]; slot_times [H] or [B, H]; ctx_k / ctx_v [L, B, Hkv, >=prefix_len, hd];
     fop [B, F, D]; delta [B].  prefix_len: one valid prefix length for every
     robot, or one per robot ([B]: robots whose contexts arrived at different
     times, Sec. 3.2).  ``trace`` (optional dict) receives intermediates.
@@ -215,9 +223,10 @@ def expert_velocity(cfg, W, buffer, slot_times, ctx_k, ctx_v, prefix_len, fop, d
 
 
 def slot_dt(slot_times):
-    """dt_j = t_j - t_{j-1} with t_{-1} = 0 (Eq. 3's Delta tau per slot)."""
+    """dt_j = t_j - t_{j-1} with t_{-1} = 0 (Eq. 3's Delta tau per slot), per
+    robot for [B, H] slot times."""
     t = _f64(slot_times)
-    return np.diff(np.concatenate([[0.0], t]))
+    return np.diff(t, axis=-1, prepend=0.0)
 
 
 def euler_roll(buffer, velocity, slot_times, seeds, counters):
@@ -228,7 +237,7 @@ def euler_roll(buffer, velocity, slot_times, seeds, counters):
     of index n_b (the robot's counter), which then advances by one.
     Returns (released [B, A], new buffer [B, H, A], new counters [B]).
     """
-    a = _f64(buffer) + slot_dt(slot_times)[None, :, None] * _f64(velocity)
+    a = _f64(buffer) + per_slot(slot_dt(slot_times)) * _f64(velocity)
     released = a[:, 0].copy()
     B, H, A = a.shape
     counters = np.asarray(counters, dtype=np.uint64)
@@ -245,13 +254,13 @@ def to_relative(buffer, slot_times, state, rel_mask):
     noise stays in model coordinates).  A slot at flow time t holds
     a = t eps + (1 - t) a_hat, so expressing a_hat relative to the state s
     moves it by -(1 - t) s on the relative dimensions (rel_mask = 1)."""
-    shift = (1.0 - _f64(slot_times))[None, :, None] * (_f64(rel_mask)[None, None, :] * _f64(state)[:, None, :])
+    shift = (1.0 - per_slot(slot_times)) * (_f64(rel_mask)[None, None, :] * _f64(state)[:, None, :])
     return _f64(buffer) - shift
 
 
 def to_absolute(buffer_rel, slot_times, state, rel_mask):
     """The inverse of to_relative at the given flow times."""
-    shift = (1.0 - _f64(slot_times))[None, :, None] * (_f64(rel_mask)[None, None, :] * _f64(state)[:, None, :])
+    shift = (1.0 - per_slot(slot_times)) * (_f64(rel_mask)[None, None, :] * _f64(state)[:, None, :])
     return _f64(buffer_rel) + shift
 
 
@@ -280,8 +289,8 @@ def roll_relative(rel, velocity, slot_times, seeds, counters, state, rel_mask):
     its new time (slot j moves from t_j to t_{j-1}, t_{-1} = 0), then the
     release / shift / append.  Returns (released, new buffer, new counters)."""
     t = _f64(slot_times)
-    t_new = np.concatenate([[0.0], t[:-1]])
-    a_rel = _f64(rel) + slot_dt(slot_times)[None, :, None] * _f64(velocity)
+    t_new = np.concatenate([np.zeros(t.shape[:-1] + (1,)), t[..., :-1]], axis=-1)
+    a_rel = _f64(rel) + per_slot(slot_dt(slot_times)) * _f64(velocity)
     a = to_absolute(a_rel, t_new, state, rel_mask)
     B, H, A = a.shape
     released = a[:, 0].copy()

@@ -163,6 +163,56 @@ def test_ideal_single_target_field_releases_targets_in_order():
     np.testing.assert_allclose(rel, targets[:steps], rtol=0, atol=1e-12)
 
 
+def test_ideal_field_with_a_schedule_per_robot():
+    # robots running their own slot-time schedules ([B, H] slot times): the
+    # single-target field is still integrated exactly, so each robot releases
+    # its targets in order (fails if a robot's dt comes from another robot's
+    # schedule, or if dt is taken along the robot axis)
+    cfg = TINY.replace(batch=2, slots=6, action_dim=4)
+    H = cfg.slots
+    t = np.stack([synth.staggered_times(H), ((np.arange(H) + 1) / H) ** 2]).astype(np.float32).astype(np.float64)
+    steps = 3 * H
+    targets = np.random.default_rng(19).standard_normal((steps + H, 2, 4))
+    seeds = synth.robot_seeds(23, 2)
+
+    def field(s, buf):
+        tgt = np.stack([targets[s + j] for j in range(H)], axis=1)
+        return (tgt - buf) / t[:, :, None]
+
+    rel = _rollout(cfg, steps, t.astype(np.float32), field, seeds)
+    np.testing.assert_allclose(rel, targets[:steps], rtol=0, atol=1e-12)
+
+
+def test_per_robot_slot_times_are_independent_robots():
+    # a step with one schedule per robot equals one-robot steps with each
+    # robot's own schedule; with equal rows it equals the shared-times step
+    cfg = TINY.replace(batch=3)
+    W, buf, t, k, v, P, z, d, cnt = _inputs(cfg)
+    H = cfg.slots
+    tb = np.stack([t, ((np.arange(H) + 1) / H) ** 2, np.sqrt((np.arange(H) + 1) / H)]).astype(np.float32)
+    seeds = synth.robot_seeds(7, 3)
+    full = expert.roll_step(cfg, W, buf, tb, k, v, P, z, d, seeds, cnt)
+    for b in range(3):
+        one = expert.roll_step(cfg.replace(batch=1), W, buf[b:b + 1], tb[b], k[:, b:b + 1], v[:, b:b + 1], P,
+                               z[b:b + 1], d[b:b + 1], seeds[b:b + 1], cnt[b:b + 1])
+        for x, y in zip(full, one):
+            np.testing.assert_allclose(np.asarray(x)[b], np.asarray(y)[0], rtol=1e-12, atol=1e-13)
+    same = expert.roll_step(cfg, W, buf, np.stack([t] * 3), k, v, P, z, d, seeds, cnt)
+    shared = expert.roll_step(cfg, W, buf, t, k, v, P, z, d, seeds, cnt)
+    for x, y in zip(same, shared):
+        np.testing.assert_allclose(np.asarray(x), np.asarray(y), rtol=1e-13, atol=1e-14)
+    # relative coordinates follow each robot's own schedule too
+    state = np.random.default_rng(4).standard_normal((3, cfg.action_dim))
+    mask = np.array([1.0, 0.0, 1.0][:cfg.action_dim] + [1.0] * max(0, cfg.action_dim - 3))
+    full = expert.roll_step(cfg, W, buf, tb, k, v, P, z, d, seeds, cnt, state=state, rel_mask=mask)
+    for b in range(3):
+        one = expert.roll_step(cfg.replace(batch=1), W, buf[b:b + 1], tb[b], k[:, b:b + 1], v[:, b:b + 1], P,
+                               z[b:b + 1], d[b:b + 1], seeds[b:b + 1], cnt[b:b + 1], state=state[b:b + 1],
+                               rel_mask=mask)
+        for x, y in zip(full, one):
+            np.testing.assert_allclose(np.asarray(x)[b], np.asarray(y)[0], rtol=1e-12, atol=1e-13)
+
+
 def test_reset_and_append_bookkeeping():
     cfg = TINY.replace(batch=3, slots=4, action_dim=6)
     seeds = synth.robot_seeds(1 << 40, 3)
