@@ -84,6 +84,12 @@ typedef struct {
                        layer's self-attention block:
                        x += tanh(a_gate) MHA(q = RMSNorm(x)(1 + a_gamma) a_wq,
                        [k | v] = RMSNorm(z)(1 + a_zgamma) a_wkv) a_wo */
+  int per_robot_times; /* 0: one slot-time schedule [H] shared by every robot;
+                       1: every robot runs its own schedule, slot_times
+                       [B, H] (the conditioning, the Euler step and the
+                       relative shift use robot b's t_bj; the modulation is
+                       then computed for B*H time rows every step, with no
+                       conditioning cache) */
 } ravel_config;
 
 /*
@@ -173,7 +179,8 @@ ravel_status ravel_set_context_robots(ravel_t* r, const int* robots, int n, cons
  * batch, enqueued on `stream` as one CUDA-graph launch:
  *   buffer      device float32 [B, H, A], read and updated in place
  *   slot_times  device float32 [H], increasing, slot_times[H-1] = 1 for the
- *               paper's schedule
+ *               paper's schedule; [B, H] (one schedule per robot) for a
+ *               handle created with per_robot_times
  *   obs_tokens  device [B, F, D] FOP tokens of the handle's dtype (NULL iff F = 0)
  *   delta       device float32 [B], context age p/K (+ bias) per robot
  *   released    device float32 [B, A], written: the action released by each robot

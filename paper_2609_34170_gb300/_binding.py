@@ -24,7 +24,7 @@ STATUS = ["RAVEL_OK", "RAVEL_EINVAL", "RAVEL_ESHAPE", "RAVEL_ENOMEM", "RAVEL_ECU
 class RavelConfig(C.Structure):
     _fields_ = [(n, C.c_int) for n in (
         "layers", "width", "n_q_heads", "n_kv_heads", "head_dim", "mlp_dim", "slots", "action_dim",
-        "max_prefix", "fop_tokens", "max_batch", "dtype", "mask_mode", "fop_adapter_every")]
+        "max_prefix", "fop_tokens", "max_batch", "dtype", "mask_mode", "fop_adapter_every", "per_robot_times")]
 
 
 WEIGHT_FIELDS = ("t_w1", "t_b1", "t_w2", "t_b2", "d_w1", "d_b1", "d_w2", "d_b2", "mod_w", "mod_b",
@@ -124,7 +124,7 @@ def ravel_create(cfg, weights: dict, device: int = 0, max_batch: int | None = No
     c = RavelConfig(cfg.layers, cfg.width, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.mlp_dim, cfg.slots,
                     cfg.action_dim, max_prefix or cfg.prefix, cfg.fop_tokens, max_batch or cfg.batch,
                     RAVEL_BF16 if cfg.dtype == "bf16" else RAVEL_FP32, mask_mode,
-                    getattr(cfg, "fop_adapter_every", 0))
+                    getattr(cfg, "fop_adapter_every", 0), getattr(cfg, "per_robot_times", 0))
     on_dev = None
     keep = []
     w = RavelWeights()

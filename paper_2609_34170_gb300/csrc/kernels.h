@@ -73,6 +73,7 @@ struct RowNorm {
   int B, H;
   const void* fop; int F; const float* gamma;
   void* Y; int row_pitch;
+  int t_stride = 0;   // as NormArgs (also the slot times' stride for the relative shift)
 };
 struct GemmArgs {
   const void* A; int lda;       // [M][K] activations of dtype dt
@@ -127,6 +128,7 @@ struct NormArgs {
   const int* drow = nullptr;    // optional: row of modv holding robot b's offset part (default H + b)
   const float* act_gain = nullptr;   // optional [D]: action rows y = x rsqrt(mean(x^2)+eps) (1 + act_gain),
                                      // without modulation (the query rows of a FOP adapter)
+  int t_stride = 0;             // modv time row of slot j of robot b: b * t_stride + j (H: a schedule per robot)
 };
 cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 
@@ -135,7 +137,7 @@ cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st);
 // the expert sees a - (1 - t_j) rel_mask * state_b (the relative ones).
 cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b,
                            float* x, cudaStream_t st, const float* state = nullptr, const float* rel_mask = nullptr,
-                           const float* slot_times = nullptr, int H = 1);
+                           const float* slot_times = nullptr, int H = 1, int t_stride = 0);
 
 // The in-projection (as launch_in_proj) of whole rows with the first layer's
 // adaRMSNorm into rn.Y (action rows and, with rn.fop, FOP rows).
@@ -206,6 +208,7 @@ struct TailArgs {
   int B, H, A;
   const float* state = nullptr;      // optional [B][A]: absolute buffer, relative expert (see launch_in_proj):
   const float* rel_mask = nullptr;   // [A]; a' = a + dt (v + rel_mask * state)
+  int t_stride = 0;                  // slot time of robot b's slot j: slot_times[b * t_stride + j]
 };
 cudaError_t launch_tail(const TailArgs& a, cudaStream_t st);
 
@@ -219,6 +222,7 @@ struct HeadArgs {
   float* v;                                    // [B*H][A] velocity (= a.vel)
   int* cnt;                                    // [B] zero-initialised counters
   int rows_per_cta;
+  int t_stride = 0;                            // as NormArgs
 };
 cudaError_t launch_head_tail(const HeadArgs& h, const TailArgs& a, cudaStream_t st);
 

@@ -379,7 +379,7 @@ __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, i
           if (act) {
             xv[rr][g] = ld4(a.x + (size_t)(b * a.H + jj) * D + c);
             if (modulated) {
-              const float* mt = a.modv + (size_t)jj * a.mod_ld + a.off;
+              const float* mt = a.modv + (size_t)(b * a.t_stride + jj) * a.mod_ld + a.off;
               ts[rr][g] = ld4(mt + c);
               th[rr][g] = ld4(mt + D + c);
             }
@@ -473,7 +473,8 @@ cudaError_t launch_ada_norm(const NormArgs& a, Dtype dt, cudaStream_t st) {
 
 __global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, const float* __restrict__ in_w,
                                const float* __restrict__ in_b, float* __restrict__ x, const float* __restrict__ state,
-                               const float* __restrict__ rel_mask, const float* __restrict__ slot_times, int H) {
+                               const float* __restrict__ rel_mask, const float* __restrict__ slot_times, int H,
+                               int t_stride) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ float arow[];   // the action row of this slot
@@ -482,7 +483,8 @@ __global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, cons
     float a = buf[(size_t)r * A + i];
     if (state) {   // relative coordinates of the expert: a - (1 - t_j) m s_b
       const int b = r / H, j = r % H;
-      a = __fsub_rn(a, __fmul_rn(__fsub_rn(1.f, slot_times[j]), __fmul_rn(rel_mask[i], state[(size_t)b * A + i])));
+      a = __fsub_rn(a, __fmul_rn(__fsub_rn(1.f, slot_times[b * t_stride + j]),
+                                 __fmul_rn(rel_mask[i], state[(size_t)b * A + i])));
     }
     arow[i] = a;
   }
@@ -495,10 +497,11 @@ __global__ void in_proj_kernel(const float* __restrict__ buf, int A, int D, cons
 }
 
 cudaError_t launch_in_proj(const float* buf, int BH, int A, int D, const float* in_w, const float* in_b, float* x,
-                           cudaStream_t st, const float* state, const float* rel_mask, const float* slot_times, int H) {
+                           cudaStream_t st, const float* state, const float* rel_mask, const float* slot_times, int H,
+                           int t_stride) {
   if (BH <= 0) return cudaSuccess;
   return launch_kernel(in_proj_kernel, dim3((D + 255) / 256, BH), dim3(256), A * sizeof(float), st, 1, buf, A, D,
-                       in_w, in_b, x, state, rel_mask, slot_times, H);
+                       in_w, in_b, x, state, rel_mask, slot_times, H, t_stride);
 }
 
 // The in-projection of whole rows with the first layer's adaRMSNorm: one
@@ -524,7 +527,8 @@ __global__ void __launch_bounds__(256) in_proj_norm_kernel(const float* __restri
     for (int i = threadIdx.x; i < A; i += blockDim.x) {
       float a = buf[(size_t)r * A + i];
       if (state)   // relative coordinates of the expert: a - (1 - t_j) m s_b
-        a = __fsub_rn(a, __fmul_rn(__fsub_rn(1.f, slot_times[j]), __fmul_rn(rel_mask[i], state[(size_t)b * A + i])));
+        a = __fsub_rn(a, __fmul_rn(__fsub_rn(1.f, slot_times[b * rn.t_stride + j]),
+                                   __fmul_rn(rel_mask[i], state[(size_t)b * A + i])));
       arow[i] = a;
     }
     __syncthreads();
@@ -541,7 +545,7 @@ __global__ void __launch_bounds__(256) in_proj_norm_kernel(const float* __restri
       }
     }
     const float inv = rsqrtf(block_sum(ss, red) / (float)D + 1e-6f);
-    const float* mt = rn.modv + (size_t)j * rn.mod_ld + rn.off;
+    const float* mt = rn.modv + (size_t)(b * rn.t_stride + j) * rn.mod_ld + rn.off;
     const float* md = rn.modv + (size_t)(rn.drow ? rn.drow[b] : rn.H + b) * rn.mod_ld + rn.off;
     const float* mb = rn.mod_b + rn.off;
     T* Y = (T*)rn.Y + (size_t)(b * rn.row_pitch + j) * D;
@@ -827,8 +831,9 @@ __device__ void tail_robot(const TailArgs& a, int b, float* sa) {
   const float* v = a.vel + (size_t)b * H * A;
   for (int i = threadIdx.x; i < H * A; i += blockDim.x) {
     const int j = i / A;
-    const float t1 = a.slot_times[j];
-    const float t0 = j ? a.slot_times[j - 1] : 0.f;
+    const float* tb = a.slot_times + (size_t)b * a.t_stride;   // robot b's schedule
+    const float t1 = tb[j];
+    const float t0 = j ? tb[j - 1] : 0.f;
     const float dt = __fsub_rn(t1, t0);
     // absolute buffer, relative expert: the slot also moves by dt m s as its
     // flow time drops from t_j to t_{j-1}
@@ -891,7 +896,7 @@ __global__ void __launch_bounds__(256) head_tail_kernel(HeadArgs h, TailArgs a) 
   const float* mb = h.mod_b + h.off;
   for (int j = j0; j < j1; ++j) {
     const float* xr = h.x + (size_t)(b * a.H + j) * D;
-    const float* mt = h.modv + (size_t)j * h.mod_ld + h.off;
+    const float* mt = h.modv + (size_t)(b * h.t_stride + j) * h.mod_ld + h.off;
     // sum of squares of the row (4 features per thread per pass)
     float ss = 0.f;
     for (int f = 4 * threadIdx.x; f < D; f += 4 * blockDim.x) {

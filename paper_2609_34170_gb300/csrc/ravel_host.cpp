@@ -384,7 +384,8 @@ ravel_status ravel_denoise_chunk(ravel_t* r, float* chunk, int n_steps, const vo
     for (int n = 0; n < n_steps && e == cudaSuccess; ++n) {
       const float t_now = (float)(1.0 - (double)n / n_steps);
       const float t_next = n + 1 < n_steps ? (float)(1.0 - (double)(n + 1) / n_steps) : 0.f;
-      e = launch_fill_times(r->plan.dn_times, c.slots, t_now, r->cap_stream);
+      e = launch_fill_times(r->plan.dn_times, c.per_robot_times ? r->batch * c.slots : c.slots, t_now,
+                            r->cap_stream);
       if (e == cudaSuccess) {
         const DenoisePass dn{t_now, t_next};
         int nk = 0;

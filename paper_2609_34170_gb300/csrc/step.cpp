@@ -27,6 +27,7 @@ bool validate_config(const ravel_config& c, std::string* why) {
   if (c.max_prefix < 1 || c.fop_tokens < 0 || c.max_batch < 1) return bad("max_prefix, max_batch >= 1, fop_tokens >= 0");
   if (c.dtype != RAVEL_FP32 && c.dtype != RAVEL_BF16) return bad("dtype must be RAVEL_FP32 or RAVEL_BF16");
   if (c.mask_mode != RAVEL_MASK_FULL && c.mask_mode != RAVEL_MASK_SLOT_ISOLATED) return bad("unknown mask_mode");
+  if (c.per_robot_times != 0 && c.per_robot_times != 1) return bad("per_robot_times must be 0 or 1");
   if (c.fop_adapter_every < 0 || c.fop_adapter_every > c.layers)
     return bad("fop_adapter_every must be 0 or in [1, layers]");
   if (c.fop_adapter_every > 0 && (c.fop_tokens < 1 || c.fop_tokens > 64))
@@ -126,7 +127,10 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
     AL(p->ctx_v[s], ctx_bytes);
   }
   AL(p->ctx_state, (size_t)Bm * 2 * sizeof(int));   // per robot {active slot, prefix length}
-  const size_t rows_c = (size_t)H + Bm, rows_a = (size_t)Bm * H, rows_y = (size_t)Bm * (H + F);
+  // conditioning rows: the time rows (H, or B*H with a schedule per robot),
+  // then the robots' offset rows
+  const size_t rows_t = c.per_robot_times ? (size_t)Bm * H : (size_t)H;
+  const size_t rows_c = rows_t + Bm, rows_a = (size_t)Bm * H, rows_y = (size_t)Bm * (H + F);
   AL(p->E, rows_c * D * es); AL(p->H1, rows_c * D * es); AL(p->HC, rows_c * D * es);
   AL(p->omega, (size_t)(D / 2) * sizeof(double));
   AL(p->modv, (rows_c + kCondCache) * p->mod_dim * 4);
@@ -149,7 +153,7 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   p->tcws.n_counters = 4096;
   AL(p->tcws.ws, p->tcws.ws_bytes);
   AL(p->tcws.counters, p->tcws.n_counters * sizeof(int));
-  AL(p->dn_times, (size_t)H * sizeof(float));
+  AL(p->dn_times, rows_t * sizeof(float));
   AL(p->rel_mask, (size_t)A * sizeof(float));
   p->n_adapters = c.fop_adapter_every > 0 ? L / c.fop_adapter_every : 0;
   const int NA = p->n_adapters, nkv = 2 * c.n_kv_heads * c.head_dim;
@@ -325,33 +329,38 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   // the same every step and the context age takes a handful of values, so
   // the modulation rows usually exist already; the launches below then
   // compute nothing (cond_check sets the skip flag)
-  CondArgs ca{p.cond, p.cond_tkey, p.cond_drow, p.cond_commit, io.slot_times, io.delta, H, B, c.max_batch,
-              p.modv, p.mod_dim, p.cond_cache ? 1 : 0};
+  // time rows of the conditioning: the H slot times, or B*H with a schedule
+  // per robot (norms then read robot b's row b*H + j: t_stride = H)
+  const int Ht = c.per_robot_times ? B * H : H, t_stride = c.per_robot_times ? H : 0;
+  CondArgs ca{p.cond, p.cond_tkey, p.cond_drow, p.cond_commit, io.slot_times, io.delta, Ht, B, c.max_batch,
+              p.modv, p.mod_dim, (p.cond_cache && !c.per_robot_times) ? 1 : 0};
   const int* skip = &p.cond->skip;
   pdl_enabled() = false;
   RUN(KK_COND_CACHE, launch_cond_check(ca, st));
   pdl_enabled() = p.use_pdl && !trace;
-  RUN(KK_EMBED, launch_embed(io.slot_times, H, io.delta, B, D, p.omega, p.E, dt, st, skip));
-  RUN(KK_GEMM_COND, gemm(p.E, D, p.t_w1, H, D, D, EPI_STORE_SILU, p.H1, D, dt, p.t_b1, 0, skip));
-  RUN(KK_GEMM_COND, gemm(rowp(p.E, H, D), D, p.d_w1, B, D, D, EPI_STORE_SILU, (void*)rowp(p.H1, H, D), D, dt, p.d_b1,
+  RUN(KK_EMBED, launch_embed(io.slot_times, Ht, io.delta, B, D, p.omega, p.E, dt, st, skip));
+  RUN(KK_GEMM_COND, gemm(p.E, D, p.t_w1, Ht, D, D, EPI_STORE_SILU, p.H1, D, dt, p.t_b1, 0, skip));
+  RUN(KK_GEMM_COND, gemm(rowp(p.E, Ht, D), D, p.d_w1, B, D, D, EPI_STORE_SILU, (void*)rowp(p.H1, Ht, D), D, dt, p.d_b1,
                          0, skip));
-  RUN(KK_GEMM_COND, gemm(p.H1, D, p.t_w2, H, D, D, EPI_STORE, p.HC, D, dt, p.t_b2, 0, skip));
-  RUN(KK_GEMM_COND, gemm(rowp(p.H1, H, D), D, p.d_w2, B, D, D, EPI_STORE, (void*)rowp(p.HC, H, D), D, dt, p.d_b2, 0,
+  RUN(KK_GEMM_COND, gemm(p.H1, D, p.t_w2, Ht, D, D, EPI_STORE, p.HC, D, dt, p.t_b2, 0, skip));
+  RUN(KK_GEMM_COND, gemm(rowp(p.H1, Ht, D), D, p.d_w2, B, D, D, EPI_STORE, (void*)rowp(p.HC, Ht, D), D, dt, p.d_b2, 0,
                          skip));
-  RUN(KK_GEMM_MOD, gemm(p.HC, D, p.mod_w, H + B, p.mod_dim, D, EPI_STORE, p.modv, p.mod_dim, DT_F32, nullptr, 0, skip));
+  RUN(KK_GEMM_MOD, gemm(p.HC, D, p.mod_w, Ht + B, p.mod_dim, D, EPI_STORE, p.modv, p.mod_dim, DT_F32, nullptr, 0,
+                        skip));
   RUN(KK_COND_CACHE, launch_cond_commit(ca, st));
   // residual stream
   // in-projection; with the fused norms, also the first layer's first norm
   const bool fuse_in = p.fuse_norm && p.dt == DT_BF16 && D <= 4096;
   if (fuse_in) {
     const int FF0 = (io.obs && !(p.n_adapters > 0)) ? F : 0;
-    const RowNorm rn0{p.modv, p.mod_dim, p.mod_b, 0, p.cond_drow, B, H, FF0 ? io.obs : nullptr, F, p.fop_gamma, p.Y,
+    RowNorm rn0{p.modv, p.mod_dim, p.mod_b, 0, p.cond_drow, B, H, FF0 ? io.obs : nullptr, F, p.fop_gamma, p.Y,
                       H + FF0};
+    rn0.t_stride = t_stride;
     RUN(KK_IN_PROJ, launch_in_proj_norm(io.buffer, A, D, p.in_w, p.in_b, p.x, io.state, p.rel_mask, io.slot_times,
                                         rn0, dt, st));
   } else {
     RUN(KK_IN_PROJ, launch_in_proj(io.buffer, B * H, A, D, p.in_w, p.in_b, p.x, st, io.state, p.rel_mask,
-                                   io.slot_times, H));
+                                   io.slot_times, H, t_stride));
   }
   const bool adapters = p.n_adapters > 0 && io.obs;
   const int FF = (io.obs && !adapters) ? F : 0;   // FOP tokens as keys of the self-attention
@@ -360,6 +369,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   for (int l = 0; l < L; ++l) {
     NormArgs n1{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D, FF ? io.obs : nullptr, F,
                 p.fop_gamma + (size_t)l * D, p.Y, RPR, p.cond_drow};
+    n1.t_stride = t_stride;
     if (l > 0 || !fuse_in) RUN(KK_NORM, launch_ada_norm(n1, dt, st));
     const void* wqkv = (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es;
     if (p.use_tc_attn) {
@@ -406,6 +416,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
                            p.x, D, DT_F32, nullptr));
     }
     NormArgs n2{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * l * D + 2 * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
+    n2.t_stride = t_stride;
     RUN(KK_NORM, launch_ada_norm(n2, dt, st));
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
     GemmArgs gu{p.Y, D, wgu, D, BH, 2 * Fm, D, EPI_GEGLU, p.Hm, Fm, dt, nullptr};
@@ -423,13 +434,16 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     // final norm, velocity head and tail in one launch, about eight CTAs per SM
     TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A, io.state,
                 p.rel_mask};
+    ta.t_stride = t_stride;
     const int rpc = std::max(1, (B * H + 8 * p.num_sms - 1) / (8 * p.num_sms));
     HeadArgs hd{p.x, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, p.cond_drow, p.out_w, p.out_b, p.V, p.head_cnt, rpc};
+    hd.t_stride = t_stride;
     RUN(KK_HEAD_TAIL, launch_head_tail(hd, ta, st));
     if (n_kernels) *n_kernels = nk;
     return e;
   }
   NormArgs nf{p.x, B, H, D, p.modv, p.mod_dim, p.mod_b, 4 * L * D, nullptr, 0, nullptr, p.Y, H, p.cond_drow};
+  nf.t_stride = t_stride;
   RUN(KK_NORM, launch_ada_norm(nf, dt, st));
   RUN(KK_GEMM_OUT, gemm(p.Y, D, p.out_w, BH, A, D, EPI_STORE, p.V, A, DT_F32, p.out_b));
   if (dn) {
@@ -437,6 +451,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
   } else {
     TailArgs ta{io.buffer, p.V, io.slot_times, io.released, io.velocity, p.seeds, p.counters, B, H, A, io.state,
                 p.rel_mask};
+    ta.t_stride = t_stride;
     RUN(KK_TAIL, launch_tail(ta, st));
   }
 #undef RUN

@@ -38,7 +38,9 @@ class RollingSession:
         self.released = t.empty((Bn, A), device=self.device, dtype=t.float32)
         self.velocity = t.empty((Bn, H, A), device=self.device, dtype=t.float32)
         # persistent step inputs: the step graph is captured on their addresses
-        self.slot_times = t.zeros((H,), device=self.device, dtype=t.float32)
+        # one schedule for every robot, or one per robot
+        nt = Bn * H if getattr(self.cfg, "per_robot_times", 0) else H
+        self.slot_times = t.zeros((nt,), device=self.device, dtype=t.float32)
         self.obs = t.zeros((Bn, self.cfg.fop_tokens, self.cfg.width), device=self.device, dtype=self.dtype)
         self.delta = t.zeros((Bn,), device=self.device, dtype=t.float32)
         B.ravel_reset(self.handle, Bn, seeds, self.buffer, stream)
@@ -60,7 +62,8 @@ class RollingSession:
         targets and the expert works relative to that state (see
         ravel_roll_step_rel and set_relative_dims)."""
         t = self.torch
-        self.slot_times.copy_(self.to_dev(slot_times, t.float32))
+        ts = self.to_dev(slot_times, t.float32).reshape(-1)
+        self.slot_times[:ts.numel()].copy_(ts)
         if self.cfg.fop_tokens:
             self.obs.copy_(self.to_dev(obs))
         self.delta.copy_(self.to_dev(delta, t.float32))

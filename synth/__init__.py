@@ -56,6 +56,7 @@ class ExpertConfig:
     # k > 0: they enter layers k-1, 2k-1, ... through gated cross-attention
     # adapters instead (and are not keys of the self-attention)
     fop_adapter_every: int = 0
+    per_robot_times: int = 0     # 1: slot times [B, H], one schedule per robot
 
     @property
     def n_adapters(self) -> int:
