@@ -577,7 +577,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
         bulk_copy_s2g(p.out + (size_t)(b * p.H + jj) * p.ld_out + (size_t)(g * p.G + r % p.G) * p.hd, srow,
                       (uint32_t)(2 * p.hd));
         bulk_commit();
-        bulk_wait<0>();   // written out before the shared memory goes away
+        bulk_wait_read<0>();   // read out before the shared memory goes away
       }
     } else if (p.xch) {
       // rows holding a slot: (m, l) to every rank; O / l as bf16, head-dim

@@ -62,7 +62,7 @@ constexpr int STG_LD = 132;                  // SIMT staging pitch (floats): 16 
 constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
 constexpr uint32_t XCH_BYTES = 32 * STG_LD * 4;  // GeGLU transpose tile (TMA epilogue): <= 32 tokens x 128 rows
 
-enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3 };
+enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3, RED_DSMEM32 = 4 };
 // Epilogue kind of an instantiation: outputs through TMA boxes as fp32, bf16
 // (+ the V^T side output), a reduce-add into the fp32 residual stream or the
 // GeGLU pair -- fixed, so that a long persistent launch carries only the code
@@ -99,7 +99,7 @@ struct TcParams {
   uint32_t stg_off;     // SIMT transpose tile, or two TMA output boxes
   uint32_t xch_off;     // GeGLU exchange
   uint32_t vts_off;     // V^T side output (TMA epilogue): the chunk as [128 tile rows][box_m + 10] bf16
-  uint32_t rcv_off;     // RED_DSMEM: the partials received from the splits, [split][cpr / 4][128 rows]
+  uint32_t rcv_off;     // RED_DSMEM*: the partials received from the splits, [split][cpr / 4][128 rows]
                         // float4, overlaid on the operand ring (free once every CTA of the cluster
                         // has finished its MMAs), else on the output boxes + exchange (used only
                         // after the sum)
@@ -238,8 +238,27 @@ __device__ __forceinline__ void reduce_slice_l2(const float* b0, int S, size_t s
 }
 
 // v[4g + e] (g < NG <= 8) = sum over splits s = 0..S-1 (in order) of the
-// received partials: b0 points at this thread's row of split 0, group 0;
-// group g of split s is (s * NG + g) * 128 float4 further.
+// received bf16 partials: b0 points at this thread's four tokens of split 0,
+// group 0 (half of a two-row message); group g of split s is (s * NG + g) *
+// 128 uint2 further.
+template <int NG>
+__device__ __forceinline__ void reduce_slice_smem(const uint2* b0, int S, float v[32]) {
+  for (int s = 0; s < S; ++s) {
+    uint2 x[NG];
+#pragma unroll
+    for (int g = 0; g < NG; ++g) x[g] = b0[(size_t)(s * NG + g) * TC_BM];
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      v[4 * g] += __uint_as_float(x[g].x << 16);
+      v[4 * g + 1] += __uint_as_float(x[g].x & 0xFFFF0000u);
+      v[4 * g + 2] += __uint_as_float(x[g].y << 16);
+      v[4 * g + 3] += __uint_as_float(x[g].y & 0xFFFF0000u);
+    }
+  }
+}
+
+// As above for fp32 partials: b0 points at this thread's row of split 0,
+// group 0; group g of split s is (s * NG + g) * 128 float4 further.
 template <int NG>
 __device__ __forceinline__ void reduce_slice_smem(const float4* b0, int S, float v[32]) {
   for (int s = 0; s < S; ++s) {
@@ -474,7 +493,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;      // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
-  uint64_t* rcv_bar = acc_empty + 2;    // RED_DSMEM: every split's slice of this rank has arrived
+  uint64_t* rcv_bar = acc_empty + 2;    // RED_DSMEM*: every split's slice of this rank has arrived
   uint32_t* tmem_slot = (uint32_t*)(rcv_bar + 1);
   int* flags = (int*)(tmem_slot + 1);   // [0] abort, [1] last split, [2] issued, [3] consumed
 
@@ -487,6 +506,9 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
   const int npre = has_work ? min(S, kb1_first - kb0_first) : 0;
   const int cpr = BN / p.splits;   // tokens of the slice each split rank owns (a multiple of 4)
   constexpr bool TMA_OUT = EK != EK_GENERIC;
+  // partials exchanged through distributed shared memory: RED_DSMEM in bf16
+  // (two rows per message), RED_DSMEM32 in fp32
+  constexpr bool DSM = RED == RED_DSMEM || RED == RED_DSMEM32;
 
   pdl_trigger();
   uint64_t pol_w = 0, pol_x = 0;
@@ -499,11 +521,11 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 128);
     }
-    mbar_init(rcv_bar, 1);   // RED_DSMEM: the partials' arrival; otherwise armed by nobody
+    mbar_init(rcv_bar, 1);   // RED_DSMEM*: the partials' arrival; otherwise armed by nobody
     flags[0] = flags[1] = flags[2] = flags[3] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // the slices of all splits (this one's included): 128 rows x cpr tokens each
-    if constexpr (RED == RED_DSMEM) mbar_expect_tx(rcv_bar, (uint32_t)(BN * TC_BM * 4));
+    if constexpr (DSM) mbar_expect_tx(rcv_bar, (uint32_t)(BN * TC_BM * (RED == RED_DSMEM ? 2 : 4)));
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     // Weights never depend on earlier kernels: stream the first stages' weight
     // tiles while the previous kernel is still finishing.
@@ -584,9 +606,9 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       flags[2] = it;
     }
     __syncwarp();
-    // RED_DSMEM: one arrival per thread on the cluster barrier that opens the
+    // RED_DSMEM*: one arrival per thread on the cluster barrier that opens the
     // exchange (the epilogue warps arrive once their MMAs are complete)
-    if constexpr (RED == RED_DSMEM) cluster_arrive_release();
+    if constexpr (DSM) cluster_arrive_release();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(TC_BM, BN);
@@ -594,7 +616,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       bool ok = true;
       int tn, tm, sp;
       // fault injection: an arrival that never comes (rcv_bar is armed by
-      // nobody outside RED_DSMEM, which the host never combines with this)
+      // nobody outside the RED_DSMEM modes, which the host never combines with this)
       if (p.withhold && !mbar_wait(rcv_bar, 0, p.wait_ns)) {
         flags[0] = 1;
         ok = false;
@@ -646,7 +668,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       flags[3] = it;
     }
     __syncwarp();
-    if constexpr (RED == RED_DSMEM) cluster_arrive_release();
+    if constexpr (DSM) cluster_arrive_release();
   } else {
     // epilogue warps 2..5: TMEM lane quarter q = warp % 4, tile row r
     const int q = warp & 3;
@@ -656,7 +678,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     for (int i = 0; work_item(p, i, tn, tm, sp); ++i) {
       const int b = i & 1;
       const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[b], (uint32_t)(i >> 1) & 1u, p.wait_ns));
-      if constexpr (RED == RED_DSMEM) {
+      if constexpr (DSM) {
         // past this barrier every CTA of the cluster has finished its MMAs
         // (its operand ring may be overwritten) and armed its receive barrier;
         // every thread arrives exactly once, whatever happened before
@@ -698,6 +720,48 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
           }
         }
       } else if constexpr (RED == RED_DSMEM) {
+        // token slice q of this split's partial goes to rank q (= split q) of
+        // the cluster in bf16, two rows per 16-byte message: the lanes of rows
+        // r and r+1 swap halves of their packed 4-token groups 2k and 2k+1,
+        // so that the even lane sends group 2k of both rows and the odd lane
+        // group 2k+1; group g of the slice for row pair r/2 lands at
+        // [sp][g][r/2] there
+        const int ngs = cpr / 4;
+        const bool odd = lane & 1;
+        const uint32_t rcv0 = smem_u32(smem + p.rcv_off) + (uint32_t)(sp * ngs * 64 + (r >> 1)) * 16u;
+        const uint32_t bar0 = smem_u32(rcv_bar);
+        // destination rank and group of this lane's next message (group 2k + odd)
+        int dst = (odd && ngs == 1) ? 1 : 0, gl = (odd && ngs > 1) ? 1 : 0;
+        for (int c0 = 0; c0 < BN; c0 += 64) {   // up to four TMEM loads in flight, one wait
+          const int nq = min(4, (BN - c0) / 16);   // BN is a multiple of 16
+          uint32_t raw[64];
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq)
+            if (qq < nq) tmem_ld16_async(trow + c0 + 16 * qq, raw + 16 * qq);
+          tmem_wait_ld();
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) tmem_reg_fence16(raw + 16 * qq);
+          for_upto<8, 2>(2 * nq, [&](int k) {
+            const uint32_t* a = raw + 8 * k;
+            const uint32_t p0 = pack_bf16x2(__uint_as_float(a[0]), __uint_as_float(a[1]));
+            const uint32_t p1 = pack_bf16x2(__uint_as_float(a[2]), __uint_as_float(a[3]));
+            const uint32_t p2 = pack_bf16x2(__uint_as_float(a[4]), __uint_as_float(a[5]));
+            const uint32_t p3 = pack_bf16x2(__uint_as_float(a[6]), __uint_as_float(a[7]));
+            const uint32_t got0 = __shfl_xor_sync(0xffffffffu, odd ? p0 : p2, 1);
+            const uint32_t got1 = __shfl_xor_sync(0xffffffffu, odd ? p1 : p3, 1);
+            const uint4 w = odd ? make_uint4(got0, got1, p2, p3) : make_uint4(p0, p1, got0, got1);
+            st_async_u4(mapa_shared(rcv0 + (uint32_t)gl * 1024u, (uint32_t)dst), w, mapa_shared(bar0, (uint32_t)dst));
+            // two groups on: a select per rank boundary, not a branch
+            gl += 2;
+            bool wrap = gl >= ngs;
+            gl = wrap ? gl - ngs : gl;
+            dst += wrap ? 1 : 0;
+            wrap = gl >= ngs;
+            gl = wrap ? gl - ngs : gl;
+            dst += wrap ? 1 : 0;
+          });
+        }
+      } else if constexpr (RED == RED_DSMEM32) {
         // token slice q of this split's partial goes to rank q (= split q) of
         // the cluster: float4 group g of the slice lands at [sp][g][r] there
         const int ngs = cpr / 4;
@@ -783,8 +847,9 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         }
       }
     }
-    // every TMA output box has been written to global memory
-    if (TMA_OUT && threadIdx.x == 64) bulk_wait<0>();
+    // every TMA output box has been read out of shared memory (the grid's
+    // completion makes the writes visible to the dependent launch)
+    if (TMA_OUT && threadIdx.x == 64) bulk_wait_read<0>();
   }
   tc_fence_before();
   cta_sync();
@@ -796,7 +861,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
     }
     cta_sync();
   }
-  if constexpr (RED == RED_DSMEM) {
+  if constexpr (DSM) {
     // Rank q sums its slice of tokens [q*cpr, (q+1)*cpr) over the splits in
     // order once every split's bytes have arrived (the wait also keeps this
     // CTA alive until no store into its shared memory is in flight), then
@@ -811,23 +876,37 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       } else {
         const int n = tn0 * TC_BM + r;
         const float brow = (p.bias && n < p.N) ? p.bias[n] : 0.f;
-        const float4* b0 = (const float4*)(smem + p.rcv_off) + r;
         float v[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) v[k] = 0.f;
-        switch (cpr / 4) {
-          case 1: reduce_slice_smem<1>(b0, p.splits, v); break;
-          case 2: reduce_slice_smem<2>(b0, p.splits, v); break;
-          case 3: reduce_slice_smem<3>(b0, p.splits, v); break;
-          case 4: reduce_slice_smem<4>(b0, p.splits, v); break;
-          case 5: reduce_slice_smem<5>(b0, p.splits, v); break;
-          case 6: reduce_slice_smem<6>(b0, p.splits, v); break;
-          case 7: reduce_slice_smem<7>(b0, p.splits, v); break;
-          default: reduce_slice_smem<8>(b0, p.splits, v); break;
+        if constexpr (RED == RED_DSMEM) {
+          const uint2* b0 = (const uint2*)(smem + p.rcv_off) + 2 * (r >> 1) + (r & 1);
+          switch (cpr / 4) {
+            case 1: reduce_slice_smem<1>(b0, p.splits, v); break;
+            case 2: reduce_slice_smem<2>(b0, p.splits, v); break;
+            case 3: reduce_slice_smem<3>(b0, p.splits, v); break;
+            case 4: reduce_slice_smem<4>(b0, p.splits, v); break;
+            case 5: reduce_slice_smem<5>(b0, p.splits, v); break;
+            case 6: reduce_slice_smem<6>(b0, p.splits, v); break;
+            case 7: reduce_slice_smem<7>(b0, p.splits, v); break;
+            default: reduce_slice_smem<8>(b0, p.splits, v); break;
+          }
+        } else {
+          const float4* b0 = (const float4*)(smem + p.rcv_off) + r;
+          switch (cpr / 4) {
+            case 1: reduce_slice_smem<1>(b0, p.splits, v); break;
+            case 2: reduce_slice_smem<2>(b0, p.splits, v); break;
+            case 3: reduce_slice_smem<3>(b0, p.splits, v); break;
+            case 4: reduce_slice_smem<4>(b0, p.splits, v); break;
+            case 5: reduce_slice_smem<5>(b0, p.splits, v); break;
+            case 6: reduce_slice_smem<6>(b0, p.splits, v); break;
+            case 7: reduce_slice_smem<7>(b0, p.splits, v); break;
+            default: reduce_slice_smem<8>(b0, p.splits, v); break;
+          }
         }
         int ebuf = 0;
         if constexpr (TMA_OUT) epilogue_tma<EK, 32>(p, &tmO, tn0, tm0 * BN + sp0 * cpr, r, v, brow, stg_raw, xch, ebuf);
-        if (threadIdx.x == 64) bulk_wait<0>();
+        if (threadIdx.x == 64) bulk_wait_read<0>();
       }
     }
   }
@@ -878,7 +957,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         if constexpr (TMA_OUT) epilogue_tma<EK>(p, &tmO, tn0, m0, r, v, brow, stg_raw, xch, ebuf);
         else epilogue_chunk(p, tn0, m0, nc, r, v, stage);
       }
-      if (TMA_OUT && threadIdx.x == 64) bulk_wait<0>();
+      if (TMA_OUT && threadIdx.x == 64) bulk_wait_read<0>();
     }
   }
   if (warp == 1) {
@@ -1105,7 +1184,7 @@ __global__ void __launch_bounds__(TC_PAIR_THREADS, 1)
         }
       }
     }
-    if (threadIdx.x == 64 + 128 * set) bulk_wait<0>();   // this set's stores are complete
+    if (threadIdx.x == 64 + 128 * set) bulk_wait_read<0>();   // this set's boxes have been read out
   }
   tc_fence_before();
   cta_sync();
@@ -1148,7 +1227,7 @@ TcKernel tc_kernel(int red, int ek) {
   RAVEL_TC_K(RED_NONE, EK_F32) RAVEL_TC_K(RED_NONE, EK_BF16) RAVEL_TC_K(RED_NONE, EK_ADD)
   RAVEL_TC_K(RED_NONE, EK_GEGLU) RAVEL_TC_K(RED_NONE, EK_GENERIC)
   RAVEL_TC_K(RED_L2_CLUSTER, EK_TMA_ANY) RAVEL_TC_K(RED_L2_CLUSTER, EK_GENERIC)
-  RAVEL_TC_K(RED_DSMEM, EK_TMA_ANY)
+  RAVEL_TC_K(RED_DSMEM, EK_TMA_ANY) RAVEL_TC_K(RED_DSMEM32, EK_TMA_ANY)
   RAVEL_TC_K(RED_WORKSPACE, EK_GENERIC)
 #undef RAVEL_TC_K
   return nullptr;
@@ -1308,7 +1387,7 @@ cudaError_t init_tc_gemm() {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
   std::vector<const void*> kernels;
-  for (int red = 0; red < 4; ++red)
+  for (int red = 0; red < 5; ++red)
     for (int ek = 0; ek <= EK_TMA_ANY; ++ek)
       if (TcKernel k = tc_kernel(red, ek)) kernels.push_back((const void*)k);
   for (int ek = 0; ek < EK_GENERIC; ++ek) kernels.push_back((const void*)tc_pair_kernel(ek));
@@ -1407,6 +1486,8 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   const int es = out_bf ? 2 : 4;
   const bool tma_out = reduce != RED_WORKSPACE && ((uintptr_t)g.out & 15) == 0 && ((size_t)g.ldo * es) % 16 == 0;
   int box_m = 0;
+  // partials exchanged in bf16 where the caller allows it, else in fp32
+  const bool xbf = g.xbf16 != 0;
   uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, vts_off = 0, rcv_off = 0, bar_off = 0;
   size_t smem = 0;
   auto layout = [&](bool dsmem) {
@@ -1419,7 +1500,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
     const size_t vts_bytes = (tma_out && g.vt) ? ((size_t)TC_BM * (box_m + 10) * 2 + 1023) / 1024 * 1024 : 0;
     // received partials (all splits' slices of this rank) overlay the operand
     // ring, else the boxes + exchange
-    const size_t rcv_bytes = dsmem ? (size_t)TC_BM * bn * 4 : 0;
+    const size_t rcv_bytes = dsmem ? (size_t)TC_BM * bn * (xbf ? 2 : 4) : 0;
     const bool in_ring = rcv_bytes <= ring;
     xch_off = stg_off + (uint32_t)stg_bytes;
     vts_off = xch_off + (uint32_t)xch_bytes;
@@ -1435,7 +1516,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
     dsmem = false;
     layout(false);
   }
-  if (dsmem) reduce = RED_DSMEM;
+  if (dsmem) reduce = xbf ? RED_DSMEM : RED_DSMEM32;
   CUtensorMap mw, mx, mo;
   memset(&mo, 0, sizeof(mo));
   cudaError_t e = oneshot ? encode_kt(&mw, g.W, g.N, g.K, g.ldw, TC_BM, kb_per_item)
@@ -1465,7 +1546,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
                  : g.epi == EPI_GEGLU ? EK_GEGLU : g.epi == EPI_ADD_F32 ? EK_ADD : out_bf ? EK_BF16 : EK_F32;
   const TcKernel k = tc_kernel(reduce, ek);
   if (!k) return cudaErrorInvalidConfiguration;
-  const bool clustered = reduce == RED_L2_CLUSTER || reduce == RED_DSMEM;
+  const bool clustered = reduce == RED_L2_CLUSTER || reduce == RED_DSMEM || reduce == RED_DSMEM32;
   return launch_kernel(k, grid, block, smem, st, clustered ? (unsigned)splits : 1u, mw, mx, mo, p);
 }
 

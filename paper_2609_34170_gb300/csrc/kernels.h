@@ -90,6 +90,10 @@ struct GemmArgs {
   int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
   int max_splits = 0;           // tcgen05 path: cap on the split-K factor (0: chosen from the shape)
   const int* skip = nullptr;    // optional device flag: nonzero at run time -> the launch computes nothing
+  // tcgen05 split-K inside a cluster: the splits' partials may travel between
+  // the SMs in bf16 (half the bytes of fp32; the sum itself stays fp32), which
+  // the step's projections take; 0 keeps them in fp32
+  int xbf16 = 0;
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, Dtype dt, cudaStream_t st);
 

@@ -313,10 +313,11 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     }                                   \
   } while (0)
   auto gemm = [&](const void* Aop, int lda, const void* W, int M, int N, int K, Epi epi, void* out, int ldo,
-                  Dtype out_dt, const float* bias, int split_cap = 0, const int* skip = nullptr) {
+                  Dtype out_dt, const float* bias, int split_cap = 0, const int* skip = nullptr, int xbf16 = 0) {
     GemmArgs g{Aop, lda, W, K, M, N, K, epi, out, ldo, out_dt, bias};
     g.max_splits = split_cap;
     g.skip = skip;
+    g.xbf16 = xbf16;
     return run_gemm(p, g, st);
   };
   auto rowp = [&](const void* base, size_t row, size_t ld) { return (const void*)((const char*)base + row * ld * es); };
@@ -382,6 +383,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       gq.vt_kvp = p.kvp;
       gq.vt_hkv = c.n_kv_heads;
       gq.max_splits = p.split_cap[0];
+      gq.xbf16 = 1;
       RUN(KK_GEMM_QKV, run_gemm(p, gq, st));
       AttnTcArgs at{p.QKV, p.nqkv, p.Vt, p.kvp, {p.ctx_k[0], p.ctx_k[1]}, {p.ctx_v[0], p.ctx_v[1]}, L, l,
                     c.max_batch, c.max_prefix, p.pst, p.ctx_state, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim,
@@ -397,7 +399,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       RUN(KK_ATTENTION, launch_attention_simt(at, dt, st));
     }
     RUN(KK_GEMM_O, gemm(p.O, p.qdim, (const char*)p.w_o + (size_t)l * D * p.qdim * es, BH, D, p.qdim, EPI_ADD_F32, p.x,
-                        D, DT_F32, nullptr, p.split_cap[1]));
+                        D, DT_F32, nullptr, p.split_cap[1], nullptr, 1));
     if (adapters && (l + 1) % c.fop_adapter_every == 0) {
       // gated cross-attention adapter: the action rows attend to the FOP tokens
       const int ai = (l + 1) / c.fop_adapter_every - 1, nkv = 2 * c.n_kv_heads * c.head_dim;
@@ -421,6 +423,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     const void* wgu = (const char*)p.w_gu + (size_t)l * 2 * Fm * D * es;
     GemmArgs gu{p.Y, D, wgu, D, BH, 2 * Fm, D, EPI_GEGLU, p.Hm, Fm, dt, nullptr};
     gu.max_splits = p.split_cap[2];
+    gu.xbf16 = 1;
     if (p.use_tc && tc_gemm_supported(gu)) {
       RUN(KK_GEMM_GATE_UP, launch_gemm_tc(gu, p.tcws, p.num_sms, st));   // GeGLU fused in the epilogue
     } else {
@@ -428,7 +431,7 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
       RUN(KK_GEGLU, launch_geglu(p.GU, BH, Fm, p.Hm, dt, st));
     }
     RUN(KK_GEMM_DOWN, gemm(p.Hm, Fm, (const char*)p.w_down + (size_t)l * D * Fm * es, BH, D, Fm, EPI_ADD_F32, p.x, D,
-                           DT_F32, nullptr, p.split_cap[3]));
+                           DT_F32, nullptr, p.split_cap[3], nullptr, 1));
   }
   if (!dn && dt == DT_BF16 && A <= 32 && D % 4 == 0) {
     // final norm, velocity head and tail in one launch, about eight CTAs per SM
