@@ -315,11 +315,14 @@ __device__ __forceinline__ float4 ld4(const bf16* p) {
 //   FOP row (b, f):     y = z * rsqrt(mean(z^2) + eps) * (1 + gamma)
 // A thread owns columns 4*tid + 1024*g (g < G) of every row of the block, so
 // the per-robot part M_delta[b] + bias (or gamma) is read once per block and
-// kept in registers; rows go through in batches of R with one barrier each
-// (the batch's row sums are reduced through a double-buffered table).
+// kept in registers; rows go through one at a time with one barrier each
+// (the row sums are reduced through a double-buffered table).  Few rows per
+// block: the row's loads are the block's critical path, and spreading the
+// rows over more blocks (one each when they fit the SMs) beat batching four
+// rows per round trip.
 template <typename T, int G>
 __global__ void __launch_bounds__(256) ada_norm_kernel(NormArgs a, int rb_act, int nb_act, int rb_fop, int nb_fop) {
-  constexpr int R = (G >= 4) ? 1 : 4 / G;
+  constexpr int R = 1;
   __shared__ float red[2][R][8];
   pdl_trigger();
   const int D = a.D, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -441,10 +444,9 @@ cudaError_t launch_ada_norm_t(const NormArgs& a, cudaStream_t st) {
       g_norm_sms = 132;
   }
   const int G = (a.D + 1023) / 1024;
-  const int R = (G >= 4) ? 1 : 4 / G;
-  // rows per block: one batch of R rows, so that every block's loads are in
-  // flight at once (a block that walks several batches pays one L2 round
-  // trip per batch); up to 8 blocks of 256 threads are resident per SM
+  const int R = 1;
+  // rows per block: as few as fill up to 8 resident blocks of 256 threads per
+  // SM (one row each when the rows fit)
   const int nf = a.fop ? a.F : 0;
   const int total = a.B * (a.H + nf);
   int rb_all = (total + 8 * g_norm_sms - 1) / (8 * g_norm_sms);
