@@ -243,6 +243,7 @@ __device__ __forceinline__ void reduce_slice_l2(const float* b0, int S, size_t s
 // 128 uint2 further.
 template <int NG>
 __device__ __forceinline__ void reduce_slice_smem(const uint2* b0, int S, float v[32]) {
+  #pragma unroll 1
   for (int s = 0; s < S; ++s) {
     uint2 x[NG];
 #pragma unroll
@@ -261,6 +262,7 @@ __device__ __forceinline__ void reduce_slice_smem(const uint2* b0, int S, float 
 // group 0; group g of split s is (s * NG + g) * 128 float4 further.
 template <int NG>
 __device__ __forceinline__ void reduce_slice_smem(const float4* b0, int S, float v[32]) {
+  #pragma unroll 1
   for (int s = 0; s < S; ++s) {
     float4 x[NG];
 #pragma unroll
@@ -587,6 +589,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
       int tn, tm, sp;
       for (int i = 0; ok && work_item(p, i, tn, tm, sp); ++i) {
         const int kb0 = (int)((long)sp * p.num_kb / p.splits), kb1 = (int)((long)(sp + 1) * p.num_kb / p.splits);
+        #pragma unroll 1
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % S;
           if (it < npre) {   // weight tile already in flight
@@ -625,6 +628,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         ok = mbar_wait(&full[0], 0, p.wait_ns);
         if (ok) {
           tc_fence_after();
+          #pragma unroll 1
           for (int kb = 0; kb < kb1_first - kb0_first; ++kb) {
             const uint64_t ad = sw128_desc(smem_u32(a_s + (size_t)kb * TC_A_BYTES));
             const uint64_t bd = sw128_desc(smem_u32(b_s + (size_t)kb * b_bytes));
@@ -648,6 +652,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)b * p.acc_cols;
         const int kb0 = (int)((long)sp * p.num_kb / p.splits), kb1 = (int)((long)(sp + 1) * p.num_kb / p.splits);
+        #pragma unroll 1
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % S;
           if (!mbar_wait(&full[s], (uint32_t)(it / S) & 1u, p.wait_ns)) {
@@ -701,6 +706,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         tmem_ld16_async(trow, nxt);
         tmem_wait_ld();
         tmem_reg_fence16(nxt);
+        #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 16) {
           float v[16];
 #pragma unroll
@@ -732,6 +738,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         const uint32_t bar0 = smem_u32(rcv_bar);
         // destination rank and group of this lane's next message (group 2k + odd)
         int dst = (odd && ngs == 1) ? 1 : 0, gl = (odd && ngs > 1) ? 1 : 0;
+        #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 64) {   // up to four TMEM loads in flight, one wait
           const int nq = min(4, (BN - c0) / 16);   // BN is a multiple of 16
           uint32_t raw[64];
@@ -768,6 +775,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         const uint32_t rcv0 = smem_u32(smem + p.rcv_off) + (uint32_t)(sp * ngs * TC_BM + r) * 16u;
         const uint32_t bar0 = smem_u32(rcv_bar);
         int dst = 0, gl = 0;   // destination rank and group of the next float4
+        #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 64) {   // up to four TMEM loads in flight, one wait
           const int nq = min(4, (BN - c0) / 16);   // BN is a multiple of 16
           uint32_t raw[64];
@@ -792,6 +800,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         // thread stores float4 of 4 consecutive columns, a warp one 512-byte run
         const size_t cl = (size_t)tm * gridDim.x + tn;
         float* w = p.ws + ((cl * p.splits + sp) * (size_t)(BN / 4)) * (TC_BM * 4) + (size_t)r * 4;
+        #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 64) {   // up to four TMEM loads in flight, one wait
           const int nq = min(4, (BN - c0) / 16);   // BN is a multiple of 16
           uint32_t raw[64];
@@ -813,6 +822,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         // workspace mode: [split][tile][col][row] partials, last arrival reduces
         const int tiles = gridDim.x * gridDim.y;
         const int tile_id = tm * gridDim.x + tn;
+        #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 16) {
           float v[16];
           tmem_ld16(trow + c0, v);
@@ -829,6 +839,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         epi_bar();
         if (flags[1]) {
           __threadfence();
+          #pragma unroll 1
           for (int c0 = 0; c0 < BN; c0 += 16) {
             float v[16];
 #pragma unroll
@@ -944,6 +955,7 @@ __global__ void __launch_bounds__(TC_THREADS, 2)
         }
         if constexpr (TMA_OUT) epilogue_tma<EK, 32>(p, &tmO, tn0, tm0 * BN + rank * cpr, r, v, brow, stg_raw, xch, ebuf);
       }
+      #pragma unroll 1
       for (int cc = 0; !whole && cc < cpr; cc += p.box_m) {
         const int nc = p.box_m;
         float v[16];
