@@ -44,7 +44,10 @@
 namespace ravel {
 namespace {
 
-constexpr int AT_THREADS = 192;
+// warp 0: loads; warp 1: MMAs; warps 2-5: softmax (a thread per query row);
+// warps 6-7 join only the merge of the key splits, so that each thread takes
+// one (row, 8-column) item of a 64-row tile's slice instead of two
+constexpr int AT_THREADS = 256;
 constexpr int AT_BM = 128;
 constexpr int AT_BKV = 64;
 constexpr int AT_SMEM_MAX = 227 * 1024;
@@ -437,6 +440,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     }
     __syncwarp();
     if (p.xch == 1) cluster_arrive_release();
+  } else if (warp >= 6) {
+    // merge-only warps: one arrival on the cluster barrier that opens the exchange
+    if (p.xch == 1) cluster_arrive_release();
   } else {
     // softmax / epilogue: thread owns query row r (TMEM lane r)
     const int q4 = warp & 3;
@@ -717,7 +723,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     // published its (O, m, l), rank q merges head-dim columns
     // [q*hdp/S, (q+1)*hdp/S):  O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
     cluster_sync();
-    if (warp >= 2) {
+    if (warp >= 2 && warp < 6) {
       const int r = (warp & 3) * 32 + lane;
       const int Sp = p.splits;
       const int cps = p.hdp / Sp;   // a multiple of 4
