@@ -70,7 +70,10 @@ typedef struct {
   int max_batch;    /* largest B accepted by ravel_reset */
   int dtype;        /* RAVEL_FP32: all arithmetic fp32; RAVEL_BF16: weights, prefix,
                        FOP tokens and GEMM activations bf16, fp32 accumulation,
-                       fp32 residual stream, norms, softmax and buffer */
+                       fp32 residual stream, norms, softmax and buffer; where a
+                       projection or the attention splits its reduction over
+                       SMs (few tokens), each split's share crosses between
+                       the SMs as bf16 and the shares are summed in fp32 */
   int mask_mode;    /* RAVEL_MASK_FULL: every action query sees the valid prefix,
                        all FOP tokens and all H slots; RAVEL_MASK_SLOT_ISOLATED
                        (a test mode): action query j sees the prefix, the FOP
@@ -270,6 +273,8 @@ ravel_status ravel_profile_step(ravel_t* r, float* buffer, const float* slot_tim
  *          gelu_tanh(gate + bias) * (up + bias) for f < N/2, each bias
  *          that of its W row
  *   out device [M, ldo], out_dtype RAVEL_FP32 or RAVEL_BF16; bias device [N] or NULL
+ * Accumulation is fp32 throughout and split-K partials stay fp32 here (the
+ * step's own projections send theirs between the SMs as bf16).
  * Enqueued on `stream`; uses the handle's split-K workspace, so it must not
  * overlap another call on the same handle.  Like ravel_roll_step it first
  * reports a device error raised by earlier work (RAVEL_EDEVICE /
