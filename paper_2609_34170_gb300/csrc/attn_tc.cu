@@ -59,11 +59,10 @@ struct AtParams {
   int TQ, q_tiles;
   int Pmax, n_pre, n_kv, splits;
   int layer, Bmax, mask_mode;
-  int nblk, k_slots, v_slots;         // head-dim blocks of 64; K and V^T ring depths
+  int nblk, k_slots, v_slots;         // head-dim blocks of 64; K and V ring depths
   int xch;                            // splits > 1: partials through L2 (0) or shared memory, sent once every
                                       // split's MMAs are done (1: cluster barrier) or once every split's S
                                       // MMAs are done (2: the receive area lies in Q and the K ring)
-  uint32_t vt_bytes;                  // bytes of one transposed-V chunk (hd rows x 128 B)
   const int* ctx_state;
   bf16* out;
   int ld_out;
@@ -73,8 +72,10 @@ struct AtParams {
   float scale_log2;                   // log2(e) / sqrt(hd)
 };
 
+// K and V chunks alike: [64 keys][64-wide head-dim block] boxes, 128-byte
+// swizzled; V is the B operand of P V in its natural layout (MN-major)
 struct AtMaps {
-  CUtensorMap q, k, vt, pk0, pk1, pv0, pv1;
+  CUtensorMap q, k, v, pk0, pk1, pv0, pv1;
 };
 
 // The idx-th chunk this CTA processes (prefix chunks past the valid prefix
@@ -189,12 +190,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   // 1024-byte aligned; derived from smem_raw by pointer arithmetic so that the
   // compiler keeps it (and everything indexed from it) in the shared window
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  const int SK = p.k_slots, SV = p.v_slots;   // K and V^T ring depths
-  const uint32_t k_bytes = (uint32_t)p.nblk * AT_KBLK;
+  const int SK = p.k_slots, SV = p.v_slots;   // K and V ring depths
+  const uint32_t k_bytes = (uint32_t)p.nblk * AT_KBLK;   // one K or V chunk
   uint8_t* q_s = smem;
-  uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;   // K ring, then V^T ring
+  uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;   // K ring, then V ring
   uint8_t* v_ring = kv_s + (size_t)SK * k_bytes;
-  uint64_t* bars = (uint64_t*)(v_ring + (size_t)SV * p.vt_bytes);
+  uint64_t* bars = (uint64_t*)(v_ring + (size_t)SV * k_bytes);
   // K and V^T of a stage have their own barriers: K is released as soon as
   // S = Q K^T has been computed, V^T only after P V, so the next K load does
   // not wait for the softmax and the PV of the chunk it replaces
@@ -278,12 +279,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
     for (int blk = 0; blk < p.nblk; ++blk) tma_load_3d(km, &k_full[s], ks + (size_t)blk * AT_KBLK, blk * 64, ky, kz, pol);
   };
   auto load_v = [&](int c, int s, uint64_t pol) {
-    uint8_t* vs = v_ring + (size_t)s * p.vt_bytes;
-    mbar_expect_tx(&v_full[s], 128u * (uint32_t)p.hd);
+    uint8_t* vs = v_ring + (size_t)s * k_bytes;
+    mbar_expect_tx(&v_full[s], k_bytes);
     const bool pre = c < p.n_pre;
     const int cc = c - p.n_pre;
-    const int vx = (pre ? c : cc) * AT_BKV, vz = pre ? ctx_z : b * p.Hkv + g;
-    tma_load_3d(pre ? pv : &maps.vt, &v_full[s], vs, vx, 0, vz, pol);
+    const CUtensorMap* vm = pre ? pv : &maps.v;
+    const int vy = pre ? c * AT_BKV : g, vz = pre ? ctx_z : b * rows_per_robot + cc * AT_BKV;
+    for (int blk = 0; blk < p.nblk; ++blk) tma_load_3d(vm, &v_full[s], vs + (size_t)blk * AT_KBLK, blk * 64, vy, vz, pol);
   };
   if (threadIdx.x == 0) {
     uint64_t pol_kv;
@@ -373,7 +375,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc_s = idesc_bf16(AT_BM, AT_BKV);
-      const uint32_t idesc_o = idesc_bf16(AT_BM, p.hdp);
+      const uint32_t idesc_o = idesc_bf16_bmn(AT_BM, p.hdp);
       bool ok = mbar_wait(q_full, 0);
       // Issue S of the next chunk and PV of the oldest chunk whose P is ready,
       // whichever can go: PV(i) never waits for chunk i+1's K/V (that would
@@ -417,10 +419,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
           const int s = i % SV;
           // A = P from TMEM (the S tile's first 32 columns, two bf16 per column)
           const uint32_t pa = tmem + (uint32_t)(i & 1) * AT_BKV;
-          const uint64_t bd = sw128_desc(smem_u32(v_ring + (size_t)s * p.vt_bytes));
+          // B = V [64 keys][hd], MN-major: 16 keys (two 8-row groups) per K step
+          const uint64_t bd = sw128_mn_desc(smem_u32(v_ring + (size_t)s * k_bytes), AT_KBLK);
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_bf16_ts(tmem + o_col, pa + 8 * k, bd + 2 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
+            umma_bf16_ts(tmem + o_col, pa + 8 * k, bd + 128 * k, idesc_o, (i > 0 || k > 0) ? 1u : 0u);
           umma_commit(&v_empty[s]);
           umma_commit(&pv_done[i & 1]);
           ++i;
@@ -829,7 +832,6 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   p.n_kv = (a.H + a.F + AT_BKV - 1) / AT_BKV;
   p.layer = a.layer; p.Bmax = a.Bmax; p.mask_mode = a.mask_mode;
   p.nblk = (a.hd + 63) / 64;
-  p.vt_bytes = (uint32_t)((p.hdp * 128 + 1023) / 1024 * 1024);
   p.ctx_state = a.ctx_state;
   p.out = (bf16*)a.out; p.ld_out = a.ld_out;
   p.err = a.err;
@@ -869,16 +871,16 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
   // slice, and the receive area (O groups + (m, l) of every split) within
   // Q + the rings (checked below)
   p.xch = splits > 1 && (p.hdp / splits) % 8 == 0 ? 1 : 0;
-  // K slots: as many whole K + V^T stages as fit (<= 4); V^T slots: the K
-  // count plus what the remaining bytes hold (<= 2 more): K is free again as
-  // soon as S = Q K^T is done, V^T only after P V, so V^T needs the depth
+  // K slots: as many whole K + V stages as fit (<= 4); V slots: the K count
+  // plus what the remaining bytes hold (<= 2 more): K is free again as soon
+  // as S = Q K^T is done, V only after P V, so V needs the depth
   const size_t k_bytes = (size_t)p.nblk * AT_KBLK;
-  const size_t stage = k_bytes + p.vt_bytes;
+  const size_t stage = 2 * k_bytes;
   const size_t fixed = 1024 + (size_t)p.nblk * AT_QBLK + 512;
   if (fixed + stage > (size_t)AT_SMEM_MAX) return cudaErrorInvalidConfiguration;
   const int sk = (int)std::min<size_t>(4, (AT_SMEM_MAX - fixed) / stage);
-  const int sv = sk + (int)std::min<size_t>(2, (AT_SMEM_MAX - fixed - sk * stage) / p.vt_bytes);
-  const size_t rings = (size_t)sk * k_bytes + (size_t)sv * p.vt_bytes;
+  const int sv = sk + (int)std::min<size_t>(2, (AT_SMEM_MAX - fixed - sk * stage) / k_bytes);
+  const size_t rings = (size_t)(sk + sv) * k_bytes;
   // the epilogue stages 128 bf16 rows of O in the rings and stores them with
   // 16-byte writes
   if ((size_t)AT_BM * (size_t)(((2 * p.hdp + 63) & ~63) + 16) > rings) return cudaErrorInvalidConfiguration;
@@ -900,51 +902,21 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st) {
     e = enc3(&m.k, (const bf16*)a.qkv + (size_t)a.Hq * hd, hd, a.Hkv, rows, (uint64_t)hd * 2, (uint64_t)a.ld_qkv * 2,
              64, 1, AT_BKV);
   if (e == cudaSuccess)
-    e = enc3(&m.vt, a.vt, rpr, hd, (uint64_t)a.B * a.Hkv, (uint64_t)a.kvp * 2, (uint64_t)hd * a.kvp * 2, AT_BKV, hd, 1);
+    e = enc3(&m.v, (const bf16*)a.qkv + (size_t)(a.Hq + a.Hkv) * hd, hd, a.Hkv, rows, (uint64_t)hd * 2,
+             (uint64_t)a.ld_qkv * 2, 64, 1, AT_BKV);
   const uint64_t zc = (uint64_t)(a.layers * a.Bmax * a.Hkv);
   for (int s = 0; s < 2 && e == cudaSuccess; ++s) {
     e = enc3(s ? &m.pk1 : &m.pk0, a.ctx_k[s], hd, a.Pmax, zc, (uint64_t)hd * 2, (uint64_t)a.Pmax * hd * 2, 64,
              AT_BKV, 1);
     if (e == cudaSuccess)
-      e = enc3(s ? &m.pv1 : &m.pv0, a.ctx_vt[s], a.Pmax, hd, zc, (uint64_t)a.pst * 2, (uint64_t)hd * a.pst * 2,
-               AT_BKV, hd, 1);
+      e = enc3(s ? &m.pv1 : &m.pv0, a.ctx_v[s], hd, a.Pmax, zc, (uint64_t)hd * 2, (uint64_t)a.Pmax * hd * 2, 64,
+               AT_BKV, 1);
   }
   if (e != cudaSuccess) return e;
   dim3 grid(p.q_tiles, a.B * a.Hkv, splits);
   e = launch_kernel_cluster(attn_tc_kernel, grid, dim3(AT_THREADS), smem, st, dim3(1, 1, splits), m, p);
   if (a.n_launched) ++*a.n_launched;
   return e;
-}
-
-// Context V [L][n][Hkv][P][hd] of the listed robots -> their slots
-// Vt [L][Bmax][Hkv][hd][pst] (keys contiguous).
-__global__ void transpose_ctx_v_kernel(const bf16* __restrict__ src, int src_n, int i0, bf16* __restrict__ dst0,
-                                       bf16* __restrict__ dst1, int Bmax, int Hkv, int P, int hd, int pst, CtxList f) {
-  __shared__ bf16 tile[32][33];
-  const int z = blockIdx.z;                 // (l * f.n + i) * Hkv + g
-  const int g = z % Hkv, li = z / Hkv;
-  const int i = li % f.n, l = li / f.n;
-  const bf16* s = src + ((size_t)(l * src_n + i0 + i) * Hkv + g) * P * hd;
-  bf16* d = (f.slot[i] ? dst1 : dst0) + ((size_t)(l * Bmax + f.robot[i]) * Hkv + g) * hd * pst;
-  const int p0 = blockIdx.x * 32, d0 = blockIdx.y * 32;
-  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
-    const int pp = p0 + i, dd = d0 + threadIdx.x;
-    tile[i][threadIdx.x] = (pp < P && dd < hd) ? s[(size_t)pp * hd + dd] : __float2bfloat16_rn(0.f);
-  }
-  cta_sync();
-  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
-    const int dd = d0 + i, pp = p0 + threadIdx.x;
-    if (dd < hd && pp < P) d[(size_t)dd * pst + pp] = tile[threadIdx.x][i];
-  }
-}
-
-cudaError_t launch_transpose_ctx_v(const void* src, int src_n, int i0, void* dst0, void* dst1, int L, int Bmax,
-                                   int Hkv, int P, int hd, int pst, const CtxList& f, cudaStream_t st) {
-  if (f.n <= 0) return cudaSuccess;
-  dim3 grid((P + 31) / 32, (hd + 31) / 32, L * f.n * Hkv), block(32, 8);
-  transpose_ctx_v_kernel<<<grid, block, 0, st>>>((const bf16*)src, src_n, i0, (bf16*)dst0, (bf16*)dst1, Bmax, Hkv, P,
-                                                 hd, pst, f);
-  return cudaGetLastError();
 }
 
 }  // namespace ravel

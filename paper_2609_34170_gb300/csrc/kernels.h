@@ -169,13 +169,12 @@ struct AttnArgs {
 };
 cudaError_t launch_attention_simt(const AttnArgs& a, Dtype dt, cudaStream_t st);
 
-// tcgen05 attention (bf16).  V operands transposed: the context slots hold
-// Vt [L][Bmax][Hkv][hd][pst]; the step's FOP/slot V is vt [B][Hkv][hd][kvp].
+// tcgen05 attention (bf16).  K and V as the step stores them: the context
+// slots [L][Bmax][Hkv][Pmax][hd], the FOP/slot keys in the QKV rows.
 struct AttnTcArgs {
   const void* qkv; int ld_qkv;
-  const void* vt; int kvp;
-  const void* ctx_k[2]; const void* ctx_vt[2];
-  int layers, layer, Bmax, Pmax, pst;
+  const void* ctx_k[2]; const void* ctx_v[2];
+  int layers, layer, Bmax, Pmax;
   const int* ctx_state;
   int B, H, F, Hq, Hkv, hd, mask_mode;
   void* out; int ld_out;
@@ -186,12 +185,6 @@ struct AttnTcArgs {
 cudaError_t init_attention_tc();
 bool attention_tc_supported(int hd, int G);
 cudaError_t launch_attention_tc(const AttnTcArgs& a, cudaStream_t st);
-// bf16 context V [L][src_n][Hkv][P][hd] (list entry i at source position
-// i0 + i) -> the listed robots' slots Vt_{f.slot[i]} [L][Bmax][Hkv][hd][pst]
-// (keys contiguous)
-struct CtxList;
-cudaError_t launch_transpose_ctx_v(const void* src, int src_n, int i0, void* dst0, void* dst1, int L, int Bmax,
-                                   int Hkv, int P, int hd, int pst, const CtxList& f, cudaStream_t st);
 
 // ---- gated cross-attention of a FOP adapter ------------------------------------------
 // out[b*H + j][h*hd + c] = tanh(gate[0]) * sum_f softmax_f(q . k_f / sqrt(hd)) v_f[c] over the

@@ -215,16 +215,9 @@ static ravel_status set_context_impl(ravel_t* r, const int* robots, int n, const
     RV_CUDA(r, launch_ctx_scatter(k, n, i0, p.ctx_k[0], p.ctx_k[1], c.layers, c.max_batch, c.n_kv_heads, prefix_len,
                                   c.max_prefix, (size_t)c.head_dim * es, f, side),
             (w + ": copy K").c_str());
-    if (p.use_tc_attn) {
-      // the tensor-core attention reads V transposed (keys contiguous)
-      RV_CUDA(r, launch_transpose_ctx_v(v, n, i0, p.ctx_v[0], p.ctx_v[1], c.layers, c.max_batch, c.n_kv_heads,
-                                        prefix_len, c.head_dim, p.pst, f, side),
-              (w + ": transpose V").c_str());
-    } else {
-      RV_CUDA(r, launch_ctx_scatter(v, n, i0, p.ctx_v[0], p.ctx_v[1], c.layers, c.max_batch, c.n_kv_heads, prefix_len,
-                                    c.max_prefix, (size_t)c.head_dim * es, f, side),
-              (w + ": copy V").c_str());
-    }
+    RV_CUDA(r, launch_ctx_scatter(v, n, i0, p.ctx_v[0], p.ctx_v[1], c.layers, c.max_batch, c.n_kv_heads, prefix_len,
+                                  c.max_prefix, (size_t)c.head_dim * es, f, side),
+            (w + ": copy V").c_str());
     for (int i = 0; i < f.n; ++i) {
       r->ctx_pend[f.robot[i]] = f.slot[i];
       r->ctx_pend_len[f.robot[i]] = prefix_len;

@@ -120,8 +120,7 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->in_w, (size_t)A * D * 4); AL(p->in_b, D * 4);
   AL(p->fop_gamma, (size_t)L * D * 4);
   AL(p->out_b, A * 4);
-  p->pst = (c.max_prefix + 7) / 8 * 8;
-  const size_t ctx_bytes = (size_t)L * Bm * c.n_kv_heads * p->pst * c.head_dim * es;
+  const size_t ctx_bytes = (size_t)L * Bm * c.n_kv_heads * c.max_prefix * c.head_dim * es;
   for (int s = 0; s < 2; ++s) {
     AL(p->ctx_k[s], ctx_bytes);
     AL(p->ctx_v[s], ctx_bytes);
@@ -145,8 +144,6 @@ ravel_status plan_create(StepPlan* p, const ravel_config& c, const ravel_weights
   AL(p->GU, rows_a * 2 * Fm * 4);
   AL(p->Hm, rows_a * Fm * es);
   AL(p->V, rows_a * A * 4);
-  p->kvp = (H + F + 7) / 8 * 8;
-  AL(p->Vt, (size_t)Bm * c.n_kv_heads * c.head_dim * p->kvp * es);
   p->attn_ws_bytes = (size_t)32 << 20;
   AL(p->attn_ws, p->attn_ws_bytes);
   p->tcws.ws_bytes = (size_t)24 << 20;
@@ -374,19 +371,13 @@ cudaError_t enqueue_step(const StepPlan& p, int B, const StepIO& io, cudaStream_
     if (l > 0 || !fuse_in) RUN(KK_NORM, launch_ada_norm(n1, dt, st));
     const void* wqkv = (const char*)p.w_qkv + (size_t)l * p.nqkv * D * es;
     if (p.use_tc_attn) {
-      // QKV projection also writes V transposed (keys contiguous) for the tensor-core attention
+      // the tensor-core attention reads K and V straight from the QKV rows
       GemmArgs gq{p.Y, D, wqkv, D, BY, p.nqkv, D, EPI_STORE, p.QKV, p.nqkv, dt, nullptr};
-      gq.vt = p.Vt;
-      gq.v_col0 = (c.n_q_heads + c.n_kv_heads) * c.head_dim;
-      gq.vt_hd = c.head_dim;
-      gq.vt_tokens = RPR;
-      gq.vt_kvp = p.kvp;
-      gq.vt_hkv = c.n_kv_heads;
       gq.max_splits = p.split_cap[0];
       gq.xbf16 = 1;
       RUN(KK_GEMM_QKV, run_gemm(p, gq, st));
-      AttnTcArgs at{p.QKV, p.nqkv, p.Vt, p.kvp, {p.ctx_k[0], p.ctx_k[1]}, {p.ctx_v[0], p.ctx_v[1]}, L, l,
-                    c.max_batch, c.max_prefix, p.pst, p.ctx_state, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim,
+      AttnTcArgs at{p.QKV, p.nqkv, {p.ctx_k[0], p.ctx_k[1]}, {p.ctx_v[0], p.ctx_v[1]}, L, l,
+                    c.max_batch, c.max_prefix, p.ctx_state, B, H, FF, c.n_q_heads, c.n_kv_heads, c.head_dim,
                     c.mask_mode, p.O, p.qdim, p.attn_ws, p.attn_ws_bytes, p.err, p.num_sms};
       int launched = 0;
       at.n_launched = &launched;

@@ -33,11 +33,10 @@ struct StepPlan {
   void *w_qkv = nullptr, *w_o = nullptr, *w_gu = nullptr, *w_down = nullptr, *out_w = nullptr;
   float *t_b1 = nullptr, *t_b2 = nullptr, *d_b1 = nullptr, *d_b2 = nullptr, *mod_b = nullptr;
   float *in_w = nullptr, *in_b = nullptr, *fop_gamma = nullptr, *out_b = nullptr;
-  // VLM context double buffer [2] x [L][Bmax][Hkv][Pmax][hd] and its device state {active, len}
-  // (bf16 mode: ctx_v holds V transposed, [L][Bmax][Hkv][hd][pst], for the tensor-core attention)
+  // VLM context double buffer [2] x [L][Bmax][Hkv][Pmax][hd] (K and V alike) and its
+  // device state per robot {active slot, prefix length}
   void* ctx_k[2] = {nullptr, nullptr};
   void* ctx_v[2] = {nullptr, nullptr};
-  int pst = 0;              // key pitch of the transposed context V (max_prefix rounded up to 8)
   int* ctx_state = nullptr;
   // activations
   void* E = nullptr;      // [H+Bmax][D]  sinusoidal embeddings (times, then offsets)
@@ -59,8 +58,6 @@ struct StepPlan {
   float* GU = nullptr;    // [Bmax*H][2Fm]  interleaved gate/up (SIMT path)
   void* Hm = nullptr;     // [Bmax*H][Fm]
   float* V = nullptr;     // [Bmax*H][A]   velocity
-  void* Vt = nullptr;     // [Bmax][Hkv][hd][kvp]  transposed V of the FOP + slot keys (bf16 mode)
-  int kvp = 0;            // key pitch of Vt: (H + F) rounded up to 8
   float* attn_ws = nullptr;  // split-KV partials of the tensor-core attention
   size_t attn_ws_bytes = 0;
   bool use_tc_attn = false;

@@ -107,10 +107,25 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return d;
 }
 
+// The same for an MN-major tile (rows along K, the MN extent contiguous):
+// the 128-byte swizzle atom is 8 K-rows of 64 bf16 along MN; mn_stride is the
+// byte offset of the next 64 MN elements, 8-row groups along K 1024 bytes
+// apart.  A K step of 16 advances the start address by 2048 bytes.
+__device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr, uint32_t mn_stride) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((mn_stride & 0x3FFFFu) >> 4) << 16;   // leading byte offset: next 64 along MN
+  d |= (uint64_t)(1024 >> 4) << 32;                     // stride byte offset: next 8 rows along K
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
 // Instruction descriptor of kind::f16 with bf16 A/B, fp32 D, both K-major.
 __device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
+// ... with B MN-major (its K rows hold the N extent contiguously)
+__device__ __forceinline__ uint32_t idesc_bf16_bmn(int m, int n) { return idesc_bf16(m, n) | (1u << 16); }
 
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
   asm volatile(
