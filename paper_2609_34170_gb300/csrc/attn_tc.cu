@@ -196,8 +196,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   uint8_t* kv_s = q_s + (size_t)p.nblk * AT_QBLK;   // K ring, then V ring
   uint8_t* v_ring = kv_s + (size_t)SK * k_bytes;
   uint64_t* bars = (uint64_t*)(v_ring + (size_t)SV * k_bytes);
-  // K and V^T of a stage have their own barriers: K is released as soon as
-  // S = Q K^T has been computed, V^T only after P V, so the next K load does
+  // K and V of a stage have their own barriers: K is released as soon as
+  // S = Q K^T has been computed, V only after P V, so the next K load does
   // not wait for the softmax and the PV of the chunk it replaces
   uint64_t* q_full = bars;
   uint64_t* k_full = bars + 1;
@@ -267,7 +267,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
   if (p.xch == 2) cluster_sync();
   const CUtensorMap* pk = slot ? &maps.pk1 : &maps.pk0;
   const CUtensorMap* pv = slot ? &maps.pv1 : &maps.pv0;
-  // K and V^T of chunk c into stage s, each CTA loading its own copy (query
+  // K and V of chunk c into stage s, each CTA loading its own copy (query
   // tiles of one (b, g) pair read the same chunk, which L2 serves to all)
   auto load_k = [&](int c, int s, uint64_t pol) {
     uint8_t* ks = kv_s + (size_t)s * k_bytes;
@@ -335,7 +335,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       for (int blk = 0; blk < p.nblk; ++blk)
         tma_load_3d(&maps.q, q_full, q_s + (size_t)blk * AT_QBLK, blk * 64, g * p.G, b * rows_per_robot + qt * p.TQ,
                     pol_q);
-      // K of chunk nk and V^T of chunk nv (nv <= nk), each as soon as its slot
+      // K of chunk nk and V of chunk nv (nv <= nk), each as soon as its slot
       // is free; K may run ahead of V
       int nk = npre, nv = npre;
       unsigned long long t_last = globaltimer();
@@ -439,7 +439,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_tc_kernel(const __grid_con
       if (p.xch == 2 && !sdone_sent) umma_commit_mc(sdone, smask);
       if (!ok) flags[0] = 1;
       flags[2] = ns;   // chunks whose K arrival was consumed
-      flags[4] = i;    // chunks whose V^T arrival was consumed
+      flags[4] = i;    // chunks whose V arrival was consumed
     }
     __syncwarp();
     if (p.xch == 1) cluster_arrive_release();

@@ -63,10 +63,10 @@ constexpr uint32_t STG_BYTES = 16 * STG_LD * 4;
 constexpr uint32_t XCH_BYTES = 32 * STG_LD * 4;  // GeGLU transpose tile (TMA epilogue): <= 32 tokens x 128 rows
 
 enum { RED_NONE = 0, RED_L2_CLUSTER = 1, RED_WORKSPACE = 2, RED_DSMEM = 3, RED_DSMEM32 = 4 };
-// Epilogue kind of an instantiation: outputs through TMA boxes as fp32, bf16
-// (+ the V^T side output), a reduce-add into the fp32 residual stream or the
-// GeGLU pair -- fixed, so that a long persistent launch carries only the code
-// of its own epilogue -- or any of these chosen at run time (EK_TMA_ANY: the
+// Epilogue kind of an instantiation: outputs through TMA boxes as fp32, bf16,
+// a reduce-add into the fp32 residual stream or the GeGLU pair -- fixed, so
+// that a long persistent launch carries only the code of its own epilogue --
+// or any of these chosen at run time (EK_TMA_ANY: the
 // short split-K launches of one step then all run one binary, whose code the
 // previous launch has left in the SM's instruction cache), or stored by the
 // threads (EK_GENERIC: any epilogue; unaligned outputs and the workspace
@@ -89,8 +89,6 @@ struct TcParams {
   float* ws;
   int* counters;
   int* err;
-  bf16* vt;
-  int v_col0, vt_hd, vt_tokens, vt_kvp, vt_hkv;
   int tma_out;          // outputs leave through TMA boxes
   int oneshot;          // split launch whose whole K range fits the ring: tmW / tmX are 3-D maps
                         // (64, rows, K / 64) and one box each brings all of its k-tiles
@@ -98,7 +96,6 @@ struct TcParams {
   uint32_t box_bytes;   // bytes of one TMA output box (1024-aligned)
   uint32_t stg_off;     // SIMT transpose tile, or two TMA output boxes
   uint32_t xch_off;     // GeGLU exchange
-  uint32_t vts_off;     // V^T side output (TMA epilogue): the chunk as [128 tile rows][box_m + 10] bf16
   uint32_t rcv_off;     // RED_DSMEM*: the partials received from the splits, [split][cpr / 4][128 rows]
                         // float4, overlaid on the operand ring (free once every CTA of the cluster
                         // has finished its MMAs), else on the output boxes + exchange (used only
@@ -109,7 +106,7 @@ struct TcParams {
                         // nobody makes, so the launch gives up after wait_ns and unwinds
   const int* skip;      // optional device flag read after the dependency wait: nonzero -> the launch
                         // completes the copies it started and exits without computing
-  uint32_t set_bytes;   // pair kernel: bytes from epilogue set 0's boxes / exchange / V^T tile to set 1's
+  uint32_t set_bytes;   // pair kernel: bytes from epilogue set 0's boxes / exchange to set 1's
 };
 
 // The TMA epilogue kind of a launch (EK_F32 .. EK_GEGLU).
@@ -168,46 +165,6 @@ __device__ __forceinline__ void reduce_splits_l2(const float* b0, int S, size_t 
         v[4 * g + 2] += x[u][g].z;
         v[4 * g + 3] += x[u][g].w;
       }
-  }
-}
-
-// V^T side output of the QKV projection for tokens m0 .. m0+nv-1 of this
-// thread's tile row: token m -> (robot m / T, key m % T).  Eight keys that
-// start on a multiple of 8 within one robot go out as one 16-byte store (rows
-// of V^T are a multiple of 8 keys apart), the rest one by one.
-template <int NV = 16>
-__device__ __forceinline__ void store_vt(const TcParams& p, int tile_n, int m0, int nv, int r, const float v[NV]) {
-  const int n = tile_n * TC_BM + r;
-  if (n < p.v_col0 || n >= p.N) return;
-  const float bb = p.bias ? p.bias[n] : 0.f;
-  const int g = (n - p.v_col0) / p.vt_hd, d = (n - p.v_col0) % p.vt_hd;
-  const int T = p.vt_tokens;
-  int rb = m0 / T, kk = m0 % T;
-  bf16* dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
-#pragma unroll
-  for (int i0 = 0; i0 < NV; i0 += 8) {
-    if (i0 >= nv) break;
-    if ((kk & 7) == 0 && kk + 8 <= T && i0 + 8 <= nv) {
-      *(uint4*)(dst + kk) = make_uint4(pack_bf16x2(v[i0] + bb, v[i0 + 1] + bb), pack_bf16x2(v[i0 + 2] + bb, v[i0 + 3] + bb),
-                                       pack_bf16x2(v[i0 + 4] + bb, v[i0 + 5] + bb), pack_bf16x2(v[i0 + 6] + bb, v[i0 + 7] + bb));
-      kk += 8;
-      if (kk == T) {
-        kk = 0;
-        ++rb;
-        dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
-      }
-    } else {
-#pragma unroll
-      for (int i = i0; i < i0 + 8; ++i) {
-        if (i >= nv) break;
-        dst[kk] = __float2bfloat16_rn(v[i] + bb);
-        if (++kk == T) {
-          kk = 0;
-          ++rb;
-          dst = p.vt + ((size_t)(rb * p.vt_hkv + g) * p.vt_hd + d) * p.vt_kvp;
-        }
-      }
-    }
   }
 }
 
@@ -281,12 +238,11 @@ __device__ __forceinline__ void reduce_slice_smem(const float4* b0, int S, float
 // is this thread's tile row r at token m0+i.  All 128 epilogue threads call it
 // together.  The chunk is transposed through `stage` so that each thread then
 // writes one token's 16 (or, for GeGLU, 8) consecutive outputs as 16-byte
-// stores.  The V columns of the QKV projection also go out transposed.
+// stores.
 __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, int m0, int nc, int r,
                                                const float v[16], float* stage) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) stage[i * STG_LD + r] = v[i];
-  if (p.vt) store_vt(p, tile_n, m0, min(nc, p.M - m0), r, v);
   epi_bar();
   const int c = r >> 3, fg = r & 7;
   const int m = m0 + c;
@@ -360,10 +316,6 @@ __device__ __forceinline__ void epilogue_chunk(const TcParams& p, int tile_n, in
   epi_bar();
 }
 
-// The V^T staging tile of the TMA epilogue.
-__device__ __forceinline__ bf16* vt_stage(const TcParams& p, uint8_t* boxes) {
-  return (bf16*)(boxes - p.stg_off + p.vts_off);
-}
 
 // TMA epilogue of tokens m0 .. m0+box_m-1 of tile row block tile_n: v[i] is
 // this thread's tile row r at token m0+i, brow its bias.  All 128 epilogue
@@ -398,21 +350,11 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   // the thread of the set that issues and waits for its TMA stores
   const int set = threadIdx.x >= 192 ? 1 : 0;
   const bool issuer = threadIdx.x == 64 + 128 * set;
-  // the box written two chunks ago must have been read by its TMA store (and
-  // every thread is done with the V^T tile of the previous chunk)
+  // the box written two chunks ago must have been read by its TMA store
   if (issuer) bulk_wait_read<1>();
   epi_bar_set(set);
   uint8_t* box = boxes + (size_t)ebuf * p.box_bytes;
-  const int vpitch = bm + 10;   // bf16 per V^T tile row: an odd number of words, no bank conflicts
-  // V^T side output through a transposed staging tile (below); one path for
-  // every chunk: a second, register-to-global path made the kernel's code, and
-  // every launch of it, slower
   const int kind = EK == EK_TMA_ANY ? tma_kind(p) : EK;   // a constant in the fixed-kind instantiations
-  const bool vtile = kind == EK_BF16 && p.vt && (tile_n + 1) * TC_BM > p.v_col0;
-  if (vtile) {   // this thread's row of the chunk, feature-major, for the V^T side output below
-    uint32_t* vrow = (uint32_t*)(vt_stage(p, boxes) + (size_t)r * vpitch);
-    for_upto<NV / 2, 2>((bm + 1) / 2, [&](int h) { vrow[h] = pack_bf16x2(v[2 * h] + brow, v[2 * h + 1] + brow); });
-  }
   if (kind == EK_GEGLU) {
     // tile rows 0..63 are gate features, 64..127 the matching up features:
     // transpose through xch so that every thread then forms 8 outputs of one
@@ -452,23 +394,6 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
     if (kind == EK_ADD) tma_reduce_add_2d(tmO, box, tile_n * TC_BM, m0);
     else tma_store_2d(tmO, box, kind == EK_GEGLU ? tile_n * 64 : tile_n * TC_BM, m0);
     bulk_commit();
-  }
-  if (vtile) {
-    // V columns of the QKV projection also go out transposed, V^T[robot][g][d][key]:
-    // warp w writes tile rows 32w..32w+31 one after the other, lane i the
-    // chunk's token i, so that each store covers one contiguous run of keys
-    const bf16* vs = vt_stage(p, boxes);
-    const int w = (threadIdx.x >> 5) & 3, lane = threadIdx.x & 31;
-    const int m = m0 + lane;
-    if (lane < bm && m < p.M) {
-      const int rb = m / p.vt_tokens, kk = m - rb * p.vt_tokens;
-      bf16* vb = p.vt + (size_t)rb * p.vt_hkv * p.vt_hd * p.vt_kvp + kk;   // row (g, d) is (g*hd + d)*kvp further
-      for (int fi = 0; fi < 32; ++fi) {
-        const int f = 32 * w + fi, n = tile_n * TC_BM + f;
-        if (n < p.v_col0 || n >= p.N) continue;
-        vb[(size_t)(n - p.v_col0) * p.vt_kvp] = vs[(size_t)f * vpitch + lane];
-      }
-    }
   }
   ebuf ^= 1;
 }
@@ -1360,9 +1285,8 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
       (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
   const size_t stg_bytes = 2 * (size_t)box_bytes;
   const size_t xch_bytes = g.epi == EPI_GEGLU ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
-  const size_t vts_bytes = g.vt ? ((size_t)TC_BM * (box_m + 10) * 2 + 1023) / 1024 * 1024 : 0;
-  // each of the two epilogue warp sets has its own boxes, exchange tile and V^T tile
-  const size_t set_bytes = stg_bytes + xch_bytes + vts_bytes;
+  // each of the two epilogue warp sets has its own boxes and exchange tile
+  const size_t set_bytes = stg_bytes + xch_bytes;
   const size_t fixed = 1024 + 2 * set_bytes + 256;
   const int stage_bytes = TC_A_BYTES + (bn / 2) * TC_BK * 2;
   const int stages = std::min(8, (int)((TC_SMEM_MAX - fixed) / stage_bytes));
@@ -1370,7 +1294,6 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
   const size_t ring = ((size_t)stages * stage_bytes + 1023) / 1024 * 1024;
   const uint32_t stg_off = (uint32_t)ring;
   const uint32_t xch_off = stg_off + (uint32_t)stg_bytes;
-  const uint32_t vts_off = xch_off + (uint32_t)xch_bytes;
   const uint32_t bar_off = stg_off + 2 * (uint32_t)set_bytes;
   const size_t smem = 1024 + bar_off + (size_t)(2 * stages + 4) * 8 + 4 + 16 + 64;
   if (smem > (size_t)TC_SMEM_MAX) return cudaErrorInvalidConfiguration;
@@ -1382,9 +1305,8 @@ cudaError_t launch_gemm_pair(const GemmArgs& g, const TcWorkspace& ws, int num_s
                    g.epi == EPI_GEGLU ? 64 : TC_BM, box_m);
   if (e != cudaSuccess) return e;
   TcParams p{g.M, g.N, g.K, bn, stages, 1, num_kb, RED_NONE, (uint32_t)ring, acc_cols, tiles_n, tiles_m, num_tiles,
-             (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
-             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, 1, 0, box_m, box_bytes, stg_off, xch_off,
-             vts_off, 0, bar_off, kTcTimeoutNs, 0, g.skip};
+             (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err,
+             1, 0, box_m, box_bytes, stg_off, xch_off, 0, bar_off, kTcTimeoutNs, 0, g.skip};
   p.set_bytes = (uint32_t)set_bytes;
   const int npairs = std::min(num_tiles, slots);
   return launch_kernel_cluster(tc_pair_kernel(ek), dim3(2 * npairs), dim3(TC_PAIR_THREADS), smem, st, dim3(2, 1, 1),
@@ -1500,7 +1422,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
   int box_m = 0;
   // partials exchanged in bf16 where the caller allows it, else in fp32
   const bool xbf = g.xbf16 != 0;
-  uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, vts_off = 0, rcv_off = 0, bar_off = 0;
+  uint32_t box_bytes = 0, stg_off = (uint32_t)ring, xch_off = 0, rcv_off = 0, bar_off = 0;
   size_t smem = 0;
   auto layout = [&](bool dsmem) {
     box_m = splits == 1 ? 16
@@ -1509,15 +1431,13 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
     box_bytes = (uint32_t)(((size_t)box_m * (g.epi == EPI_GEGLU ? 64 : TC_BM) * es + 1023) / 1024 * 1024);
     const size_t stg_bytes = tma_out ? 2 * (size_t)box_bytes : (STG_BYTES + 1023) / 1024 * 1024;
     const size_t xch_bytes = (tma_out && g.epi == EPI_GEGLU) ? (XCH_BYTES + 1023) / 1024 * 1024 : 0;
-    const size_t vts_bytes = (tma_out && g.vt) ? ((size_t)TC_BM * (box_m + 10) * 2 + 1023) / 1024 * 1024 : 0;
     // received partials (all splits' slices of this rank) overlay the operand
     // ring, else the boxes + exchange
     const size_t rcv_bytes = dsmem ? (size_t)TC_BM * bn * (xbf ? 2 : 4) : 0;
     const bool in_ring = rcv_bytes <= ring;
     xch_off = stg_off + (uint32_t)stg_bytes;
-    vts_off = xch_off + (uint32_t)xch_bytes;
     rcv_off = in_ring ? 0u : stg_off;
-    bar_off = stg_off + (uint32_t)std::max(stg_bytes + xch_bytes + vts_bytes, in_ring ? (size_t)0 : rcv_bytes);
+    bar_off = stg_off + (uint32_t)std::max(stg_bytes + xch_bytes, in_ring ? (size_t)0 : rcv_bytes);
     smem = 1024 + bar_off + (size_t)(2 * stages + 5) * 8 + 4 + 16 + 64;
   };
   // partials by st.async into the owning rank's shared memory when the token
@@ -1540,9 +1460,9 @@ cudaError_t launch_gemm_tc(const GemmArgs& g, const TcWorkspace& ws, int num_sms
                    g.epi == EPI_GEGLU ? 64 : TC_BM, box_m);
   if (e != cudaSuccess) return e;
   TcParams p{g.M, g.N, g.K, bn, stages, splits, num_kb, reduce, (uint32_t)ring, acc_cols, tiles_n, tiles_m, tiles,
-             (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err, (bf16*)g.vt,
-             g.v_col0, g.vt_hd, g.vt_tokens, g.vt_kvp, g.vt_hkv, tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off,
-             vts_off, rcv_off, bar_off, kTcTimeoutNs, 0, g.skip};
+             (int)g.epi, g.out_dt == DT_BF16 ? 1 : 0, g.out, g.ldo, g.bias, ws.ws, ws.counters, ws.err,
+             tma_out ? 1 : 0, oneshot ? 1 : 0, box_m, box_bytes, stg_off, xch_off, rcv_off, bar_off, kTcTimeoutNs, 0,
+             g.skip};
   // fault injection (tests): a launch without a cluster may be told to wait
   // for an arrival that never comes, with a short limit
   if ((reduce == RED_NONE || reduce == RED_WORKSPACE) && g_withhold.load() > 0 && g_withhold.fetch_sub(1) > 0) {

@@ -83,11 +83,6 @@ struct GemmArgs {
   void* out; int ldo;           // EPI_STORE*: dtype `out_dt`; EPI_ADD_F32: float, += result
   Dtype out_dt;
   const float* bias;            // [N] or null
-  // optional second destination of the V columns (n >= v_col0), transposed:
-  // vt[((m / vt_tokens) * vt_hkv + g) * vt_hd + d][m % vt_tokens] with
-  // g = (n - v_col0) / vt_hd, d = (n - v_col0) % vt_hd, row pitch vt_kvp
-  void* vt = nullptr;
-  int v_col0 = 0, vt_hd = 0, vt_tokens = 0, vt_kvp = 0, vt_hkv = 0;
   int max_splits = 0;           // tcgen05 path: cap on the split-K factor (0: chosen from the shape)
   const int* skip = nullptr;    // optional device flag: nonzero at run time -> the launch computes nothing
   // tcgen05 split-K inside a cluster: the splits' partials may travel between
