@@ -67,7 +67,8 @@ def test_ragged_shapes(dtype):
 
 # Key chunks split over a thread-block cluster (2, 4, 16 splits; one and two
 # query tiles; two robots), with a partial last prefix chunk, and a prefix
-# shorter than the slot capacity so that some splits get no key at all.
+# shorter than the slot capacity so that some splits get no key at all; and
+# head dims that are not a multiple of 64.
 SPLIT_KV = [
     (dict(layers=2, width=256, n_q_heads=4, n_kv_heads=1, head_dim=64, mlp_dim=512, slots=20, action_dim=7,
           prefix=300, fop_tokens=5, batch=1), None),
@@ -77,6 +78,13 @@ SPLIT_KV = [
           prefix=2000, fop_tokens=3, batch=1), 1500),
     (dict(layers=1, width=256, n_q_heads=8, n_kv_heads=2, head_dim=64, mlp_dim=256, slots=40, action_dim=6,
           prefix=500, fop_tokens=8, batch=2), None),
+    # head dims that end inside a 64-wide block: P V reads V as an MN-major
+    # operand whose second block is partial (96 = 64 + 32 split, 80 = 64 + 16
+    # over 64 robots, whose query tiles are not split)
+    (dict(layers=1, width=192, n_q_heads=4, n_kv_heads=2, head_dim=96, mlp_dim=256, slots=10, action_dim=5,
+          prefix=260, fop_tokens=3, batch=1), None),
+    (dict(layers=1, width=160, n_q_heads=2, n_kv_heads=1, head_dim=80, mlp_dim=256, slots=9, action_dim=4,
+          prefix=130, fop_tokens=2, batch=64), None),
 ]
 
 
